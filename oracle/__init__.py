@@ -1,0 +1,243 @@
+"""Plain CPU oracle for the REFLEX per-forward MoE path (test infrastructure).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` may import this package.  The
+product path (``paper_2608_01784_gb300``) never imports it and shares no code
+with it.
+
+The arithmetic lives in ``reflex_oracle.c`` (plain C, ``-ffp-contract=off``);
+this module compiles it with gcc and marshals numpy arrays into it.  The C
+file's header lists which paper passage each function follows:
+
+* ``allocate``        Refinement-Role Budgeting (Eq. 5) + Frontier-Guided
+                      Expert Reallocation (forecast, Eq. 6-8, Eq. 9) + clip.
+* ``router_logits``   router scores of Sec. 3.2 (sequential fp32 fma chain).
+* ``select``          TopK of Eq. 2 and the normalised router weight.
+* ``permutation``     (expert, token)-ordered pair list that executes Eq. 2.
+* ``moe_tokens``      Eq. 2 with SwiGLU experts (+ shared expert), fp64.
+
+Parity unpinned: none of the functions above (see tests/test_oracle_pins.py);
+the paper-level AvgK / pair-reduction numbers of Table 1 need the paper's
+models and data and are not reproduced.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import shutil
+import subprocess
+from pathlib import Path
+
+import numpy as np
+
+_HERE = Path(__file__).resolve().parent
+_SRC = _HERE / "reflex_oracle.c"
+_BUILD = _HERE / "_build"
+_LIB_PATH = _BUILD / "liboracle.so"
+_lib = None
+
+
+def build(force: bool = False) -> Path:
+    """Compile reflex_oracle.c into oracle/_build/liboracle.so (gcc, -O2,
+    -ffp-contract=off, OpenMP when available)."""
+    _BUILD.mkdir(exist_ok=True)
+    if (not force and _LIB_PATH.exists()
+            and _LIB_PATH.stat().st_mtime >= _SRC.stat().st_mtime):
+        return _LIB_PATH
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        raise RuntimeError("oracle build needs gcc")
+    tmp = _BUILD / f"liboracle.{os.getpid()}.so"
+    base = [cc, "-O2", "-ffp-contract=off", "-fno-fast-math", "-std=c11",
+            "-fPIC", "-shared", str(_SRC), "-o", str(tmp), "-lm"]
+    try:
+        subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True,
+                       capture_output=True)
+    except subprocess.CalledProcessError:
+        subprocess.run(base, check=True, capture_output=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    if _lib is not None:
+        return _lib
+    lib = ctypes.CDLL(str(build()))
+    p = ctypes.c_void_p
+    i32 = ctypes.c_int32
+    f32 = ctypes.c_float
+    lib.oracle_exp_f32.restype = f32
+    lib.oracle_exp_f32.argtypes = [f32]
+    lib.oracle_exp_f32_n.restype = None
+    lib.oracle_exp_f32_n.argtypes = [p, p, ctypes.c_int64]
+    lib.oracle_fps.restype = f32
+    lib.oracle_fps.argtypes = [f32, f32, i32, f32, f32, f32, f32]
+    lib.oracle_fps_n.restype = None
+    lib.oracle_fps_n.argtypes = [p, p, p, ctypes.c_int64, f32, f32, f32, f32, p]
+    lib.oracle_allocate.restype = ctypes.c_int
+    lib.oracle_allocate.argtypes = [p, p, p, p, p, p, p, i32, i32,
+                                    i32, i32, i32, i32, i32,
+                                    f32, f32, f32, f32, f32, p, p]
+    lib.oracle_router_logits.restype = None
+    lib.oracle_router_logits.argtypes = [i32, p, p, i32, i32, i32, p]
+    lib.oracle_select.restype = ctypes.c_int
+    lib.oracle_select.argtypes = [p, p, i32, i32, i32, i32, p, p]
+    lib.oracle_permutation.restype = ctypes.c_int64
+    lib.oracle_permutation.argtypes = [p, p, i32, i32, i32, p, p, p]
+    lib.oracle_moe_tokens.restype = None
+    lib.oracle_moe_tokens.argtypes = [i32, p, p, p, p, p, i32, p, p, p, p,
+                                      i32, i32, i32, i32, p]
+    lib.oracle_num_threads.restype = ctypes.c_int
+    lib.oracle_num_threads.argtypes = []
+    _lib = lib
+    return lib
+
+
+def _ptr(a: np.ndarray | None):
+    if a is None:
+        return None
+    assert a.flags["C_CONTIGUOUS"], "oracle arrays must be C-contiguous"
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def num_threads() -> int:
+    return int(_load().oracle_num_threads())
+
+
+def exp_f32(x) -> np.ndarray:
+    x = _c(x, np.float32).ravel()
+    y = np.empty_like(x)
+    _load().oracle_exp_f32_n(_ptr(x), _ptr(y), x.size)
+    return y
+
+
+def fps(c1, c2, hist, theta, w_cf, v_ref, tau) -> np.ndarray:
+    c1 = _c(c1, np.float32).ravel()
+    c2 = _c(c2, np.float32).ravel()
+    hist = _c(hist, np.uint8).ravel()
+    s = np.empty_like(c1)
+    _load().oracle_fps_n(_ptr(c1), _ptr(c2), _ptr(hist), c1.size, theta, w_cf,
+                         v_ref, tau, _ptr(s))
+    return s
+
+
+def allocate(conf1, conf2, hist_len, masked, block_id, seq_offsets,
+             active_block, *, k_min, k_base, k_max, delta_role, delta_cur,
+             q, theta, w_cf, v_ref, tau, return_scores: bool = False):
+    """Per-token expert counts of REFLEX (Eq. 5, Eq. 9, clip); int32 [T]."""
+    conf1 = _c(conf1, np.float32)
+    conf2 = _c(conf2, np.float32)
+    hist_len = _c(hist_len, np.uint8)
+    masked = _c(masked, np.uint8)
+    block_id = _c(block_id, np.int32)
+    seq_offsets = _c(seq_offsets, np.int32)
+    active_block = _c(active_block, np.int32)
+    T = block_id.size
+    B = active_block.size
+    k = np.empty(T, np.int32)
+    s = np.empty(T, np.float32)
+    rc = _load().oracle_allocate(
+        _ptr(conf1), _ptr(conf2), _ptr(hist_len), _ptr(masked),
+        _ptr(block_id), _ptr(seq_offsets), _ptr(active_block), T, B,
+        k_min, k_base, k_max, delta_role, delta_cur, q, theta, w_cf, v_ref,
+        tau, _ptr(k), _ptr(s))
+    if rc != 0:
+        raise ValueError("oracle_allocate: invalid input")
+    return (k, s) if return_scores else k
+
+
+def _dtype_code(a: np.ndarray) -> int:
+    if a.dtype == np.float32:
+        return 0
+    if a.dtype == np.uint16:  # bf16 bit patterns
+        return 1
+    raise TypeError("oracle inputs are float32 or bf16 bits (uint16)")
+
+
+def router_logits(hidden: np.ndarray, w_router: np.ndarray) -> np.ndarray:
+    """z[T, E] fp32 by the sequential fma chain over the hidden index."""
+    hidden = np.ascontiguousarray(hidden)
+    w_router = np.ascontiguousarray(w_router)
+    dt = _dtype_code(hidden)
+    assert _dtype_code(w_router) == dt
+    T, d = hidden.shape
+    E = w_router.shape[0]
+    z = np.empty((T, E), np.float32)
+    _load().oracle_router_logits(dt, _ptr(hidden), _ptr(w_router), T, d, E,
+                                 _ptr(z))
+    return z
+
+
+def select(z: np.ndarray, k: np.ndarray, k_max: int, renorm: bool = True):
+    """(ids int32 [T, k_max], alpha fp64 [T, k_max])."""
+    z = _c(z, np.float32)
+    k = _c(k, np.int32)
+    T, E = z.shape
+    ids = np.empty((T, k_max), np.int32)
+    alpha = np.empty((T, k_max), np.float64)
+    rc = _load().oracle_select(_ptr(z), _ptr(k), T, E, k_max, int(renorm),
+                               _ptr(ids), _ptr(alpha))
+    if rc != 0:
+        raise ValueError("oracle_select: some k_t outside [1, min(k_max, E)]")
+    return ids, alpha
+
+
+def permutation(ids: np.ndarray, k: np.ndarray, E: int):
+    """(offsets int32 [E+1], perm int32 [sum k], row_of int32 [T, k_max])."""
+    ids = _c(ids, np.int32)
+    k = _c(k, np.int32)
+    T, k_max = ids.shape
+    offsets = np.empty(E + 1, np.int32)
+    perm = np.empty(max(int(k.sum()), 1), np.int32)
+    row_of = np.empty((T, k_max), np.int32)
+    n = _load().oracle_permutation(_ptr(ids), _ptr(k), T, E, k_max,
+                                   _ptr(offsets), _ptr(perm), _ptr(row_of))
+    return offsets, perm[:n].copy(), row_of
+
+
+def moe_tokens(hidden, w_gate_up, w_down, ids, alpha, k, tokens, *,
+               shared_gate_up=None, shared_down=None) -> np.ndarray:
+    """Eq. 2 (+ shared expert) for the listed tokens; fp64 [len(tokens), d]."""
+    hidden = np.ascontiguousarray(hidden)
+    w_gate_up = np.ascontiguousarray(w_gate_up)
+    w_down = np.ascontiguousarray(w_down)
+    dt = _dtype_code(hidden)
+    T, d = hidden.shape
+    inter = w_down.shape[-1]
+    ids = _c(ids, np.int32)
+    alpha = _c(alpha, np.float64)
+    k = _c(k, np.int32)
+    tokens = _c(tokens, np.int32)
+    k_max = ids.shape[1]
+    s_inter = 0
+    if shared_gate_up is not None:
+        shared_gate_up = np.ascontiguousarray(shared_gate_up)
+        shared_down = np.ascontiguousarray(shared_down)
+        s_inter = shared_down.shape[-1]
+    out = np.empty((tokens.size, d), np.float64)
+    _load().oracle_moe_tokens(dt, _ptr(hidden), _ptr(w_gate_up), _ptr(w_down),
+                              _ptr(shared_gate_up), _ptr(shared_down), s_inter,
+                              _ptr(ids), _ptr(alpha), _ptr(k), _ptr(tokens),
+                              tokens.size, d, inter, k_max, _ptr(out))
+    return out
+
+
+def moe_layer(hidden, w_router, w_gate_up, w_down, k, k_max, *, tokens=None,
+              renorm=True, shared_gate_up=None, shared_down=None) -> dict:
+    """Whole layer in the paper's order: scores -> TopK/alpha -> pairs ->
+    Eq. 2 for ``tokens`` (all tokens when None)."""
+    E = w_router.shape[0]
+    z = router_logits(hidden, w_router)
+    ids, alpha = select(z, k, k_max, renorm)
+    offsets, perm, row_of = permutation(ids, k, E)
+    if tokens is None:
+        tokens = np.arange(hidden.shape[0], dtype=np.int32)
+    out = moe_tokens(hidden, w_gate_up, w_down, ids, alpha, k, tokens,
+                     shared_gate_up=shared_gate_up, shared_down=shared_down)
+    return dict(z=z, ids=ids, alpha=alpha, offsets=offsets, perm=perm,
+                row_of=row_of, tokens=np.asarray(tokens, np.int32), out=out)

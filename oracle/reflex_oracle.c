@@ -1,0 +1,411 @@
+/*
+ * reflex_oracle.c — plain, slow CPU oracle for the REFLEX per-forward MoE path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the
+ * cpu_baseline / reference legs of bench.py may load this library.  The
+ * product path (include/reflex.h, paper_2608_01784_gb300/) never calls it and
+ * shares no code, header, table or constant with it.
+ *
+ * What it computes (paper section / equation it follows):
+ *   oracle_exp_f32       own fp32 exp: Cody-Waite argument reduction (Cody &
+ *                        Waite 1980) + degree-7 Taylor polynomial, separate
+ *                        IEEE operations only.  Used by the FPS sigmoids.
+ *   oracle_allocate      Refinement-Role Budgeting (Sec. 4.2, Eq. 5) then
+ *                        Frontier-Guided Expert Reallocation (Sec. 4.3,
+ *                        forecast, Eq. 6-8 and Eq. 9), then the clip of every
+ *                        count to [K_min, K_max] required by Eq. 3.
+ *   oracle_router_logits router scores r = h . W_r (Sec. 3.2) as a sequential
+ *                        fp32 fused-multiply-add chain over the hidden index,
+ *                        k = 0 .. d-1, starting from +0 (the summation-order
+ *                        contract the GPU router also follows).
+ *   oracle_select        TopK_e(r, k_i) of Eq. 2 (ties: lower expert index)
+ *                        and the normalised router weight alpha in fp64.
+ *   oracle_permutation   token-expert pairs sorted by (expert, token): the
+ *                        per-expert row ranges that execute Eq. 2 sparsely.
+ *   oracle_moe_tokens    Eq. 2 for a list of tokens: sum over selected experts
+ *                        of alpha * SwiGLU expert, plus an optional always-on
+ *                        shared expert (alpha = 1), in fp64.
+ *
+ * Floating-point contract: build with -O2 -ffp-contract=off so that every
+ * a*b+c written below is two rounded operations unless fmaf() is called.
+ *
+ * Parity pins live in tests/test_oracle_pins.py; every function above has at
+ * least one pin that does not re-run the function's own formula.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define OR_OK 0
+#define OR_EINVAL 1
+
+/* ------------------------------------------------------------------------ */
+/* bf16 helpers: a bf16 value is the top 16 bits of an IEEE binary32.        */
+/* ------------------------------------------------------------------------ */
+static float or_bf16_to_f32(uint16_t b) {
+    uint32_t u = ((uint32_t)b) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return f;
+}
+
+static float or_load(const void* base, int32_t dtype, int64_t idx) {
+    /* dtype 0 = fp32 element, 1 = bf16 element (widened exactly) */
+    if (dtype == 0) return ((const float*)base)[idx];
+    return or_bf16_to_f32(((const uint16_t*)base)[idx]);
+}
+
+/* ------------------------------------------------------------------------ */
+/* exp in fp32 from a published method.                                      */
+/*   x = k*ln2 + r,  k = round-half-even(x / ln2),  |r| <= ln2/2             */
+/*   r computed with ln2 split in a high part of few bits (k*hi exact) and   */
+/*   a low part (Cody & Waite 1980).                                         */
+/*   e^r by its Taylor series to degree 7 in Horner form (truncation error   */
+/*   below 2^-27 relative on |r| <= ln2/2).                                  */
+/*   Result scaled by 2^k as two exact power-of-two factors so that neither  */
+/*   factor overflows and a subnormal result is rounded once.                */
+/* ------------------------------------------------------------------------ */
+static float or_pow2i(int32_t e) {
+    /* 2^e for e in [-126, 127], built from its bit pattern */
+    uint32_t u = ((uint32_t)(e + 127)) << 23;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return f;
+}
+
+float oracle_exp_f32(float x) {
+    const float inv_ln2 = 1.44269502162933349609375f;      /* fp32(1/ln 2) */
+    const float ln2_hi = 0.693145751953125f;               /* 0x3F317200   */
+    const float ln2_lo = 1.428606765330187045037746429443359375e-06f;
+    if (x != x) return x;
+    if (x >= 89.0f) return INFINITY;
+    if (x <= -104.0f) return 0.0f;
+    float t = x * inv_ln2;
+    float kf = rintf(t); /* default rounding mode: nearest, ties to even */
+    int32_t k = (int32_t)kf;
+    float r = x - kf * ln2_hi;
+    r = r - kf * ln2_lo;
+    /* Taylor coefficients 1/n!, n = 7 .. 0 */
+    float p = 1.98412701138295233249664306640625e-04f;    /* 1/5040 */
+    p = p * r + 1.388888922519981861114501953125e-03f;      /* 1/720  */
+    p = p * r + 8.33333376795053482055664062500000e-03f;   /* 1/120  */
+    p = p * r + 4.16666679084300994873046875000000e-02f;   /* 1/24   */
+    p = p * r + 1.66666671633720397949218750000000e-01f;   /* 1/6    */
+    p = p * r + 0.5f;
+    p = p * r + 1.0f;
+    p = p * r + 1.0f;
+    int32_t k1 = k >> 1; /* floor(k/2) for negative k as well */
+    int32_t k2 = k - k1;
+    float y = p * or_pow2i(k1);
+    y = y * or_pow2i(k2);
+    return y;
+}
+
+static float or_sigmoid(float x) {
+    float e = oracle_exp_f32(-x);
+    float den = 1.0f + e;
+    return 1.0f / den;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Frontier-Progress Score of one token (Sec. 4.3).                          */
+/* hist: number of past confidence observations available (0, 1, 2+).       */
+/* Operation order (all fp32, one rounding per operation):                  */
+/*   v    = hist>=2 ? c1 - c2 : 0                    lagged change          */
+/*   vbar = clip(v, -w/2, w/2)                                              */
+/*   chat = clip(c1 + vbar, 0, 1)                    forecast               */
+/*   F    = sig(((chat - theta) + w) / tau) * sig((theta - chat) / tau) Eq.6 */
+/*   P    = hist>=2 ? sig((v_ref - vbar) / tau) : 1                   Eq.7 */
+/*   S    = F * P                                                     Eq.8 */
+/* ------------------------------------------------------------------------ */
+float oracle_fps(float c1, float c2, int32_t hist, float theta, float w_cf,
+                 float v_ref, float tau) {
+    float v = (hist >= 2) ? (c1 - c2) : 0.0f;
+    float half_w = w_cf * 0.5f;
+    float vbar = fminf(fmaxf(v, -half_w), half_w);
+    float chat = fminf(fmaxf(c1 + vbar, 0.0f), 1.0f);
+    float x1 = ((chat - theta) + w_cf) / tau;
+    float x2 = (theta - chat) / tau;
+    float F = or_sigmoid(x1) * or_sigmoid(x2);
+    float P = (hist >= 2) ? or_sigmoid((v_ref - vbar) / tau) : 1.0f;
+    return F * P;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Allocation: RRB (Eq. 5) then FGER (Eq. 9) then clip to [K_min, K_max].   */
+/* Per sequence s (tokens seq_off[s] .. seq_off[s+1]-1, active block a):     */
+/*  1. k_i = H(|b(i) - a|), prompt tokens carry b = 0.                       */
+/*  2. J_h = masked tokens of block a with at least one past confidence.     */
+/*     Other tokens of block a keep K_cur = H(0).                            */
+/*  3. Rank J_h by (S descending, position ascending); n = floor(q |J_h|);   */
+/*     the first n get K_cur + delta_cur, the last n get K_cur - delta_cur.  */
+/*  4. Clip every k to [K_min, K_max].                                       */
+/* Returns OR_EINVAL when an active block index is < 1.                      */
+/* s_out (nullable) receives S for members of J_h and NaN elsewhere.         */
+/* ------------------------------------------------------------------------ */
+static int32_t or_role_count(int32_t dist, int32_t k_base, int32_t d_role) {
+    if (dist <= 1) return k_base + d_role;
+    if (dist == 2) return k_base;
+    return k_base - d_role;
+}
+
+int oracle_allocate(const float* conf1, const float* conf2,
+                    const uint8_t* hist_len, const uint8_t* masked,
+                    const int32_t* block_id, const int32_t* seq_off,
+                    const int32_t* active_block, int32_t T, int32_t B,
+                    int32_t k_min, int32_t k_base, int32_t k_max,
+                    int32_t delta_role, int32_t delta_cur, float q,
+                    float theta, float w_cf, float v_ref, float tau,
+                    int32_t* k_out, float* s_out) {
+    if (T < 0 || B < 0) return OR_EINVAL;
+    if (T > 0 && seq_off[B] != T) return OR_EINVAL;
+    for (int32_t i = 0; i < T; ++i) {
+        if (s_out) s_out[i] = NAN;
+    }
+    for (int32_t s = 0; s < B; ++s) {
+        int32_t lo = seq_off[s], hi = seq_off[s + 1];
+        int32_t a = active_block[s];
+        if (a < 1) return OR_EINVAL;
+        int32_t k_cur = k_base + delta_role;
+        /* step 1: role map */
+        for (int32_t i = lo; i < hi; ++i) {
+            int32_t dist = abs(block_id[i] - a);
+            k_out[i] = or_role_count(dist, k_base, delta_role);
+        }
+        /* step 2: collect J_h with its score */
+        int32_t nj = 0;
+        int32_t* idx = (int32_t*)malloc(sizeof(int32_t) * (size_t)(hi - lo + 1));
+        float* sc = (float*)malloc(sizeof(float) * (size_t)(hi - lo + 1));
+        for (int32_t i = lo; i < hi; ++i) {
+            if (block_id[i] == a && masked[i] && hist_len[i] >= 1) {
+                idx[nj] = i;
+                sc[nj] = oracle_fps(conf1[i], conf2[i], hist_len[i], theta,
+                                    w_cf, v_ref, tau);
+                if (s_out) s_out[i] = sc[nj];
+                ++nj;
+            }
+        }
+        /* step 3: sort J_h by (S desc, position asc) with insertion sort */
+        for (int32_t x = 1; x < nj; ++x) {
+            int32_t ci = idx[x];
+            float cs = sc[x];
+            int32_t y = x - 1;
+            while (y >= 0 && (sc[y] < cs || (sc[y] == cs && idx[y] > ci))) {
+                idx[y + 1] = idx[y];
+                sc[y + 1] = sc[y];
+                --y;
+            }
+            idx[y + 1] = ci;
+            sc[y + 1] = cs;
+        }
+        int32_t n = (int32_t)floorf(q * (float)nj);
+        for (int32_t r = 0; r < nj; ++r) {
+            int32_t i = idx[r];
+            int32_t k = k_cur;
+            if (r < n) k = k_cur + delta_cur;
+            else if (r >= nj - n) k = k_cur - delta_cur;
+            k_out[i] = k;
+        }
+        free(idx);
+        free(sc);
+        /* step 4: clip */
+        for (int32_t i = lo; i < hi; ++i) {
+            int32_t k = k_out[i];
+            if (k < k_min) k = k_min;
+            if (k > k_max) k = k_max;
+            k_out[i] = k;
+        }
+    }
+    return OR_OK;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Router scores: z[t,e] = sum_k h[t,k] * W_r[e,k], as the chain             */
+/*   acc = +0;  for k = 0..d-1: acc = fmaf(h[t,k], W_r[e,k], acc)            */
+/* Inputs are widened exactly from bf16 when dtype = 1.                      */
+/* ------------------------------------------------------------------------ */
+void oracle_router_logits(int32_t dtype, const void* hidden,
+                          const void* w_router, int32_t T, int32_t d,
+                          int32_t E, float* z) {
+#pragma omp parallel for schedule(static)
+    for (int32_t t = 0; t < T; ++t) {
+        for (int32_t e = 0; e < E; ++e) {
+            float acc = 0.0f;
+            for (int32_t k = 0; k < d; ++k) {
+                float h = or_load(hidden, dtype, (int64_t)t * d + k);
+                float w = or_load(w_router, dtype, (int64_t)e * d + k);
+                acc = fmaf(h, w, acc);
+            }
+            z[(int64_t)t * E + e] = acc;
+        }
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* TopK_e(z, k_t) with ties to the lower expert index, then alpha (fp64):    */
+/*   p_e = exp(z_e - max z) / sum_e' exp(z_e' - max z)   (softmax over E)    */
+/*   renorm = 1: alpha_j = p_{ids_j} / sum over the selected set             */
+/*   renorm = 0: alpha_j = p_{ids_j}                                         */
+/* ids/alpha are [T, k_max]; slots j >= k_t hold -1 / 0.                     */
+/* Returns OR_EINVAL when some k_t is outside [1, min(k_max, E)].            */
+/* ------------------------------------------------------------------------ */
+int oracle_select(const float* z, const int32_t* k, int32_t T, int32_t E,
+                  int32_t k_max, int32_t renorm, int32_t* ids,
+                  double* alpha) {
+    int32_t* order = (int32_t*)malloc(sizeof(int32_t) * (size_t)E);
+    for (int32_t t = 0; t < T; ++t) {
+        const float* zt = z + (int64_t)t * E;
+        int32_t kt = k[t];
+        if (kt < 1 || kt > k_max || kt > E) {
+            free(order);
+            return OR_EINVAL;
+        }
+        /* selection: repeatedly take the best remaining expert */
+        for (int32_t e = 0; e < E; ++e) order[e] = e;
+        for (int32_t j = 0; j < kt; ++j) {
+            int32_t best = j;
+            for (int32_t c = j + 1; c < E; ++c) {
+                int32_t ec = order[c], eb = order[best];
+                if (zt[ec] > zt[eb] || (zt[ec] == zt[eb] && ec < eb)) best = c;
+            }
+            int32_t tmp = order[j];
+            order[j] = order[best];
+            order[best] = tmp;
+        }
+        double zmax = (double)zt[order[0]];
+        double all = 0.0, sel = 0.0;
+        for (int32_t e = 0; e < E; ++e) all += exp((double)zt[e] - zmax);
+        for (int32_t j = 0; j < kt; ++j) sel += exp((double)zt[order[j]] - zmax);
+        for (int32_t j = 0; j < k_max; ++j) {
+            int64_t o = (int64_t)t * k_max + j;
+            if (j < kt) {
+                double pe = exp((double)zt[order[j]] - zmax);
+                ids[o] = order[j];
+                alpha[o] = renorm ? pe / sel : pe / all;
+            } else {
+                ids[o] = -1;
+                alpha[o] = 0.0;
+            }
+        }
+    }
+    free(order);
+    return OR_OK;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Pair permutation: the pairs (t, j), j < k_t, ordered by expert, then by   */
+/* token.  perm[p] = t * k_max + j; offsets[e] = first row of expert e;      */
+/* row_of[t*k_max + j] = p (or -1 for unused slots).  Returns sum k_t.        */
+/* ------------------------------------------------------------------------ */
+int64_t oracle_permutation(const int32_t* ids, const int32_t* k, int32_t T,
+                           int32_t E, int32_t k_max, int32_t* offsets,
+                           int32_t* perm, int32_t* row_of) {
+    int64_t pos = 0;
+    for (int64_t o = 0; o < (int64_t)T * k_max; ++o) row_of[o] = -1;
+    for (int32_t e = 0; e < E; ++e) {
+        offsets[e] = (int32_t)pos;
+        for (int32_t t = 0; t < T; ++t) {
+            for (int32_t j = 0; j < k[t]; ++j) {
+                int64_t o = (int64_t)t * k_max + j;
+                if (ids[o] == e) {
+                    perm[pos] = (int32_t)o;
+                    row_of[o] = (int32_t)pos;
+                    ++pos;
+                }
+            }
+        }
+    }
+    offsets[E] = (int32_t)pos;
+    return pos;
+}
+
+/* ------------------------------------------------------------------------ */
+/* One SwiGLU expert on one token, fp64 accumulation:                        */
+/*   g_c = h . Wg[c], u_c = h . Wu[c], a_c = silu(g_c) * u_c,                */
+/*   y_n = sum_c a_c * Wd[n, c]                                              */
+/* w_gate_up rows [0, inter) are gate, [inter, 2 inter) are up; w_down is    */
+/* [d, inter].  y (length d) is accumulated with weight scale.               */
+/* ------------------------------------------------------------------------ */
+static void or_expert_accumulate(int32_t dtype, const double* h,
+                                 const void* w_gate_up, const void* w_down,
+                                 int64_t gu_base, int64_t dn_base, int32_t d,
+                                 int32_t inter, double scale, double* act,
+                                 double* y) {
+    for (int32_t c = 0; c < inter; ++c) {
+        double g = 0.0, u = 0.0;
+        for (int32_t kk = 0; kk < d; ++kk) {
+            g += h[kk] * (double)or_load(w_gate_up, dtype, gu_base + (int64_t)c * d + kk);
+            u += h[kk] * (double)or_load(w_gate_up, dtype, gu_base + (int64_t)(inter + c) * d + kk);
+        }
+        double silu = g / (1.0 + exp(-g));
+        act[c] = silu * u;
+    }
+    for (int32_t n = 0; n < d; ++n) {
+        double acc = 0.0;
+        for (int32_t c = 0; c < inter; ++c)
+            acc += act[c] * (double)or_load(w_down, dtype, dn_base + (int64_t)n * inter + c);
+        y[n] += scale * acc;
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Eq. 2 for the listed tokens:                                              */
+/*   out[r, :] = sum_{j < k_t} alpha[t, j] * E_{ids[t, j]}(h_t)              */
+/*             + shared(h_t)            (when shared_inter > 0)              */
+/* with t = tokens[r].  out is [n_tokens, d] fp64.                           */
+/* ------------------------------------------------------------------------ */
+void oracle_moe_tokens(int32_t dtype, const void* hidden, const void* w_gate_up,
+                       const void* w_down, const void* shared_gate_up,
+                       const void* shared_down, int32_t shared_inter,
+                       const int32_t* ids, const double* alpha,
+                       const int32_t* k, const int32_t* tokens,
+                       int32_t n_tokens, int32_t d, int32_t inter,
+                       int32_t k_max, double* out) {
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int32_t r = 0; r < n_tokens; ++r) {
+        int32_t t = tokens[r];
+        double* h = (double*)malloc(sizeof(double) * (size_t)d);
+        int32_t amax = inter > shared_inter ? inter : shared_inter;
+        double* act = (double*)malloc(sizeof(double) * (size_t)(amax > 0 ? amax : 1));
+        double* y = out + (int64_t)r * d;
+        for (int32_t kk = 0; kk < d; ++kk) {
+            h[kk] = (double)or_load(hidden, dtype, (int64_t)t * d + kk);
+            y[kk] = 0.0;
+        }
+        for (int32_t j = 0; j < k[t]; ++j) {
+            int64_t o = (int64_t)t * k_max + j;
+            int64_t e = ids[o];
+            or_expert_accumulate(dtype, h, w_gate_up, w_down,
+                                 e * 2 * (int64_t)inter * d,
+                                 e * (int64_t)d * inter, d, inter, alpha[o],
+                                 act, y);
+        }
+        if (shared_inter > 0)
+            or_expert_accumulate(dtype, h, shared_gate_up, shared_down, 0, 0,
+                                 d, shared_inter, 1.0, act, y);
+        free(h);
+        free(act);
+    }
+}
+
+int oracle_num_threads(void) {
+#ifdef _OPENMP
+    extern int omp_get_max_threads(void);
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/* Array forms used by the pins and by the parity tests. */
+void oracle_exp_f32_n(const float* x, float* y, int64_t n) {
+    for (int64_t i = 0; i < n; ++i) y[i] = oracle_exp_f32(x[i]);
+}
+
+void oracle_fps_n(const float* c1, const float* c2, const uint8_t* hist,
+                  int64_t n, float theta, float w_cf, float v_ref, float tau,
+                  float* s) {
+    for (int64_t i = 0; i < n; ++i)
+        s[i] = oracle_fps(c1[i], c2[i], hist[i], theta, w_cf, v_ref, tau);
+}
