@@ -1,0 +1,421 @@
+"""Benchmark of the REFLEX per-forward MoE hot path on GB300.
+
+One step = one denoising forward's hot path on one batch:
+  reflex_allocate (per-token counts, Eq. 5 / Eq. 9 + clip)
+  + reflex_moe_forward (router scores, variable-count TopK, pair dispatch,
+    grouped SwiGLU expert GEMMs on tcgen05, weighted combine; Eq. 2).
+Default workload: the LLaDA-MoE-shaped layer (T = 1024 tokens: 512 prompt +
+512 generated in blocks of 32; d = 2048, E = 64 SwiGLU experts with inter =
+1024; K in [2, 12]; bf16 storage, fp32 accumulation), synthetic inputs.
+
+Prints ONE JSON line (rank 0).  `value` = MoE-layer tokens/s over all ranks;
+`expert_tflops` = 6 d inter sum(k) / step time (Eq. 10); the same kernels at
+fixed top-K_base run beside it; `roofline` is for the dominant kernel, the
+grouped gate/up (SwiGLU) GEMM; `e2e` times the same step from pinned host
+buffers through the C ABI with the copies inside the timed region.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reflex|reference]
+                  [--config NAME] [--no-cpu-baseline]
+Under torchrun each rank runs its own batch on its own GPU (weak scaling, no
+data-path collective; a barrier and a max-reduce of the times only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2608_01784_gb300 import workloads as W  # noqa: E402
+
+# Bytes moved by the dominant kernel per launch, from an ncu capture of the
+# current kernel (profiles/); None when the kernel changed since the capture.
+NCU_TRAFFIC_BYTES = None
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="reflex", choices=["reflex", "reference"])
+    ap.add_argument("--config", default="llada_moe", choices=sorted(W.CONFIGS))
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target seconds of oracle work for cpu_baseline")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"],
+                    bf16_sustained=d.get("bf16_tflops_sustained"),
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,"
+              "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return dict(sm_mhz=None, sm_max_mhz=None, reasons=[], samples=0)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out = ""
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return dict(sm_mhz=statistics.median(sm) if sm else None,
+                    sm_max_mhz=max(mx) if mx else None,
+                    reasons=sorted(reasons), samples=len(sm))
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle leg (cpu_baseline and --impl reference)
+# ---------------------------------------------------------------------------
+def oracle_step(cfg, layer, state, tokens):
+    """The oracle's whole path for the listed tokens: allocation (whole batch;
+    the count rule couples the tokens of an active block), router scores,
+    TopK / alpha, pair order, Eq. 2."""
+    import oracle
+    k = oracle.allocate(state["conf1"], state["conf2"], state["hist_len"],
+                        state["masked"], state["block_id"], state["seq_offsets"],
+                        state["active_block"], **cfg.alloc_params())
+    h = layer["hidden"][tokens]
+    z = oracle.router_logits(h, layer["w_router"])
+    ks = k[tokens]
+    ids, alpha = oracle.select(z, ks, cfg.k_max)
+    oracle.permutation(ids, ks, cfg.E)
+    sub = np.arange(len(tokens), dtype=np.int32)
+    oracle.moe_tokens(h, layer["w_gate_up"], layer["w_down"], ids, alpha, ks, sub,
+                      shared_gate_up=layer.get("shared_gate_up"),
+                      shared_down=layer.get("shared_down"))
+    return int(ks.sum())
+
+
+def oracle_rate(cfg, layer, state, target_s, seed=0):
+    """tokens/s of the oracle on a seeded token sample sized to ~target_s."""
+    import oracle
+    oracle.build()
+    T = layer["hidden"].shape[0]
+    rng = np.random.default_rng(seed)
+    n = min(T, 16)
+    t0 = time.perf_counter()
+    oracle_step(cfg, layer, state, np.sort(rng.choice(T, n, replace=False)).astype(np.int32))
+    dt = time.perf_counter() - t0
+    n2 = int(min(T, max(n, n * target_s / max(dt, 1e-6))))
+    toks = np.sort(rng.choice(T, n2, replace=False)).astype(np.int32)
+    t0 = time.perf_counter()
+    oracle_step(cfg, layer, state, toks)
+    dt = time.perf_counter() - t0
+    return n2 / dt, n2, dt, oracle.num_threads()
+
+
+def run_reference(args, cfg, rank, world):
+    import torch  # noqa: F401  (keeps the launch environment identical)
+    if rank != 0:
+        return
+    layer = W.make_layer(cfg, args.seed)
+    state = W.make_state(cfg, args.seed)
+    import oracle
+    oracle.build()
+    T = cfg.T
+    rng = np.random.default_rng(args.seed)
+    # per step: a seeded token sample sized so that W + K steps stay within a
+    # few minutes
+    per_step_s = max(0.5, min(5.0, 150.0 / max(1, args.steps + args.warmup)))
+    n = min(T, 8)
+    t0 = time.perf_counter()
+    oracle_step(cfg, layer, state, np.arange(n, dtype=np.int32))
+    dt = time.perf_counter() - t0
+    n = int(min(T, max(1, n * per_step_s / max(dt, 1e-6))))
+    for _ in range(args.warmup):
+        oracle_step(cfg, layer, state, np.sort(rng.choice(T, n, replace=False)).astype(np.int32))
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_step(cfg, layer, state, np.sort(rng.choice(T, n, replace=False)).astype(np.int32))
+    dt = time.perf_counter() - t0
+    value = n * args.steps / dt
+    line = dict(metric="moe_layer_tokens_per_s", value=value, unit="tokens/s",
+                impl="reference", n_gpus=args.gpus, steps=args.steps,
+                warmup=args.warmup, ms_per_step=1e3 * dt / args.steps,
+                higher_is_better=True, scaling="weak", vs_baseline=None,
+                dtype="f64", data="synthetic",
+                config=dict(workload=cfg.name, description=cfg.description,
+                            tokens_per_step_sample=n),
+                cpu_baseline=dict(value=value, unit="tokens/s", kind="oracle",
+                                  cores=oracle.num_threads(),
+                                  sample=f"{n} seeded tokens of the {T}-token "
+                                         f"batch per step (allocation on the "
+                                         f"whole batch)"),
+                e2e=dict(value=value, unit="tokens/s", h2d_bytes_per_step=0,
+                         d2h_bytes_per_step=0))
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU leg
+# ---------------------------------------------------------------------------
+def run_gpu(args, cfg, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    from paper_2608_01784_gb300 import _binding as B
+    from paper_2608_01784_gb300 import api, build
+
+    build.build()
+    B.load()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    seed = args.seed + rank
+    layer = W.make_layer(cfg, seed)
+    state = W.make_state(cfg, seed)
+    T, d, E, I, S, km = cfg.T, cfg.d, cfg.E, cfg.inter, cfg.shared_inter, cfg.k_max
+    dl = api.layer_to_device(layer, cfg.dtype, dev)
+    ds = api.state_to_device(state, dev)
+    moe = api.MoELayer(dl, dtype=cfg.dtype, d=d, E=E, inter=I, shared_inter=S,
+                       k_max=km, max_tokens=T, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    p_reflex = B.make_params(**cfg.alloc_params())
+    p_fixed = B.make_params(**cfg.alloc_params(delta_role=0, delta_cur=0))
+    k_buf = torch.empty(T, dtype=torch.int32, device=dev)
+    k_sum = torch.zeros(1, dtype=torch.int64, device=dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    out = torch.empty((T, d), dtype=moe.tdtype, device=dev)
+    F = B.REFLEX_FLAG_RENORM_TOPK
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+
+    def step(params, up_events=None, hidden=None):
+        api.allocate(ds, params, E, stream, k_buf, k_sum, st)
+        h = dl["hidden"] if hidden is None else hidden
+        moe.forward(h, k_buf, out, F | B.REFLEX_STAGE_ROUTE | B.REFLEX_STAGE_DISPATCH)
+        if up_events is not None:
+            up_events[0].record(stream)
+        moe.forward(h, k_buf, out, F | B.REFLEX_STAGE_EXPERT_UP)
+        if up_events is not None:
+            up_events[1].record(stream)
+        moe.forward(h, k_buf, out, F | B.REFLEX_STAGE_EXPERT_DOWN | B.REFLEX_STAGE_COMBINE)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    def timed(params, steps, warmup, up_times=None):
+        for _ in range(warmup):
+            step(params)
+        barrier()
+        start, stop = (torch.cuda.Event(enable_timing=True) for _ in range(2))
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)]
+               for _ in range(steps)] if up_times is not None else None
+        start.record(stream)
+        for i in range(steps):
+            step(params, evs[i] if evs else None)
+        stop.record(stream)
+        barrier()
+        ms = start.elapsed_time(stop)
+        if up_times is not None:
+            up_times.extend(e[0].elapsed_time(e[1]) for e in evs)
+        return ms
+
+    def max_over_ranks(x: float) -> float:
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    # correctness gate before timing: counts and routing status clean
+    step(p_reflex)
+    torch.cuda.synchronize(dev)
+    assert B.reflex_read_status(st) == B.REFLEX_OK
+    assert moe.status() == B.REFLEX_OK
+    pairs = int(k_sum.item())
+    rec = moe.record()
+    counts = rec["counts"].cpu().numpy()
+    step(p_fixed)
+    torch.cuda.synchronize(dev)
+    pairs_fixed = int(k_sum.item())
+
+    # ---- timed region: REFLEX counts ----
+    clk = ClockSampler(local_rank)
+    clk.start()
+    up_times: list[float] = []
+    ms = timed(p_reflex, args.steps, args.warmup, up_times)
+    clocks = clk.stop()
+    ms = max_over_ranks(ms)
+    ms_step = ms / args.steps
+    # ---- same kernels at fixed top-K_base ----
+    ms_fixed = max_over_ranks(timed(p_fixed, max(1, args.steps // 2), 2)) / max(1, args.steps // 2)
+
+    # ---- end to end from pinned host buffers ----
+    host_in = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
+               for k, v in state.items()}
+    host_h = torch.from_numpy(np.ascontiguousarray(layer["hidden"]).view(
+        np.int16 if cfg.dtype == "bf16" else np.float32)).pin_memory()
+    host_out = torch.empty((T, d), dtype=moe.tdtype).pin_memory()
+    dev_h = torch.empty_like(dl["hidden"])
+    h2d = sum(int(v.numel() * v.element_size()) for v in host_in.values()) + \
+        int(host_h.numel() * host_h.element_size())
+    d2h = int(host_out.numel() * host_out.element_size())
+
+    def e2e_step():
+        for k, v in host_in.items():
+            ds[k].copy_(v, non_blocking=True)
+        dev_h.view(host_h.dtype).copy_(host_h, non_blocking=True)
+        step(p_reflex, hidden=dev_h)
+        host_out.copy_(out, non_blocking=True)
+
+    for _ in range(max(3, args.warmup // 2)):
+        e2e_step()
+    barrier()
+    n_e2e = max(3, args.steps // 2)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(n_e2e):
+        e2e_step()
+    e1.record(stream)
+    barrier()
+    ms_e2e = max_over_ranks(e0.elapsed_time(e1)) / n_e2e
+
+    if rank != 0:
+        return
+    peaks = load_peaks()
+    tokens_per_s = T * world / (ms_step * 1e-3)
+    flops_step = 6.0 * d * I * pairs          # Eq. 10, routed experts
+    # dominant kernel: grouped gate/up GEMM; algorithmic bytes per launch =
+    # gate/up weights of the experts that received pairs + gathered rows read
+    # + activations written (bf16)
+    es = 2 if cfg.dtype == "bf16" else 4
+    touched = int((counts > 0).sum())
+    up_bytes = touched * 2 * I * d * es + pairs * d * es + pairs * I * es
+    if S:
+        up_bytes += 2 * S * d * es + T * d * es + T * S * es
+    up_flops = 4.0 * pairs * d * I + (4.0 * T * d * S if S else 0.0)
+    up_ms = statistics.mean(up_times) if up_times else float("nan")
+    achieved_gbs = up_bytes / (up_ms * 1e-3) / 1e9
+    hbm_bound = up_bytes / (peaks["hbm"] * 1e9) >= up_flops / (peaks["bf16"] * 1e12)
+    if hbm_bound:
+        roof = dict(bound="hbm", achieved=achieved_gbs, peak=peaks["hbm"],
+                    unit="GB/s", frac=achieved_gbs / peaks["hbm"])
+    else:
+        tf = up_flops / (up_ms * 1e-3) / 1e12
+        roof = dict(bound="tensor", achieved=tf, peak=peaks["bf16"],
+                    unit="TFLOP/s", frac=tf / peaks["bf16"])
+    roof.update(kernel="grouped_gemm_kernel<256, SwiGLU> (gate/up + SwiGLU)",
+                traffic=NCU_TRAFFIC_BYTES, algorithmic_bytes=up_bytes,
+                algorithmic_flops=up_flops, avg_launch_ms=up_ms,
+                peak_source=peaks["source"] + " (burst)")
+    # layer roofline: all expert weights touched + hidden in/out vs Eq. 10 flops
+    layer_bytes = touched * 3 * I * d * es + 2 * T * d * es + E * d * es
+    if S:
+        layer_bytes += 3 * S * d * es
+    layer_flops = flops_step + (6.0 * d * S * T if S else 0.0)
+    t_roof = max(layer_bytes / (peaks["hbm"] * 1e9), layer_flops / (peaks["bf16"] * 1e12))
+    launches_per_step = 10 + (2 if S else 0)
+    line = dict(
+        metric="moe_layer_tokens_per_s", value=tokens_per_s, unit="tokens/s",
+        n_gpus=world, steps=args.steps, warmup=args.warmup, ms_per_step=ms_step,
+        higher_is_better=True, scaling="weak", vs_baseline=None, dtype="bf16"
+        if cfg.dtype == "bf16" else "f32", data="synthetic",
+        config=dict(workload=cfg.name, description=cfg.description,
+                    tokens_per_step=T, parallelism=f"replicas{world}",
+                    l2="no flush: expert weights > 129 MB L2 stream from HBM every step"),
+        expert_tflops=flops_step * world / (ms_step * 1e-3) / 1e12,
+        layer_roofline_frac=t_roof / (ms_step * 1e-3),
+        avg_k=pairs / T, pairs=pairs,
+        fixed_topk=dict(k=cfg.k_base, pairs=pairs_fixed, ms_per_step=ms_fixed,
+                        value=T * world / (ms_fixed * 1e-3),
+                        expert_tflops=6.0 * d * I * pairs_fixed * world / (ms_fixed * 1e-3) / 1e12),
+        roofline=roof,
+        e2e=dict(value=T * world / (ms_e2e * 1e-3), unit="tokens/s",
+                 h2d_bytes_per_step=h2d, d2h_bytes_per_step=d2h,
+                 ms_per_step=ms_e2e),
+        gpu_launches=launches_per_step * args.steps,
+        clocks=dict(sm_mhz=clocks["sm_mhz"], sm_max_mhz=clocks["sm_max_mhz"],
+                    reasons=clocks["reasons"], samples=clocks["samples"]),
+    )
+    if not args.no_cpu_baseline and world == 1:
+        rate, n, dt, cores = oracle_rate(cfg, layer, state, args.cpu_seconds, seed)
+        line["cpu_baseline"] = dict(
+            value=rate, unit="tokens/s", cores=cores, kind="oracle",
+            sample=f"{n} seeded tokens of the {T}-token batch, full oracle path "
+                   f"(allocation on the whole batch), {dt:.1f} s")
+    elif world > 1:
+        line["cpu_baseline"] = None
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    cfg = W.CONFIGS[args.config]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if args.impl == "reflex" else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local_rank)
+        dist.init_process_group(backend=backend)
+    try:
+        if args.impl == "reference":
+            run_reference(args, cfg, rank, world)
+        else:
+            run_gpu(args, cfg, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,213 @@
+/*
+ * reflex.h — C ABI of the REFLEX per-forward MoE hot path on one GB300
+ * (sm_103a).  Library: paper_2608_01784_gb300/_build/libreflex.so.
+ *
+ * REFLEX (arxiv 2608.01784) splits token-choice MoE inference into expert
+ * ranking (left to the default router) and expert-count allocation.  This
+ * library implements both halves of one denoising forward:
+ *
+ *   reflex_allocate     the allocation rule k = Pi(S_t, K^Sigma) of Eq. 3,
+ *                       realised by Refinement-Role Budgeting (Sec. 4.2,
+ *                       Eq. 5) and Frontier-Guided Expert Reallocation
+ *                       (Sec. 4.3, Eq. 6-9), clipped to [K_min, K_max].
+ *   reflex_moe_forward  the variable-count MoE layer of Eq. 2: router scores,
+ *                       TopK(r_i, k_i), normalised router weights, SwiGLU
+ *                       experts on the selected token-expert pairs, weighted
+ *                       sum (plus an optional always-on shared expert).
+ *
+ * Conventions shared by every call
+ *   - All array arguments are DEVICE pointers unless stated otherwise; the
+ *     caller owns them.  The library never allocates or frees device memory
+ *     and never synchronises the stream, except reflex_moe_status and
+ *     reflex_read_status, which synchronise to read an error word.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy stream).  All
+ *     work is enqueued asynchronously on it.
+ *   - Row-major layouts.  Integer arrays are int32 unless stated.
+ *   - Return value: a REFLEX_* status.  Host-side checks (null pointers,
+ *     shapes, workspace size) return before anything is enqueued.  Checks
+ *     that need device data (a count k_i out of range, too many active-block
+ *     tokens) set bits in a device error word; read it with
+ *     reflex_moe_status / reflex_read_status.
+ */
+#ifndef REFLEX_H
+#define REFLEX_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------- */
+#define REFLEX_OK 0
+#define REFLEX_EINVAL 1        /* null pointer, bad shape or parameter       */
+#define REFLEX_EKRANGE 2       /* a count outside its allowed range          */
+#define REFLEX_EWORKSPACE 3    /* workspace missing or smaller than needed   */
+#define REFLEX_ECUDA 4         /* a CUDA runtime / launch error              */
+#define REFLEX_ETIMEOUT 5      /* a bounded device wait expired              */
+#define REFLEX_EUNSUPPORTED 6  /* shape not supported by the selected path   */
+#define REFLEX_ECAPACITY 7     /* more active-block tokens than supported    */
+
+/* ---- element types ------------------------------------------------------ */
+#define REFLEX_DTYPE_F32 0     /* fp32 storage and fp32 arithmetic           */
+#define REFLEX_DTYPE_BF16 1    /* bf16 storage, fp32 accumulation            */
+
+/* ---- reflex_moe_forward flags ------------------------------------------ */
+/* alpha renormalised over the selected experts (default reading of the
+ * "normalized router weight" of Sec. 3.2); without it alpha is the softmax
+ * over all E experts. */
+#define REFLEX_FLAG_RENORM_TOPK 0x1u
+/* bf16 only: run the expert GEMMs on the SIMT kernels instead of the
+ * tcgen05/TMEM kernels (cross-checking; the fp32 path always uses SIMT). */
+#define REFLEX_FLAG_SIMT_EXPERTS 0x2u
+/* Stage selection.  No stage bit = all five stages in order.  Stages read
+ * what the previous stages left in the same workspace; running a stage whose
+ * predecessors did not run on that workspace gives unspecified values (every
+ * index read from the workspace is range-checked on the device, so no
+ * out-of-bounds access results). */
+#define REFLEX_STAGE_ROUTE 0x100u       /* router scores, TopK, alpha        */
+#define REFLEX_STAGE_DISPATCH 0x200u    /* pair counts, offsets, permutation */
+#define REFLEX_STAGE_EXPERT_UP 0x400u   /* gate/up GEMM + SwiGLU (+ shared)  */
+#define REFLEX_STAGE_EXPERT_DOWN 0x800u /* down GEMM (+ shared)              */
+#define REFLEX_STAGE_COMBINE 0x1000u    /* weighted sum back to token order  */
+
+/* ---- allocation hyper-parameters (Sec. 4.2-4.3; defaults in Sec. 5.1) --- */
+typedef struct {
+    int32_t k_min;      /* lower clip bound of every count, >= 1            */
+    int32_t k_base;     /* K_base of Eq. 5                                  */
+    int32_t k_max;      /* upper clip bound, >= k_min                       */
+    int32_t delta_role; /* delta_role of Eq. 5 (0 = no role prior)          */
+    int32_t delta_cur;  /* delta_cur of Eq. 9 (0 = no reallocation)         */
+    float q;            /* outer-group fraction of Eq. 9, in (0, 1/2]       */
+    float theta;        /* commitment threshold of Eq. 6                    */
+    float w_cf;         /* commitment-frontier width of Eq. 6 and the
+                           velocity clip, > 0                               */
+    float v_ref;        /* velocity reference of Eq. 7                      */
+    float tau;          /* gate temperature of Eq. 6-7, > 0                 */
+} reflex_alloc_params;
+
+/* Fills the Sec. 5.1 defaults: k_base 8, delta_role 4, delta_cur 2, q 0.25,
+ * theta 0.9, w_cf 0.30 (LLaDA-MoE; 0.25 for LLaDA2.0-mini), v_ref 0.01,
+ * tau 0.05, and the clip [k_min, k_max] = [2, 12]. */
+void reflex_default_params(reflex_alloc_params* p);
+
+/*
+ * reflex_allocate — per-token expert counts k_i for one denoising forward
+ * (Eq. 3 realised by Eq. 5 and Eq. 9, Sec. 4.2-4.3).
+ *
+ *   router_scores  [T, E] fp32, nullable.  Accepted for the shape of the
+ *                  allocation problem; REFLEX's rule does not read it (the
+ *                  router only ranks experts, Sec. 3.3).
+ *   conf_prev1     [T] fp32  c_i^{t-1}, the latest confidence observation.
+ *   conf_prev2     [T] fp32  c_i^{t-2}; read only where hist_len >= 2.
+ *   hist_len       [T] u8    number of past observations (0, 1, >= 2).
+ *   masked         [T] u8    1 = position is [MASK] (member of M_t).
+ *   block_id       [T] int32 b(i): 0 for prompt positions, 1..Q for target
+ *                            blocks.
+ *   seq_offsets    [B+1]     token range of each sequence; seq_offsets[0] = 0,
+ *                            seq_offsets[B] = T, non-decreasing.
+ *   active_block   [B]       a_t of each sequence, >= 1.
+ *   p              HOST pointer to the hyper-parameters.
+ *   k_out          [T] int32 output counts, each in [k_min, k_max].
+ *   k_sum_out      [1] int64 nullable: sum of k_out (the realised budget).
+ *   dev_status     [1] int32 nullable device error word; cleared by this
+ *                  call, then OR-ed with error bits (see reflex_read_status).
+ * Tokens of the active block that are masked and have at least one
+ * observation form J_h and are ranked by the Frontier-Progress Score (ties:
+ * lower position first); at most 4096 such tokens per sequence (more sets
+ * REFLEX_ECAPACITY in dev_status and leaves them at K_cur, clipped).
+ * Host errors: REFLEX_EINVAL for null required pointers, T < 0, B < 1, or
+ * parameters violating 1 <= k_min <= k_max, k_base >= 1, delta_* >= 0,
+ * 0 < q <= 0.5, w_cf > 0, tau > 0.  Counts below k_min (or above k_max)
+ * produced by Eq. 5 / Eq. 9 are clipped.
+ */
+int reflex_allocate(const float* router_scores, const float* conf_prev1,
+                    const float* conf_prev2, const uint8_t* hist_len,
+                    const uint8_t* masked, const int32_t* block_id,
+                    const int32_t* seq_offsets, const int32_t* active_block,
+                    int32_t T, int32_t B, int32_t E,
+                    const reflex_alloc_params* p, int32_t* k_out,
+                    int64_t* k_sum_out, int32_t* dev_status, void* stream);
+
+/* Device pointers into the workspace after a forward (the routing record). */
+typedef struct {
+    int32_t* ids;     /* [T, k_max] selected experts in router rank order,
+                         -1 in slots j >= k_i                               */
+    float* alpha;     /* [T, k_max] normalised router weights, 0 padded     */
+    int32_t* counts;  /* [E] pairs per expert                               */
+    int32_t* offsets; /* [E+1] first pair row of each expert                */
+    int32_t* perm;    /* [sum k] pair rows: token * k_max + slot, ordered by
+                         (expert, token)                                    */
+    int32_t* row_of;  /* [T, k_max] pair row of (token, slot), -1 unused    */
+    int32_t* totals;  /* [2] device: sum k (pairs), number of 128-row tiles */
+} reflex_route_record;
+
+/* Bytes of workspace reflex_moe_forward needs for these shapes (0 if the
+ * shapes are invalid).  Sized for the worst case T * k_max pairs, so the
+ * forward never reads back the realised sum of k. */
+size_t reflex_moe_workspace_size(int32_t dtype, int32_t T, int32_t d,
+                                 int32_t E, int32_t inter,
+                                 int32_t shared_inter, int32_t k_max);
+
+/*
+ * reflex_moe_forward — the variable-count MoE layer, Eq. 2 (Sec. 3.2):
+ *   out_i = sum_{e in TopK(r_i, k_i)} alpha_{i,e} E_e(h_i)  [+ shared(h_i)]
+ * with r_i = h_i W_r^T (fp32; each score is the sequential fused
+ * multiply-add chain over the hidden index from +0), TopK ties broken to the
+ * lower expert index, and SwiGLU experts
+ *   E_e(h) = (silu(h W_g,e^T) * (h W_u,e^T)) W_d,e^T.
+ *
+ *   dtype           REFLEX_DTYPE_F32 or REFLEX_DTYPE_BF16 (all float arrays).
+ *   hidden          [T, d]
+ *   w_router        [E, d]
+ *   w_gate_up       [E, 2*inter, d]: rows [0, inter) gate, [inter, 2*inter) up
+ *   w_down          [E, d, inter]
+ *   shared_gate_up  [2*shared_inter, d], nullable (with shared_inter = 0)
+ *   shared_down     [d, shared_inter]
+ *   k               [T] int32 counts (from reflex_allocate or any rule);
+ *                   each must lie in [1, min(k_max, E)] (else the device
+ *                   error word gets REFLEX_EKRANGE and the count is clamped).
+ *   flags           REFLEX_FLAG_* | REFLEX_STAGE_* (see above).
+ *   workspace       >= reflex_moe_workspace_size(...) bytes, 256-B aligned.
+ *   out             [T, d] output.
+ *   rec             HOST struct, nullable: receives device pointers into the
+ *                   workspace (no copy is made).
+ * Shape rules: T >= 0, d % 64 == 0, 1 <= E <= 1024, 1 <= k_max <= 32,
+ * inter % 64 == 0, shared_inter % 64 == 0.  The bf16 tcgen05 path also needs
+ * d % 256 == 0 and inter, shared_inter % 128 == 0 (else REFLEX_EUNSUPPORTED
+ * unless REFLEX_FLAG_SIMT_EXPERTS is given).
+ */
+int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
+                       const void* w_gate_up, const void* w_down,
+                       const void* shared_gate_up, const void* shared_down,
+                       int32_t shared_inter, const int32_t* k, int32_t T,
+                       int32_t d, int32_t E, int32_t inter, int32_t k_max,
+                       uint32_t flags, void* workspace, size_t ws_bytes,
+                       void* out, reflex_route_record* rec, void* stream);
+
+/* Synchronises `stream` and returns the status recorded in the workspace's
+ * device error word by the last forward (REFLEX_OK if clean). */
+int reflex_moe_status(const void* workspace, void* stream);
+
+/* Same for a caller-owned device error word (e.g. reflex_allocate's). */
+int reflex_read_status(const int32_t* dev_status, void* stream);
+
+/* Bounded-wait self-test: launches one block that waits on an mbarrier no
+ * one arrives at, with a limit of `limit_us` microseconds (1..100000), then
+ * records REFLEX_ETIMEOUT in dev_status and returns.  Exercises the same
+ * wait routine the tcgen05 pipeline uses; nothing hangs. */
+int reflex_selftest_wait_timeout(int32_t* dev_status, uint32_t limit_us,
+                                 void* stream);
+
+/* Human-readable status. */
+const char* reflex_status_string(int status);
+
+/* Version of this ABI (major * 100 + minor). */
+int reflex_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* REFLEX_H */

@@ -1,0 +1,117 @@
+"""Torch-facing convenience over the C ABI: device buffers, workspace and
+route-record views.  PyTorch provides memory and streams only; every step of
+the path runs in libreflex.so's kernels.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import _binding as B
+
+
+def _dev(a: np.ndarray, device, dtype=None) -> torch.Tensor:
+    t = torch.from_numpy(np.ascontiguousarray(a))
+    if dtype is not None:
+        t = t.view(dtype)
+    return t.to(device, non_blocking=False)
+
+
+def layer_to_device(layer: dict, dtype: str, device="cuda") -> dict:
+    """Host arrays (fp32, or bf16 bit patterns as uint16) -> device tensors."""
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    out = {}
+    for k, v in layer.items():
+        if v.dtype == np.uint16:
+            out[k] = _dev(v.view(np.int16), device).view(tdt)
+        else:
+            out[k] = _dev(v, device)
+    return out
+
+
+def state_to_device(state: dict, device="cuda") -> dict:
+    return {k: _dev(v, device) for k, v in state.items()}
+
+
+def allocate(state: dict, params: B.reflex_alloc_params, E: int = 0,
+             stream=None, k_out: torch.Tensor | None = None,
+             k_sum: torch.Tensor | None = None,
+             status: torch.Tensor | None = None):
+    """reflex_allocate on device state tensors -> (k int32 [T], k_sum int64 [1],
+    status int32 [1])."""
+    T = int(state["block_id"].numel())
+    nseq = int(state["active_block"].numel())
+    dev = state["block_id"].device
+    k_out = torch.empty(T, dtype=torch.int32, device=dev) if k_out is None else k_out
+    k_sum = torch.zeros(1, dtype=torch.int64, device=dev) if k_sum is None else k_sum
+    status = torch.zeros(1, dtype=torch.int32, device=dev) if status is None else status
+    B.reflex_allocate(None, state["conf1"], state["conf2"], state["hist_len"],
+                      state["masked"], state["block_id"], state["seq_offsets"],
+                      state["active_block"], T, nseq, E, params, k_out, k_sum,
+                      status, stream)
+    return k_out, k_sum, status
+
+
+class MoELayer:
+    """One variable-count MoE layer on the device with its workspace sized for
+    `max_tokens` tokens at `k_max`."""
+
+    def __init__(self, weights: dict, *, dtype: str, d: int, E: int, inter: int,
+                 shared_inter: int, k_max: int, max_tokens: int, device="cuda"):
+        self.w = weights
+        self.dtype = B.REFLEX_DTYPE_BF16 if dtype == "bf16" else B.REFLEX_DTYPE_F32
+        self.tdtype = torch.bfloat16 if dtype == "bf16" else torch.float32
+        self.d, self.E, self.inter = d, E, inter
+        self.shared_inter = shared_inter
+        self.k_max = k_max
+        self.max_tokens = max_tokens
+        self.ws_bytes = B.reflex_moe_workspace_size(self.dtype, max_tokens, d, E,
+                                                    inter, shared_inter, k_max)
+        if self.ws_bytes == 0:
+            raise ValueError("unsupported MoE layer shape")
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
+        self.rec = B.reflex_route_record()
+        self._T = 0
+
+    def forward(self, hidden: torch.Tensor, k: torch.Tensor, out=None,
+                flags: int = B.REFLEX_FLAG_RENORM_TOPK, stream=None,
+                check: bool = True) -> torch.Tensor:
+        T = int(hidden.shape[0])
+        if T > self.max_tokens:
+            raise ValueError("more tokens than the workspace was sized for")
+        if out is None:
+            out = torch.empty((T, self.d), dtype=self.tdtype, device=hidden.device)
+        ws_bytes = B.reflex_moe_workspace_size(self.dtype, T, self.d, self.E,
+                                               self.inter, self.shared_inter,
+                                               self.k_max)
+        B.reflex_moe_forward(self.dtype, hidden, self.w["w_router"],
+                             self.w["w_gate_up"], self.w["w_down"],
+                             self.w.get("shared_gate_up"), self.w.get("shared_down"),
+                             self.shared_inter, k, T, self.d, self.E, self.inter,
+                             self.k_max, flags, self.ws, ws_bytes, out, self.rec,
+                             stream, check)
+        self._T = T
+        return out
+
+    def status(self, stream=None) -> int:
+        return B.reflex_moe_status(self.ws, stream)
+
+    def _view(self, addr: int, n: int, dtype=torch.int32) -> torch.Tensor:
+        off = addr - self.ws.data_ptr()
+        nbytes = n * torch.empty((), dtype=dtype).element_size()
+        return self.ws[off:off + nbytes].view(dtype)
+
+    def record(self) -> dict:
+        """Views (no copies) of the routing record of the last forward."""
+        T, km, E = self._T, self.k_max, self.E
+        totals = self._view(self.rec.totals, 2)
+        n_pairs = int(totals[0].item())
+        return dict(
+            ids=self._view(self.rec.ids, T * km).view(T, km),
+            alpha=self._view(self.rec.alpha, T * km, torch.float32).view(T, km),
+            counts=self._view(self.rec.counts, E),
+            offsets=self._view(self.rec.offsets, E + 1),
+            perm=self._view(self.rec.perm, n_pairs),
+            row_of=self._view(self.rec.row_of, T * km).view(T, km),
+            totals=totals,
+        )

@@ -1,0 +1,213 @@
+// budget.cu — per-token expert counts of one denoising forward (REFLEX,
+// Sec. 4.2-4.3): Refinement-Role Budgeting (Eq. 5), Frontier-Guided Expert
+// Reallocation with the Frontier-Progress Score (forecast, Eq. 6-8, Eq. 9),
+// then the clip to [K_min, K_max] of the count set in Eq. 3.
+//
+// One CTA per sequence.  Pass 1 writes the role count of every token and
+// gathers J_h (masked active-block tokens with history) with their scores in
+// shared memory; pass 2 ranks J_h by (S desc, position asc) with an
+// all-pairs rank count — the block holds a few dozen tokens (block length 32
+// in Sec. 5.1), so the O(|J|^2) count is a few hundred compares per thread.
+//
+// The score is computed in fp32 with one rounding per operation, in a fixed
+// order, and with an exp written here from Cody & Waite's argument reduction
+// and a degree-7 Taylor polynomial, so that the ranking (an integer result)
+// is reproducible bit for bit.
+#include "common.cuh"
+#include "internal.h"
+
+namespace rx {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kMaxJ = 4096;
+
+__device__ __forceinline__ float pow2i(int e) {  // e in [-126, 127]
+  return __int_as_float((e + 127) << 23);
+}
+
+// e^x: x = k ln2 + r with k = nearest integer to x / ln2 (ties to even);
+// r = (x - k ln2_hi) - k ln2_lo (ln2_hi has 16 significant bits, so k ln2_hi
+// is exact); e^r by the Taylor series to r^7 in Horner form; the scale 2^k is
+// applied as two powers of two so that neither overflows and a subnormal
+// result is rounded once.
+__device__ float exp_cw(float x) {
+  if (x != x) return x;
+  if (x >= 89.0f) return __int_as_float(0x7f800000);
+  if (x <= -104.0f) return 0.0f;
+  const float inv_ln2 = 1.44269502162933349609375f;
+  const float ln2_hi = 0.693145751953125f;
+  const float ln2_lo = 1.428606765330187045037746429443359375e-06f;
+  const float kf = rintf(__fmul_rn(x, inv_ln2));
+  const int k = static_cast<int>(kf);
+  float r = __fsub_rn(x, __fmul_rn(kf, ln2_hi));
+  r = __fsub_rn(r, __fmul_rn(kf, ln2_lo));
+  float p = 1.98412701138295233249664306640625e-04f;           // 1/7!
+  p = __fadd_rn(__fmul_rn(p, r), 1.388888922519981861114501953125e-03f);   // 1/6!
+  p = __fadd_rn(__fmul_rn(p, r), 8.333333767950534820556640625e-03f);      // 1/5!
+  p = __fadd_rn(__fmul_rn(p, r), 4.16666679084300994873046875e-02f);       // 1/4!
+  p = __fadd_rn(__fmul_rn(p, r), 1.6666667163372039794921875e-01f);        // 1/3!
+  p = __fadd_rn(__fmul_rn(p, r), 0.5f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  const int k1 = k >> 1;
+  const int k2 = k - k1;
+  return __fmul_rn(__fmul_rn(p, pow2i(k1)), pow2i(k2));
+}
+
+__device__ __forceinline__ float sigmoid_cw(float x) {
+  return __fdiv_rn(1.0f, __fadd_rn(1.0f, exp_cw(-x)));
+}
+
+// Frontier-Progress Score S = F * P (Eq. 6-8) from the two latest
+// confidences; hist = number of observations available.
+__device__ float fps(float c1, float c2, int hist, float theta, float w,
+                     float v_ref, float tau) {
+  const float v = hist >= 2 ? __fsub_rn(c1, c2) : 0.0f;
+  const float half_w = __fmul_rn(w, 0.5f);
+  const float vbar = fminf(fmaxf(v, -half_w), half_w);
+  const float chat = fminf(fmaxf(__fadd_rn(c1, vbar), 0.0f), 1.0f);
+  const float x1 = __fdiv_rn(__fadd_rn(__fsub_rn(chat, theta), w), tau);
+  const float x2 = __fdiv_rn(__fsub_rn(theta, chat), tau);
+  const float F = __fmul_rn(sigmoid_cw(x1), sigmoid_cw(x2));
+  const float P =
+      hist >= 2 ? sigmoid_cw(__fdiv_rn(__fsub_rn(v_ref, vbar), tau)) : 1.0f;
+  return __fmul_rn(F, P);
+}
+
+__device__ __forceinline__ int role_count(int dist, int k_base, int d_role) {
+  return dist <= 1 ? k_base + d_role : (dist == 2 ? k_base : k_base - d_role);
+}
+
+__device__ __forceinline__ int clip(int k, int lo, int hi) {
+  return k < lo ? lo : (k > hi ? hi : k);
+}
+
+__global__ void __launch_bounds__(kThreads)
+    budget_kernel(const float* __restrict__ conf1,
+                  const float* __restrict__ conf2,
+                  const uint8_t* __restrict__ hist_len,
+                  const uint8_t* __restrict__ masked,
+                  const int32_t* __restrict__ block_id,
+                  const int32_t* __restrict__ seq_off,
+                  const int32_t* __restrict__ active_block, int T, AllocArgs a,
+                  int32_t* __restrict__ k_out,
+                  unsigned long long* __restrict__ k_sum,
+                  uint32_t* __restrict__ err) {
+  __shared__ float s_score[kMaxJ];
+  __shared__ int32_t s_tok[kMaxJ];
+  __shared__ int s_nj;
+  __shared__ unsigned long long s_sum;
+  const int s = blockIdx.x;
+  const int lo = seq_off[s], hi = seq_off[s + 1];
+  if (lo < 0 || hi > T || lo > hi) {  // malformed offsets: touch nothing
+    if (threadIdx.x == 0) set_err(err, kErrIndex);
+    return;
+  }
+  int act = active_block[s];
+  if (threadIdx.x == 0) {
+    s_nj = 0;
+    s_sum = 0ull;
+    if (act < 1) set_err(err, kErrActive);
+  }
+  __syncthreads();
+  const int k_cur = a.k_base + a.delta_role;
+  unsigned long long my_sum = 0;
+  // pass 1: role counts (Eq. 5) and J_h membership with scores (Eq. 6-8)
+  for (int i = lo + threadIdx.x; i < hi; i += kThreads) {
+    const int b = block_id[i];
+    const int dist = act >= 1 ? abs(b - act) : 3;
+    int k = role_count(dist, a.k_base, a.delta_role);
+    const bool in_j = act >= 1 && b == act && masked[i] != 0 && hist_len[i] >= 1;
+    if (in_j) {
+      const int slot = atomicAdd(&s_nj, 1);
+      if (slot < kMaxJ) {
+        s_tok[slot] = i;
+        s_score[slot] = fps(conf1[i], conf2[i], hist_len[i], a.theta, a.w_cf,
+                            a.v_ref, a.tau);
+        continue;  // written in pass 2
+      }
+      k = k_cur;  // over capacity: keeps K_cur (error flagged below)
+    }
+    k = clip(k, a.k_min, a.k_max);
+    k_out[i] = k;
+    my_sum += static_cast<unsigned long long>(k);
+  }
+  __syncthreads();
+  const int nj_all = s_nj;
+  const int nj = nj_all < kMaxJ ? nj_all : kMaxJ;
+  if (nj_all > kMaxJ) {
+    // too many to rank: every stored member keeps K_cur too
+    if (threadIdx.x == 0) set_err(err, kErrCapacity);
+    for (int m = threadIdx.x; m < nj; m += kThreads) {
+      const int k = clip(k_cur, a.k_min, a.k_max);
+      k_out[s_tok[m]] = k;
+      my_sum += static_cast<unsigned long long>(k);
+    }
+  } else {
+    // pass 2: Eq. 9 groups from the rank of each member
+    const int n = static_cast<int>(floorf(__fmul_rn(a.q, static_cast<float>(nj))));
+    for (int m = threadIdx.x; m < nj; m += kThreads) {
+      const float sm = s_score[m];
+      const int tm = s_tok[m];
+      int rank = 0;
+      for (int j = 0; j < nj; ++j) {
+        const float sj = s_score[j];
+        rank += (sj > sm || (sj == sm && s_tok[j] < tm)) ? 1 : 0;
+      }
+      int k = k_cur;
+      if (rank < n)
+        k = k_cur + a.delta_cur;
+      else if (rank >= nj - n)
+        k = k_cur - a.delta_cur;
+      k = clip(k, a.k_min, a.k_max);
+      k_out[tm] = k;
+      my_sum += static_cast<unsigned long long>(k);
+    }
+  }
+  if (k_sum != nullptr) {
+    // warp sums, then one shared atomic per warp and one global per block
+    for (int o = 16; o > 0; o >>= 1) my_sum += __shfl_xor_sync(0xffffffffu, my_sum, o);
+    if ((threadIdx.x & 31) == 0) atomicAdd(&s_sum, my_sum);
+    __syncthreads();
+    if (threadIdx.x == 0) atomicAdd(k_sum, s_sum);
+  }
+}
+
+__global__ void wait_selftest_kernel(uint32_t* err, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  // nobody arrives: the wait must give up after limit_ns and report it
+  if (threadIdx.x == 0) {
+    if (!mbar_wait(&bar, 0, nullptr, limit_ns)) set_err(err, kErrTimeout);
+  }
+  __syncthreads();
+}
+
+}  // namespace
+
+cudaError_t launch_budget(const float* conf1, const float* conf2,
+                          const uint8_t* hist_len, const uint8_t* masked,
+                          const int32_t* block_id, const int32_t* seq_off,
+                          const int32_t* active_block, int T, int B,
+                          const AllocArgs& a, int32_t* k_out,
+                          unsigned long long* k_sum, uint32_t* err,
+                          cudaStream_t stream) {
+  if (B <= 0) return cudaSuccess;
+  budget_kernel<<<B, kThreads, 0, stream>>>(conf1, conf2, hist_len, masked,
+                                            block_id, seq_off, active_block, T, a,
+                                            k_out, k_sum, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_selftest(uint32_t* err, uint64_t limit_ns,
+                                 cudaStream_t stream) {
+  wait_selftest_kernel<<<1, 32, 0, stream>>>(err, limit_ns);
+  return cudaGetLastError();
+}
+
+}  // namespace rx

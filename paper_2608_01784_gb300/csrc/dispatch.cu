@@ -1,0 +1,218 @@
+// dispatch.cu — deterministic token-expert pair compaction for the sparse
+// execution of Eq. 2 (REFLEX Sec. 3.2): the pairs (t, j), j < k_t, are laid
+// out grouped by expert and, within an expert, in token order, so that each
+// expert's rows form one contiguous range of a grouped GEMM.
+//
+// Three launches, no atomics whose order matters:
+//   count   per block of 256 tokens, a bitmask per expert in shared memory
+//           (bit = token of the block selected the expert; a token selects
+//           an expert at most once) and its popcount per expert;
+//   scan    per expert, exclusive prefix over blocks; per-expert totals;
+//           exclusive prefix over experts = offsets, and over the 128-row
+//           tile counts = tile prefix for the grouped GEMM;
+//   scatter rebuilds the block's masks; the row of pair (t, j) is
+//           offsets[e] + block prefix + popcount of lower tokens' bits.
+// A fourth launch gathers X rows into pair order (one warp per pair row,
+// 16-byte vectors).
+#include "common.cuh"
+#include "internal.h"
+
+namespace rx {
+namespace {
+
+constexpr int kBlk = kDispatchBlock;  // tokens per block (8 mask words)
+constexpr int kWords = kBlk / 32;
+
+__device__ __forceinline__ int clamp_k(int kt, int kcap) {
+  return kt < 1 ? 1 : (kt > kcap ? kcap : kt);
+}
+
+__device__ void build_masks(uint32_t* mask, const int32_t* ids,
+                            const int32_t* k, int T, int E, int k_max,
+                            uint32_t* err) {
+  for (int i = threadIdx.x; i < E * kWords; i += kBlk) mask[i] = 0u;
+  __syncthreads();
+  const int t = blockIdx.x * kBlk + threadIdx.x;
+  if (t < T) {
+    const int kt = clamp_k(k[t], k_max < E ? k_max : E);
+    for (int j = 0; j < kt; ++j) {
+      const int e = ids[static_cast<int64_t>(t) * k_max + j];
+      if (e >= 0 && e < E)
+        atomicOr(&mask[e * kWords + (threadIdx.x >> 5)], 1u << (threadIdx.x & 31));
+      else
+        set_err(err, kErrIndex);
+    }
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(kBlk)
+    count_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ k,
+                 int T, int E, int k_max, int32_t* __restrict__ blk_count,
+                 uint32_t* __restrict__ err) {
+  extern __shared__ uint32_t mask[];
+  build_masks(mask, ids, k, T, E, k_max, err);
+  for (int e = threadIdx.x; e < E; e += kBlk) {
+    int c = 0;
+#pragma unroll
+    for (int w = 0; w < kWords; ++w) c += __popc(mask[e * kWords + w]);
+    blk_count[static_cast<int64_t>(blockIdx.x) * E + e] = c;
+  }
+}
+
+// Exclusive scan of one value per thread over a block of 1024 threads.
+__device__ int block_exclusive_scan(int v, int* s_warp, int* total) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) s_warp[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    int s = s_warp[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, s, o);
+      if (lane >= o) s += y;
+    }
+    s_warp[lane] = s;  // inclusive prefix of warp totals
+  }
+  __syncthreads();
+  const int before = wid > 0 ? s_warp[wid - 1] : 0;
+  *total = s_warp[31];
+  __syncthreads();
+  return before + x - v;
+}
+
+__global__ void __launch_bounds__(1024)
+    scan_kernel(const int32_t* __restrict__ blk_count, int nblk, int E,
+                int32_t* __restrict__ blk_off, int32_t* __restrict__ counts,
+                int32_t* __restrict__ offsets, int32_t* __restrict__ mt_prefix,
+                int32_t* __restrict__ totals) {
+  __shared__ int s_warp[32];
+  const int e = threadIdx.x;  // E <= 1024
+  int run = 0;
+  if (e < E) {
+    for (int b = 0; b < nblk; ++b) {
+      const int64_t o = static_cast<int64_t>(b) * E + e;
+      blk_off[o] = run;
+      run += blk_count[o];
+    }
+    counts[e] = run;
+  }
+  int total_pairs, total_tiles;
+  const int off = block_exclusive_scan(e < E ? run : 0, s_warp, &total_pairs);
+  const int tiles = e < E ? (run + kTileM - 1) / kTileM : 0;
+  const int toff = block_exclusive_scan(tiles, s_warp, &total_tiles);
+  if (e < E) {
+    offsets[e] = off;
+    mt_prefix[e] = toff;
+  }
+  if (e == 0) {
+    offsets[E] = total_pairs;
+    mt_prefix[E] = total_tiles;
+    totals[0] = total_pairs;
+    totals[1] = total_tiles;
+  }
+}
+
+__global__ void __launch_bounds__(kBlk)
+    scatter_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ k,
+                   int T, int E, int k_max,
+                   const int32_t* __restrict__ blk_off,
+                   const int32_t* __restrict__ offsets,
+                   int32_t* __restrict__ perm, int32_t* __restrict__ row_of,
+                   uint32_t* __restrict__ err) {
+  extern __shared__ uint32_t mask[];
+  build_masks(mask, ids, k, T, E, k_max, nullptr);
+  const int t = blockIdx.x * kBlk + threadIdx.x;
+  if (t >= T) return;
+  const int kt = clamp_k(k[t], k_max < E ? k_max : E);
+  const int w = threadIdx.x >> 5;
+  const uint32_t below = (1u << (threadIdx.x & 31)) - 1u;
+  for (int j = 0; j < k_max; ++j) {
+    const int64_t o = static_cast<int64_t>(t) * k_max + j;
+    int pos = -1;
+    if (j < kt) {
+      const int e = ids[o];
+      if (e >= 0 && e < E) {
+        int local = __popc(mask[e * kWords + w] & below);
+        for (int ww = 0; ww < w; ++ww) local += __popc(mask[e * kWords + ww]);
+        pos = offsets[e] + blk_off[static_cast<int64_t>(blockIdx.x) * E + e] + local;
+        perm[pos] = static_cast<int32_t>(o);
+      }
+    }
+    row_of[o] = pos;
+  }
+}
+
+template <typename Te>
+__global__ void __launch_bounds__(256)
+    gather_kernel(const Te* __restrict__ x, const int32_t* __restrict__ perm,
+                  const int32_t* __restrict__ totals, int k_max, int cap_rows,
+                  int T, int d, Te* __restrict__ xp, uint32_t* __restrict__ err) {
+  const int lane = threadIdx.x & 31;
+  int n = totals[0];
+  if (n > cap_rows) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) set_err(err, kErrIndex);
+    n = cap_rows;
+  }
+  const int warps = gridDim.x * 8;
+  for (int p = blockIdx.x * 8 + (threadIdx.x >> 5); p < n; p += warps) {
+    const int t = perm[p] / k_max;
+    if (t < 0 || t >= T) continue;
+    const Te* src = x + static_cast<int64_t>(t) * d;
+    Te* dst = xp + static_cast<int64_t>(p) * d;
+    float v[8];
+    for (int c = lane * 8; c < d; c += 256) {
+      load8(src + c, v);
+      store8(dst + c, v);
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T, int E,
+                            int k_max, const DispatchBufs& b,
+                            cudaStream_t stream) {
+  if (T == 0) return cudaSuccess;
+  const int nblk = (T + kBlk - 1) / kBlk;
+  const size_t smem = static_cast<size_t>(E) * kWords * sizeof(uint32_t);
+  if (smem > 48 * 1024) {
+    cudaError_t e1 = cudaFuncSetAttribute(count_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e2 = cudaFuncSetAttribute(scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e1 != cudaSuccess) return e1;
+    if (e2 != cudaSuccess) return e2;
+  }
+  count_kernel<<<nblk, kBlk, smem, stream>>>(ids, k, T, E, k_max, b.blk_count, b.err);
+  scan_kernel<<<1, 1024, 0, stream>>>(b.blk_count, nblk, E, b.blk_off, b.counts,
+                                      b.offsets, b.mt_prefix, b.totals);
+  scatter_kernel<<<nblk, kBlk, smem, stream>>>(ids, k, T, E, k_max, b.blk_off,
+                                               b.offsets, b.perm, b.row_of, b.err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* perm,
+                               const int32_t* totals, int k_max, int cap_rows,
+                               int d, void* x_perm, int num_sms,
+                               cudaStream_t stream) {
+  if (cap_rows == 0) return cudaSuccess;
+  const int T = cap_rows / k_max;
+  int grid = (cap_rows + 7) / 8;
+  if (grid > 16 * num_sms) grid = 16 * num_sms;
+  if (dtype == 0)
+    gather_kernel<float><<<grid, 256, 0, stream>>>(
+        static_cast<const float*>(hidden), perm, totals, k_max, cap_rows, T, d,
+        static_cast<float*>(x_perm), nullptr);
+  else
+    gather_kernel<__nv_bfloat16><<<grid, 256, 0, stream>>>(
+        static_cast<const __nv_bfloat16*>(hidden), perm, totals, k_max,
+        cap_rows, T, d, static_cast<__nv_bfloat16*>(x_perm), nullptr);
+  return cudaGetLastError();
+}
+
+}  // namespace rx

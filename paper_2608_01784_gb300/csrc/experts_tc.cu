@@ -1,0 +1,478 @@
+// experts_tc.cu — grouped SwiGLU expert GEMMs over ragged per-expert row
+// ranges on the 5th-generation tensor cores (tcgen05.mma, accumulators in
+// TMEM, operands staged by TMA), for the sparse execution of Eq. 2 (REFLEX
+// Sec. 3.2).  Routed-expert work is 6 * d * inter FLOPs per selected pair
+// (Eq. 10), two thirds in the gate/up GEMM and one third in the down GEMM.
+//
+// Problem.  Rows of the pair-ordered input A are grouped by expert
+// (rows [offsets[e], offsets[e+1]) belong to expert e).  For each group:
+//   SwiGLU mode: out[r, c] = silu(A_r . Wg[e, c]) * (A_r . Wu[e, c])
+//   Down mode:   out[r, n] = A_r . Wd[e, n]
+// with every operand K-major bf16 and fp32 accumulation; out is bf16.
+//
+// Tiles.  An output tile is 128 rows (one m-tile of a group; rows past the
+// group's end are computed from the next rows or TMA zero fill and never
+// stored) by BN columns.  In SwiGLU mode the BN-row weight tile is the
+// BN/2 gate rows followed by the matching BN/2 up rows, loaded by two TMA
+// boxes, so one MMA chain yields gate and up side by side in TMEM and the
+// epilogue emits BN/2 activations.  Tiles are numbered expert-major, then
+// n-tile, then m-tile, so CTAs running at the same time share weight tiles
+// in L2.
+//
+// Kernel.  Persistent: one CTA per SM walks tiles blockIdx.x, +gridDim.x, ...
+//   warp 0     TMA producer: 4-stage ring of (A 128x64, B BNx64) bf16 tiles,
+//              128-byte swizzle, completion on a per-stage mbarrier;
+//   warp 1     allocates 2*BN TMEM columns (two accumulators) and issues
+//              tcgen05.mma (M=128, N=BN, K=16) from one thread; each stage
+//              is released with tcgen05.commit when its MMAs have read it;
+//   warps 2-5  epilogue: tcgen05.ld 32x32b of their TMEM lane quarter,
+//              SwiGLU or conversion, 16-byte stores; the accumulator is
+//              handed back through an mbarrier, so the epilogue of tile i
+//              overlaps the main loop of tile i+1.
+// Every wait is bounded (2 s); on expiry the CTA records the timeout in the
+// error word, drains its outstanding TMA loads and MMAs, frees TMEM and
+// exits.
+#include "common.cuh"
+#include "internal.h"
+
+namespace rx {
+namespace {
+
+constexpr int BM = kTileM;   // 128
+constexpr int BK = 64;       // 64 bf16 = 128 bytes = one swizzle row
+constexpr int UMMA_K = 16;
+constexpr int kStages = 4;
+constexpr int kThreads = 192;
+constexpr int BN_SWIGLU = 256;  // 128 gate + 128 up -> 128 activations
+constexpr int BN_DOWN = 256;
+constexpr uint64_t kWaitNs = 2000000000ull;
+constexpr uint64_t kDrainNs = 1000000000ull;
+
+enum { kModeSwiGLU = 0, kModeDown = 1 };
+
+template <int BN>
+struct Cfg {
+  static constexpr int kABytes = BM * BK * 2;
+  static constexpr int kBBytes = BN * BK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kTmemCols = 2 * BN;
+  static constexpr int kBarBytes = 256;
+  static constexpr int kSmemBytes = kStages * kStageBytes + kBarBytes + 1024;
+};
+
+struct KParams {
+  int K;
+  int n_tiles;           // column tiles per group
+  int b_rows_per_group;
+  int b_up_offset;
+  GroupRows g;
+  const int32_t* mt_prefix;  // [E+1] (grouped mode)
+  int max_mtiles;            // host upper bound of m-tiles
+  __nv_bfloat16* out;
+  int ldo;
+  uint32_t* err;
+};
+
+// ---- PTX wrappers ---------------------------------------------------------
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive1(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map,
+                                            int c0, int c1, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map))
+               : "memory");
+}
+// Shared-memory matrix descriptor: K-major tile with 128-byte swizzle, rows
+// of 128 bytes, 8-row groups 1024 bytes apart.
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr) {
+  uint64_t desc = static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);  // start
+  desc |= static_cast<uint64_t>(1) << 16;            // leading offset (unused)
+  desc |= static_cast<uint64_t>(1024 >> 4) << 32;    // stride offset
+  desc |= static_cast<uint64_t>(1) << 46;            // descriptor version
+  desc |= static_cast<uint64_t>(2) << 61;            // 128-byte swizzle
+  return desc;
+}
+// Instruction descriptor of kind::f16: bf16 A and B, fp32 accumulator,
+// both K-major, M = 128, N = n.
+__host__ __device__ constexpr uint32_t idesc_bf16(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) |
+         (static_cast<uint32_t>(n >> 3) << 17) |
+         (static_cast<uint32_t>(BM >> 4) << 24);
+}
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t da,
+                                         uint64_t db, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(tmem_d),
+      "l"(da), "l"(db), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr),
+               "r"(ncols)
+               : "memory");
+}
+// 32 TMEM lanes x 32 consecutive fp32 columns: one column per register.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, "
+      "[%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+        "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
+        "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]),
+        "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// ---- tile numbering -------------------------------------------------------
+struct Tile {
+  int e, n, row0, rows;
+};
+
+__device__ __forceinline__ int total_tiles(const KParams& p) {
+  int mt;
+  if (p.g.offsets == nullptr) {
+    mt = (p.g.dense_rows + BM - 1) / BM;
+  } else {
+    mt = p.mt_prefix[p.g.E];
+    if (mt < 0) mt = 0;
+    if (mt > p.max_mtiles) mt = p.max_mtiles;
+  }
+  return mt * p.n_tiles;
+}
+
+// Tile t -> (expert, n-tile, rows); false when the workspace is inconsistent.
+__device__ __forceinline__ bool decode_tile(const KParams& p, int t, Tile& o) {
+  if (p.g.offsets == nullptr) {
+    const int mt = (p.g.dense_rows + BM - 1) / BM;
+    o.e = 0;
+    o.n = t / mt;
+    o.row0 = (t % mt) * BM;
+    o.rows = min(BM, p.g.dense_rows - o.row0);
+    return true;
+  }
+  int lo = 0, hi = p.g.E;  // n_tiles*prefix[lo] <= t < n_tiles*prefix[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (p.n_tiles * p.mt_prefix[mid] <= t) lo = mid; else hi = mid;
+  }
+  const int mt_e = p.mt_prefix[lo + 1] - p.mt_prefix[lo];
+  if (mt_e <= 0) return false;
+  const int l = t - p.n_tiles * p.mt_prefix[lo];
+  o.e = lo;
+  o.n = l / mt_e;
+  o.row0 = p.g.offsets[lo] + (l % mt_e) * BM;
+  o.rows = min(BM, p.g.offsets[lo + 1] - o.row0);
+  return o.n < p.n_tiles && o.row0 >= 0 && o.rows > 0 &&
+         o.row0 + o.rows <= p.g.cap_rows;
+}
+
+template <int BN, int MODE>
+__global__ void __launch_bounds__(kThreads, 1)
+    grouped_gemm_kernel(const __grid_constant__ CUtensorMap map_a,
+                        const __grid_constant__ CUtensorMap map_b,
+                        const KParams p) {
+  using C = Cfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* sa = smem;
+  uint8_t* sb = smem + kStages * C::kABytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * C::kStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + kStages;
+  uint64_t* acc_full = bars + 2 * kStages;
+  uint64_t* acc_empty = bars + 2 * kStages + 2;
+  uint64_t* drain = bars + 2 * kStages + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 4);  // one arrival per epilogue warp
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_map(&map_a);
+    prefetch_map(&map_b);
+  }
+  if (warp == 1) tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int ntiles = total_tiles(p);
+  const int nk = p.K / BK;
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer ----------------
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t issued_mask = 0, issued_phase = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+      Tile tl;
+      if (!decode_tile(p, t, tl)) {
+        set_err(p.err, kErrIndex);
+        *abort_flag = 1;
+        break;
+      }
+      for (int kb = 0; kb < nk; ++kb) {
+        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitNs)) {
+          ok = false;
+          break;
+        }
+        const uint32_t fb = smem_addr(&full[stage]);
+        mbar_expect_tx(fb, C::kStageBytes);
+        const int k0 = kb * BK;
+        tma_load_2d(smem_addr(sa + stage * C::kABytes), &map_a, k0, tl.row0, fb);
+        const uint32_t b_dst = smem_addr(sb + stage * C::kBBytes);
+        if (MODE == kModeSwiGLU) {
+          const int r = tl.e * p.b_rows_per_group + tl.n * (BN / 2);
+          tma_load_2d(b_dst, &map_b, k0, r, fb);
+          tma_load_2d(b_dst + (BN / 2) * BK * 2, &map_b, k0, r + p.b_up_offset, fb);
+        } else {
+          tma_load_2d(b_dst, &map_b, k0, tl.e * p.b_rows_per_group + tl.n * BN, fb);
+        }
+        issued_mask |= 1u << stage;
+        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    if (!ok) {
+      set_err(p.err, kErrTimeout);
+      *abort_flag = 1;
+    }
+    if (*abort_flag) {
+      // every issued load must land before the CTA may exit
+      for (int s = 0; s < kStages; ++s)
+        if (issued_mask & (1u << s))
+          mbar_wait(&full[s], (issued_phase >> s) & 1u, nullptr, kDrainNs);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer ----------------
+    constexpr uint32_t idesc = idesc_bf16(BN);
+    int stage = 0;
+    uint32_t phase = 0;
+    int lt = 0;
+    bool ok = true, issued_any = false;
+    for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++lt) {
+      const int ab = lt & 1;
+      const uint32_t acc_phase = (lt >> 1) & 1;
+      if (!mbar_wait(&acc_empty[ab], acc_phase ^ 1u, abort_flag, kWaitNs)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(ab * BN);
+      for (int kb = 0; kb < nk; ++kb) {
+        if (!mbar_wait(&full[stage], phase, abort_flag, kWaitNs)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a0 = smem_addr(sa + stage * C::kABytes);
+        const uint32_t b0 = smem_addr(sb + stage * C::kBBytes);
+#pragma unroll
+        for (int k = 0; k < BK / UMMA_K; ++k) {
+          mma_bf16(d_tmem, desc_sw128(a0 + k * UMMA_K * 2),
+                   desc_sw128(b0 + k * UMMA_K * 2), idesc,
+                   (kb > 0 || k > 0) ? 1u : 0u);
+        }
+        issued_any = true;
+        mma_commit(smem_addr(&empty[stage]));
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (!ok) break;
+      mma_commit(smem_addr(&acc_full[ab]));
+    }
+    if (!ok) {
+      set_err(p.err, kErrTimeout);
+      *abort_flag = 1;
+    }
+    if (*abort_flag && issued_any) {
+      // MMAs in flight must finish before TMEM is freed
+      mma_commit(smem_addr(drain));
+      mbar_wait(drain, 0, nullptr, kDrainNs);
+    }
+  } else if (warp >= 2) {
+    // ---------------- epilogue ----------------
+    const int quarter = warp & 3;  // TMEM lanes 32*quarter .. +31
+    const int row = quarter * 32 + lane;
+    int lt = 0;
+    for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++lt) {
+      Tile tl;
+      const bool tile_ok = decode_tile(p, t, tl);
+      const int ab = lt & 1;
+      const uint32_t acc_phase = (lt >> 1) & 1;
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&acc_full[ab], acc_phase, abort_flag, kWaitNs) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) {
+        if (lane == 0) {
+          if (!*abort_flag) set_err(p.err, kErrTimeout);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                             static_cast<uint32_t>(ab * BN);
+      const bool store = tile_ok && row < tl.rows;
+      __nv_bfloat16* orow =
+          p.out + static_cast<int64_t>(tl.row0 + (store ? row : 0)) * p.ldo;
+      if (MODE == kModeSwiGLU) {
+#pragma unroll 1
+        for (int c = 0; c < BN / 2; c += 32) {
+          uint32_t g[32], u[32];
+          tmem_ld32(tbase + c, g);
+          tmem_ld32(tbase + BN / 2 + c, u);
+          tmem_ld_wait();
+          if (store) {
+            uint32_t packed[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+              const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+              const float a0 = g0 / (1.0f + __expf(-g0)) * u0;
+              const float a1 = g1 / (1.0f + __expf(-g1)) * u1;
+              __nv_bfloat162 h2 = __floats2bfloat162_rn(a0, a1);
+              packed[i] = *reinterpret_cast<uint32_t*>(&h2);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(orow + tl.n * (BN / 2) + c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              dst[v] = make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
+                                  packed[4 * v + 3]);
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t v32[32];
+          tmem_ld32(tbase + c, v32);
+          tmem_ld_wait();
+          if (store) {
+            uint32_t packed[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              __nv_bfloat162 h2 = __floats2bfloat162_rn(__uint_as_float(v32[2 * i]),
+                                                        __uint_as_float(v32[2 * i + 1]));
+              packed[i] = *reinterpret_cast<uint32_t*>(&h2);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(orow + tl.n * BN + c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              dst[v] = make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
+                                  packed[4 * v + 3]);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive1(smem_addr(&acc_empty[ab]));
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem_base, C::kTmemCols);
+  }
+}
+
+template <int BN, int MODE>
+cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
+  using C = Cfg<BN>;
+  auto kernel = grouped_gemm_kernel<BN, MODE>;
+  cudaError_t e = cudaFuncSetAttribute(
+      kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  KParams p;
+  p.K = a.K;
+  p.n_tiles = MODE == kModeSwiGLU ? a.n_total / (BN / 2) : a.n_total / BN;
+  p.b_rows_per_group = a.b_rows_per_group;
+  p.b_up_offset = a.b_up_offset;
+  p.g = a.g;
+  p.max_mtiles = a.g.offsets ? (a.g.cap_rows + BM - 1) / BM + a.g.E
+                             : (a.g.dense_rows + BM - 1) / BM;
+  p.out = static_cast<__nv_bfloat16*>(a.out);
+  p.ldo = a.ldo;
+  p.err = a.err;
+  p.mt_prefix = a.g.mt_prefix;
+  const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
+  if (max_tiles == 0) return cudaSuccess;
+  const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);
+  kernel<<<grid, kThreads, C::kSmemBytes, stream>>>(*a.map_a, *a.map_b, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_swiglu_tc(const TcGemmArgs& a, cudaStream_t stream) {
+  return launch_impl<BN_SWIGLU, kModeSwiGLU>(a, stream);
+}
+cudaError_t launch_down_tc(const TcGemmArgs& a, cudaStream_t stream) {
+  return launch_impl<BN_DOWN, kModeDown>(a, stream);
+}
+int tc_swiglu_b_box_rows() { return BN_SWIGLU / 2; }
+int tc_down_b_box_rows() { return BN_DOWN; }
+int tc_swiglu_n_granule() { return BN_SWIGLU / 2; }
+int tc_down_n_granule() { return BN_DOWN; }
+
+}  // namespace rx

@@ -1,0 +1,110 @@
+// internal.h — launchers shared between the kernel files and the C-ABI host
+// code (reflex_abi.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace rx {
+
+struct AllocArgs {
+  int k_min, k_base, k_max, delta_role, delta_cur;
+  float q, theta, w_cf, v_ref, tau;
+};
+
+// ---- allocation (budget.cu) -----------------------------------------------
+cudaError_t launch_budget(const float* conf1, const float* conf2,
+                          const uint8_t* hist_len, const uint8_t* masked,
+                          const int32_t* block_id, const int32_t* seq_off,
+                          const int32_t* active_block, int T, int B,
+                          const AllocArgs& a, int32_t* k_out,
+                          unsigned long long* k_sum, uint32_t* err,
+                          cudaStream_t stream);
+cudaError_t launch_wait_selftest(uint32_t* err, uint64_t limit_ns,
+                                 cudaStream_t stream);
+
+// ---- routing (router.cu) --------------------------------------------------
+// z[T, E] = router scores (sequential fp32 fma chain over the hidden index).
+cudaError_t launch_router_logits(int dtype, const void* hidden,
+                                 const void* w_router, int T, int d, int E,
+                                 float* z, int num_sms, cudaStream_t stream);
+// ids/alpha [T, k_max] from z and the counts k.
+cudaError_t launch_router_select(const float* z, const int32_t* k, int T,
+                                 int E, int k_max, bool renorm, int32_t* ids,
+                                 float* alpha, uint32_t* err,
+                                 cudaStream_t stream);
+
+// ---- dispatch (dispatch.cu) -----------------------------------------------
+struct DispatchBufs {
+  int32_t* blk_count;  // [nblk, E]
+  int32_t* blk_off;    // [nblk, E]
+  int32_t* counts;     // [E]
+  int32_t* offsets;    // [E+1]
+  int32_t* mt_prefix;  // [E+1]
+  int32_t* perm;       // [T*k_max]
+  int32_t* row_of;     // [T*k_max]
+  int32_t* totals;     // header: total_pairs, total_mtiles
+  uint32_t* err;
+};
+constexpr int kDispatchBlock = 256;  // tokens per dispatch block
+cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T,
+                            int E, int k_max, const DispatchBufs& b,
+                            cudaStream_t stream);
+// X_perm[p] = X[perm[p] / k_max] for p < total_pairs.
+cudaError_t launch_gather_rows(int dtype, const void* hidden,
+                               const int32_t* perm, const int32_t* totals,
+                               int k_max, int cap_rows, int d, void* x_perm,
+                               int num_sms, cudaStream_t stream);
+
+// ---- experts: SIMT grouped GEMMs (experts_simt.cu) ------------------------
+// Grouped mode: rows [offsets[e], offsets[e+1]) use expert e; dense mode
+// (offsets == nullptr): rows [0, dense_rows) use the single weight set.
+struct GroupRows {
+  const int32_t* offsets;    // [E+1] or nullptr
+  const int32_t* mt_prefix;  // [E+1] prefix of 128-row tile counts
+  const int32_t* totals;     // device total rows (grouped mode)
+  int E;
+  int dense_rows;
+  int cap_rows;
+};
+cudaError_t launch_swiglu_simt(int dtype, const void* x, const void* w_gate_up,
+                               int d, int inter, const GroupRows& g, void* act,
+                               uint32_t* err, cudaStream_t stream);
+cudaError_t launch_down_simt(int dtype, const void* act, const void* w_down,
+                             int d, int inter, const GroupRows& g, void* y,
+                             uint32_t* err, cudaStream_t stream);
+
+// ---- experts: tcgen05 grouped GEMMs (experts_tc.cu) -----------------------
+struct TcGemmArgs {
+  const CUtensorMap* map_a;  // A [rows, K] bf16, box {64, 128}, 128B swizzle
+  const CUtensorMap* map_b;  // B [groups * rows_per_group, K] bf16
+  int K;                     // reduction length
+  int n_total;               // output columns per group (SwiGLU: inter)
+  int b_rows_per_group;      // SwiGLU: 2*inter, down: d
+  int b_up_offset;           // SwiGLU: inter (row offset of up weights)
+  GroupRows g;               // row groups
+  void* out;                 // [rows, ldo] bf16
+  int ldo;
+  uint32_t* err;
+  int num_sms;
+};
+// SwiGLU: out = silu(A Wg^T) * (A Wu^T).  Down: out = A Wd^T.
+cudaError_t launch_swiglu_tc(const TcGemmArgs& a, cudaStream_t stream);
+cudaError_t launch_down_tc(const TcGemmArgs& a, cudaStream_t stream);
+// Box rows of the B operand each kernel expects in its tensor map.
+int tc_swiglu_b_box_rows();
+int tc_down_b_box_rows();
+int tc_swiglu_n_granule();  // inter must be a multiple of this
+int tc_down_n_granule();    // d must be a multiple of this
+
+// ---- combine (combine.cu) -------------------------------------------------
+// out[t] = sum_{j<k_t} alpha[t,j] * y[row_of[t,j]] (+ y_shared[t]).
+cudaError_t launch_combine(int dtype, const void* y, const void* y_shared,
+                           const int32_t* row_of, const float* alpha,
+                           const int32_t* k, int T, int d, int k_max,
+                           int cap_rows, void* out, uint32_t* err, int num_sms,
+                           cudaStream_t stream);
+
+}  // namespace rx

@@ -1,0 +1,354 @@
+// reflex_abi.cu — the C ABI of include/reflex.h: argument checks, workspace
+// carving, tensor-map construction and the launch sequence of one
+// allocation call and one MoE-layer forward.  No allocation, no host sync
+// (except the explicit status readers).
+#include <cudaTypedefs.h>
+
+#include <cstring>
+#include <mutex>
+
+#include "common.cuh"
+#include "internal.h"
+#include "reflex.h"
+
+namespace {
+
+using rx::WsHeader;
+
+constexpr size_t kAlign = 256;
+size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+// Byte offsets of every workspace region (all 256-byte aligned).
+struct Layout {
+  size_t hdr, z, ids, alpha, blk_count, blk_off, counts, offsets, mt_prefix,
+      perm, row_of, xperm, amid, ash, ysh, total;
+  int64_t cap_rows;
+  int nblk;
+};
+
+bool shapes_ok(int32_t dtype, int32_t T, int32_t d, int32_t E, int32_t inter,
+               int32_t shared_inter, int32_t k_max) {
+  if (dtype != REFLEX_DTYPE_F32 && dtype != REFLEX_DTYPE_BF16) return false;
+  if (T < 0 || d <= 0 || d % 64 != 0 || E < 1 || E > 1024) return false;
+  if (inter <= 0 || inter % 64 != 0) return false;
+  if (shared_inter < 0 || shared_inter % 64 != 0) return false;
+  if (k_max < 1 || k_max > 32) return false;
+  if (static_cast<int64_t>(T) * k_max > (int64_t{1} << 30)) return false;
+  return true;
+}
+
+Layout make_layout(int32_t dtype, int32_t T, int32_t d, int32_t E,
+                   int32_t inter, int32_t shared_inter, int32_t k_max) {
+  Layout L{};
+  const size_t es = dtype == REFLEX_DTYPE_F32 ? 4 : 2;
+  const int64_t cap = static_cast<int64_t>(T) * k_max;
+  const int nblk = (T + rx::kDispatchBlock - 1) / rx::kDispatchBlock;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o += up(bytes);
+    return at;
+  };
+  L.hdr = take(sizeof(WsHeader));
+  L.z = take(static_cast<size_t>(T) * E * 4);
+  L.ids = take(cap * 4);
+  L.alpha = take(cap * 4);
+  L.blk_count = take(static_cast<size_t>(nblk) * E * 4);
+  L.blk_off = take(static_cast<size_t>(nblk) * E * 4);
+  L.counts = take(static_cast<size_t>(E) * 4);
+  L.offsets = take(static_cast<size_t>(E + 1) * 4);
+  L.mt_prefix = take(static_cast<size_t>(E + 1) * 4);
+  L.perm = take(cap * 4);
+  L.row_of = take(cap * 4);
+  L.xperm = take(cap * d * es);  // later reused for the expert outputs y
+  L.amid = take(cap * inter * es);
+  L.ash = shared_inter ? take(static_cast<size_t>(T) * shared_inter * es) : 0;
+  L.ysh = shared_inter ? take(static_cast<size_t>(T) * d * es) : 0;
+  L.total = o;
+  L.cap_rows = cap;
+  L.nblk = nblk;
+  return L;
+}
+
+int num_sms_current() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (dev >= 0 && dev < 64 && cached[dev] > 0) return cached[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    n = 148;
+  if (dev >= 0 && dev < 64) cached[dev] = n;
+  return n;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 map over a row-major [rows, cols] matrix; box = 64 columns (128
+// bytes, one swizzle row) x box_rows rows, 128-byte swizzle, zero fill.
+bool make_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols,
+              int box_rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) != 0) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
+  cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base),
+                  dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int map_err_bits(uint32_t bits) {
+  if (bits == 0) return REFLEX_OK;
+  if (bits & rx::kErrTimeout) return REFLEX_ETIMEOUT;
+  if (bits & rx::kErrKRange) return REFLEX_EKRANGE;
+  if (bits & rx::kErrCapacity) return REFLEX_ECAPACITY;
+  return REFLEX_EINVAL;
+}
+
+#define RX_CUDA(x)                                  \
+  do {                                              \
+    if ((x) != cudaSuccess) return REFLEX_ECUDA;    \
+  } while (0)
+
+}  // namespace
+
+extern "C" {
+
+int reflex_abi_version(void) { return 100; }
+
+const char* reflex_status_string(int s) {
+  switch (s) {
+    case REFLEX_OK: return "ok";
+    case REFLEX_EINVAL: return "invalid argument";
+    case REFLEX_EKRANGE: return "expert count out of range";
+    case REFLEX_EWORKSPACE: return "workspace missing or too small";
+    case REFLEX_ECUDA: return "CUDA error";
+    case REFLEX_ETIMEOUT: return "bounded device wait expired";
+    case REFLEX_EUNSUPPORTED: return "shape not supported by the selected path";
+    case REFLEX_ECAPACITY: return "too many active-block tokens in a sequence";
+    default: return "unknown status";
+  }
+}
+
+void reflex_default_params(reflex_alloc_params* p) {
+  if (p == nullptr) return;
+  p->k_min = 2;
+  p->k_base = 8;
+  p->k_max = 12;
+  p->delta_role = 4;
+  p->delta_cur = 2;
+  p->q = 0.25f;
+  p->theta = 0.9f;
+  p->w_cf = 0.30f;
+  p->v_ref = 0.01f;
+  p->tau = 0.05f;
+}
+
+int reflex_allocate(const float* router_scores, const float* conf_prev1,
+                    const float* conf_prev2, const uint8_t* hist_len,
+                    const uint8_t* masked, const int32_t* block_id,
+                    const int32_t* seq_offsets, const int32_t* active_block,
+                    int32_t T, int32_t B, int32_t E,
+                    const reflex_alloc_params* p, int32_t* k_out,
+                    int64_t* k_sum_out, int32_t* dev_status, void* stream) {
+  (void)router_scores;  // the REFLEX count rule does not read router scores
+  (void)E;
+  if (p == nullptr || T < 0 || B < 1) return REFLEX_EINVAL;
+  if (T > 0 && (conf_prev1 == nullptr || conf_prev2 == nullptr ||
+                hist_len == nullptr || masked == nullptr ||
+                block_id == nullptr || k_out == nullptr))
+    return REFLEX_EINVAL;
+  if (seq_offsets == nullptr || active_block == nullptr) return REFLEX_EINVAL;
+  if (p->k_min < 1 || p->k_min > p->k_max || p->k_base < 1 ||
+      p->delta_role < 0 || p->delta_cur < 0)
+    return REFLEX_EINVAL;
+  if (!(p->q > 0.0f && p->q <= 0.5f) || !(p->w_cf > 0.0f) || !(p->tau > 0.0f))
+    return REFLEX_EINVAL;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint32_t* err = reinterpret_cast<uint32_t*>(dev_status);
+  if (err) RX_CUDA(cudaMemsetAsync(err, 0, sizeof(int32_t), s));
+  if (k_sum_out) RX_CUDA(cudaMemsetAsync(k_sum_out, 0, sizeof(int64_t), s));
+  rx::AllocArgs a{p->k_min, p->k_base,  p->k_max, p->delta_role, p->delta_cur,
+                  p->q,     p->theta,   p->w_cf,  p->v_ref,      p->tau};
+  RX_CUDA(rx::launch_budget(conf_prev1, conf_prev2, hist_len, masked, block_id,
+                            seq_offsets, active_block, T, B, a, k_out,
+                            reinterpret_cast<unsigned long long*>(k_sum_out),
+                            err, s));
+  return REFLEX_OK;
+}
+
+size_t reflex_moe_workspace_size(int32_t dtype, int32_t T, int32_t d,
+                                 int32_t E, int32_t inter,
+                                 int32_t shared_inter, int32_t k_max) {
+  if (!shapes_ok(dtype, T, d, E, inter, shared_inter, k_max)) return 0;
+  return make_layout(dtype, T, d, E, inter, shared_inter, k_max).total;
+}
+
+int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
+                       const void* w_gate_up, const void* w_down,
+                       const void* shared_gate_up, const void* shared_down,
+                       int32_t shared_inter, const int32_t* k, int32_t T,
+                       int32_t d, int32_t E, int32_t inter, int32_t k_max,
+                       uint32_t flags, void* workspace, size_t ws_bytes,
+                       void* out, reflex_route_record* rec, void* stream) {
+  if (!shapes_ok(dtype, T, d, E, inter, shared_inter, k_max)) return REFLEX_EINVAL;
+  if (shared_inter > 0 && (shared_gate_up == nullptr || shared_down == nullptr))
+    return REFLEX_EINVAL;
+  const Layout L = make_layout(dtype, T, d, E, inter, shared_inter, k_max);
+  if (workspace == nullptr || ws_bytes < L.total) return REFLEX_EWORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & (kAlign - 1)) != 0)
+    return REFLEX_EWORKSPACE;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(ws + L.hdr);
+  int32_t* totals = &hdr->total_pairs;
+  uint32_t* err = &hdr->err;
+  auto I32 = [&](size_t off) { return reinterpret_cast<int32_t*>(ws + off); };
+  if (rec != nullptr) {
+    rec->ids = I32(L.ids);
+    rec->alpha = reinterpret_cast<float*>(ws + L.alpha);
+    rec->counts = I32(L.counts);
+    rec->offsets = I32(L.offsets);
+    rec->perm = I32(L.perm);
+    rec->row_of = I32(L.row_of);
+    rec->totals = totals;
+  }
+  if (T == 0) return REFLEX_OK;
+  if (hidden == nullptr || w_router == nullptr || w_gate_up == nullptr ||
+      w_down == nullptr || k == nullptr || out == nullptr)
+    return REFLEX_EINVAL;
+
+  const bool simt = dtype == REFLEX_DTYPE_F32 || (flags & REFLEX_FLAG_SIMT_EXPERTS);
+  if (!simt) {
+    if (d % rx::tc_down_n_granule() != 0 || inter % rx::tc_swiglu_n_granule() != 0 ||
+        (shared_inter % rx::tc_swiglu_n_granule()) != 0)
+      return REFLEX_EUNSUPPORTED;
+    if (encode_fn() == nullptr) return REFLEX_ECUDA;
+  }
+  constexpr uint32_t kAllStages = REFLEX_STAGE_ROUTE | REFLEX_STAGE_DISPATCH |
+                                  REFLEX_STAGE_EXPERT_UP | REFLEX_STAGE_EXPERT_DOWN |
+                                  REFLEX_STAGE_COMBINE;
+  uint32_t stages = flags & kAllStages;
+  if (stages == 0) stages = kAllStages;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int sms = num_sms_current();
+  const int cap = static_cast<int>(L.cap_rows);
+  float* z = reinterpret_cast<float*>(ws + L.z);
+  float* alpha = reinterpret_cast<float*>(ws + L.alpha);
+  void* xperm = ws + L.xperm;  // gathered rows, then expert outputs y
+  void* amid = ws + L.amid;
+  void* ash = shared_inter ? ws + L.ash : nullptr;
+  void* ysh = shared_inter ? ws + L.ysh : nullptr;
+
+  if (stages & REFLEX_STAGE_ROUTE) {
+    RX_CUDA(cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s));
+    RX_CUDA(rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z, sms, s));
+    RX_CUDA(rx::launch_router_select(z, k, T, E, k_max,
+                                     (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
+                                     I32(L.ids), alpha, err, s));
+  }
+  if (stages & REFLEX_STAGE_DISPATCH) {
+    rx::DispatchBufs b{I32(L.blk_count), I32(L.blk_off), I32(L.counts),
+                       I32(L.offsets),   I32(L.mt_prefix), I32(L.perm),
+                       I32(L.row_of),    totals,          err};
+    RX_CUDA(rx::launch_dispatch(I32(L.ids), k, T, E, k_max, b, s));
+    RX_CUDA(rx::launch_gather_rows(dtype, hidden, I32(L.perm), totals, k_max,
+                                   cap, d, xperm, sms, s));
+  }
+  const bool up = (stages & REFLEX_STAGE_EXPERT_UP) != 0;
+  const bool down = (stages & REFLEX_STAGE_EXPERT_DOWN) != 0;
+  if (up || down) {
+    rx::GroupRows grouped{I32(L.offsets), I32(L.mt_prefix), totals, E, 0, cap};
+    rx::GroupRows dense{nullptr, nullptr, nullptr, 1, T, T};
+    if (simt) {
+      if (up) {
+        RX_CUDA(rx::launch_swiglu_simt(dtype, xperm, w_gate_up, d, inter, grouped, amid, err, s));
+        if (shared_inter)
+          RX_CUDA(rx::launch_swiglu_simt(dtype, hidden, shared_gate_up, d, shared_inter, dense, ash, err, s));
+      }
+      if (down) {
+        RX_CUDA(rx::launch_down_simt(dtype, amid, w_down, d, inter, grouped, xperm, err, s));
+        if (shared_inter)
+          RX_CUDA(rx::launch_down_simt(dtype, ash, shared_down, d, shared_inter, dense, ysh, err, s));
+      }
+    } else {
+      CUtensorMap ma1, mb1, ma2, mb2;
+      if (!make_map(&ma1, xperm, cap, d, rx::kTileM) ||
+          !make_map(&mb1, w_gate_up, static_cast<int64_t>(E) * 2 * inter, d,
+                    rx::tc_swiglu_b_box_rows()) ||
+          !make_map(&ma2, amid, cap, inter, rx::kTileM) ||
+          !make_map(&mb2, w_down, static_cast<int64_t>(E) * d, inter,
+                    rx::tc_down_b_box_rows()))
+        return REFLEX_ECUDA;
+      rx::TcGemmArgs g1{&ma1, &mb1, d, inter, 2 * inter, inter, grouped, amid, inter, err, sms};
+      rx::TcGemmArgs g2{&ma2, &mb2, inter, d, d, 0, grouped, xperm, d, err, sms};
+      CUtensorMap sa1, sb1, sa2, sb2;
+      if (shared_inter &&
+          (!make_map(&sa1, hidden, T, d, rx::kTileM) ||
+           !make_map(&sb1, shared_gate_up, 2 * static_cast<int64_t>(shared_inter), d,
+                     rx::tc_swiglu_b_box_rows()) ||
+           !make_map(&sa2, ash, T, shared_inter, rx::kTileM) ||
+           !make_map(&sb2, shared_down, d, shared_inter, rx::tc_down_b_box_rows())))
+        return REFLEX_ECUDA;
+      rx::TcGemmArgs h1{&sa1, &sb1, d, shared_inter, 2 * shared_inter, shared_inter,
+                        dense, ash, shared_inter, err, sms};
+      rx::TcGemmArgs h2{&sa2, &sb2, shared_inter, d, d, 0, dense, ysh, d, err, sms};
+      if (up) {
+        RX_CUDA(rx::launch_swiglu_tc(g1, s));
+        if (shared_inter) RX_CUDA(rx::launch_swiglu_tc(h1, s));
+      }
+      if (down) {
+        RX_CUDA(rx::launch_down_tc(g2, s));
+        if (shared_inter) RX_CUDA(rx::launch_down_tc(h2, s));
+      }
+    }
+  }
+  if (stages & REFLEX_STAGE_COMBINE) {
+    RX_CUDA(rx::launch_combine(dtype, xperm, ysh, I32(L.row_of), alpha, k, T, d,
+                               k_max, cap, out, err, sms, s));
+  }
+  return REFLEX_OK;
+}
+
+int reflex_read_status(const int32_t* dev_status, void* stream) {
+  if (dev_status == nullptr) return REFLEX_EINVAL;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint32_t bits = 0;
+  RX_CUDA(cudaMemcpyAsync(&bits, dev_status, sizeof(bits), cudaMemcpyDeviceToHost, s));
+  RX_CUDA(cudaStreamSynchronize(s));
+  return map_err_bits(bits);
+}
+
+int reflex_moe_status(const void* workspace, void* stream) {
+  if (workspace == nullptr) return REFLEX_EINVAL;
+  const WsHeader* hdr = static_cast<const WsHeader*>(workspace);
+  return reflex_read_status(reinterpret_cast<const int32_t*>(&hdr->err), stream);
+}
+
+int reflex_selftest_wait_timeout(int32_t* dev_status, uint32_t limit_us,
+                                 void* stream) {
+  if (dev_status == nullptr || limit_us < 1 || limit_us > 100000) return REFLEX_EINVAL;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  RX_CUDA(cudaMemsetAsync(dev_status, 0, sizeof(int32_t), s));
+  RX_CUDA(rx::launch_wait_selftest(reinterpret_cast<uint32_t*>(dev_status),
+                                   static_cast<uint64_t>(limit_us) * 1000ull, s));
+  return REFLEX_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,112 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds for
+sm_103a, exports every entry point include/reflex.h declares, and rejects bad
+arguments before anything is enqueued."""
+import ctypes
+import re
+import shutil
+from pathlib import Path
+
+import pytest
+
+ROOT = Path(__file__).resolve().parents[1]
+HEADER = ROOT / "include" / "reflex.h"
+
+pytestmark = pytest.mark.skipif(shutil.which("nvcc") is None and
+                                not Path("/usr/local/cuda/bin/nvcc").exists(),
+                                reason="needs nvcc to build the library")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_01784_gb300 import build, _binding
+    build.build()
+    return _binding.load()
+
+
+def declared_functions():
+    text = HEADER.read_text()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(reflex_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for must in ("reflex_allocate", "reflex_moe_forward",
+                 "reflex_moe_workspace_size", "reflex_moe_status"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    from paper_2608_01784_gb300 import _binding
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert name in _binding.EXPORTED, name
+
+
+def test_status_strings_and_version(lib):
+    from paper_2608_01784_gb300 import _binding as B
+    assert B.reflex_status_string(B.REFLEX_OK) == "ok"
+    assert "workspace" in B.reflex_status_string(B.REFLEX_EWORKSPACE)
+    assert B.reflex_status_string(999) == "unknown status"
+    assert B.reflex_abi_version() >= 100
+
+
+def test_default_params_are_the_paper_settings(lib):
+    from paper_2608_01784_gb300 import _binding as B
+    p = B.reflex_default_params()
+    assert (p.k_base, p.delta_role, p.delta_cur) == (8, 4, 2)
+    assert p.q == pytest.approx(0.25) and p.theta == pytest.approx(0.9)
+    assert p.v_ref == pytest.approx(0.01) and p.tau == pytest.approx(0.05)
+    assert p.w_cf == pytest.approx(0.30)
+
+
+def test_workspace_size(lib):
+    from paper_2608_01784_gb300 import _binding as B
+    ws = B.reflex_moe_workspace_size
+    a = ws(1, 1024, 2048, 64, 1024, 0, 12)
+    assert a > 1024 * 12 * 2048 * 2          # at least the gathered rows
+    assert ws(1, 2048, 2048, 64, 1024, 0, 12) > a
+    assert ws(1, 1024, 2048, 64, 1024, 512, 12) > a   # shared expert buffers
+    assert ws(0, 1024, 2048, 64, 1024, 0, 12) > a     # fp32 storage
+    assert ws(1, 1024, 2000, 64, 1024, 0, 12) == 0    # d % 64
+    assert ws(1, 1024, 2048, 0, 1024, 0, 12) == 0     # E >= 1
+    assert ws(1, 1024, 2048, 64, 1024, 0, 33) == 0    # k_max <= 32
+    assert ws(7, 1024, 2048, 64, 1024, 0, 12) == 0    # dtype
+
+
+def test_host_rejections_enqueue_nothing(lib):
+    from paper_2608_01784_gb300 import _binding as B
+    p = B.reflex_default_params()
+    # null parameter block / bad parameters
+    assert lib.reflex_allocate(None, None, None, None, None, None, None, None,
+                               4, 1, 8, None, None, None, None, None) == B.REFLEX_EINVAL
+    bad = B.make_params(q=0.7)
+    assert lib.reflex_allocate(None, 1, 1, 1, 1, 1, 1, 1, 4, 1, 8,
+                               ctypes.byref(bad), 1, None, None, None) == B.REFLEX_EINVAL
+    bad = B.make_params(k_min=5, k_max=4)
+    assert lib.reflex_allocate(None, 1, 1, 1, 1, 1, 1, 1, 4, 1, 8,
+                               ctypes.byref(bad), 1, None, None, None) == B.REFLEX_EINVAL
+    assert lib.reflex_allocate(None, 1, 1, 1, 1, 1, 1, 1, 4, 0, 8,
+                               ctypes.byref(p), 1, None, None, None) == B.REFLEX_EINVAL
+    # forward: bad shapes, missing workspace
+    fw = lib.reflex_moe_forward
+    assert fw(1, 1, 1, 1, 1, None, None, 0, 1, 4, 2000, 8, 128, 4, 1, 1, 1 << 30,
+              1, None, None) == B.REFLEX_EINVAL
+    assert fw(1, 1, 1, 1, 1, None, None, 0, 1, 4, 256, 8, 128, 4, 1, None, 0,
+              1, None, None) == B.REFLEX_EWORKSPACE
+    need = B.reflex_moe_workspace_size(1, 4, 256, 8, 128, 0, 4)
+    assert fw(1, 1, 1, 1, 1, None, None, 0, 1, 4, 256, 8, 128, 4, 1, 256,
+              need - 1, 1, None, None) == B.REFLEX_EWORKSPACE
+    # misaligned workspace
+    assert fw(1, 1, 1, 1, 1, None, None, 0, 1, 4, 256, 8, 128, 4, 1, 257,
+              need, 1, None, None) == B.REFLEX_EWORKSPACE
+    # shared expert declared without weights
+    assert fw(1, 1, 1, 1, 1, None, None, 128, 1, 4, 256, 8, 128, 4, 1, 256,
+              1 << 30, 1, None, None) == B.REFLEX_EINVAL
+    # T = 0 is a no-op that still fills the record
+    rec = B.reflex_route_record()
+    assert fw(1, None, None, None, None, None, None, 0, None, 0, 256, 8, 128, 4,
+              1, 256, 1 << 20, None, ctypes.byref(rec), None) == B.REFLEX_OK
+    assert rec.ids == 256 + 256          # first region after the header
+    assert lib.reflex_selftest_wait_timeout(None, 10, None) == B.REFLEX_EINVAL
+    assert lib.reflex_read_status(None, None) == B.REFLEX_EINVAL

@@ -1,0 +1,260 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle on the
+same seeded inputs.  Allocation, selected experts, pair offsets and the pair
+permutation must match bit for bit; router weights within 2e-5 relative;
+layer outputs within rel-L2 1e-2 / max-abs 2e-2 for bf16 storage with fp32
+accumulation (1e-5 / 1e-4 for fp32 storage)."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_01784_gb300 import _binding as B
+from paper_2608_01784_gb300 import api
+from paper_2608_01784_gb300 import workloads as W
+from tests import gpu_cases as G
+
+pytestmark = pytest.mark.gpu
+
+CFG = W.CONFIGS
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2608_01784_gb300 import build
+    build.build()
+    B.load()
+    oracle.build()
+
+
+# ---------------------------------------------------------------------------
+# bounded waits
+# ---------------------------------------------------------------------------
+def test_wait_timeout_is_reported_and_context_survives():
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    assert B.reflex_selftest_wait_timeout(st, 2000) == B.REFLEX_OK
+    assert B.reflex_read_status(st) == B.REFLEX_ETIMEOUT
+    # the context is still usable afterwards
+    cfg = CFG["tiny_fp32"]
+    state = W.make_state(cfg, 0)
+    k, ksum, status = G.gpu_allocate(state, G.params_of(cfg))
+    assert status == B.REFLEX_OK and ksum == int(k.sum())
+
+
+# ---------------------------------------------------------------------------
+# allocation (Eq. 5, Eq. 6-9, clip)
+# ---------------------------------------------------------------------------
+ALLOC_VARIANTS = {
+    "reflex": {},
+    "fixed": dict(delta_role=0, delta_cur=0),
+    "rrb_only": dict(delta_cur=0),
+    "fger_only": dict(delta_role=0),
+    "wide_clip": dict(k_max=14),
+    "tight_tau": dict(tau=0.01),
+}
+
+
+@pytest.mark.parametrize("name", ["tiny_fp32", "llada_moe", "llada2_mini", "llada_moe_b32"])
+@pytest.mark.parametrize("hist", [0, 1, 2])
+@pytest.mark.parametrize("variant", list(ALLOC_VARIANTS))
+def test_allocate_bit_exact(name, hist, variant):
+    cfg = CFG[name]
+    for seed in range(3):
+        state = W.make_state(cfg, seed, hist_len=hist)
+        p = G.params_of(cfg, **ALLOC_VARIANTS[variant])
+        k_gpu, ksum, status = G.gpu_allocate(state, p)
+        k_ref = G.oracle_allocate(state, p)
+        assert status == B.REFLEX_OK
+        assert np.array_equal(k_gpu, k_ref)
+        assert ksum == int(k_ref.sum())
+
+
+def test_allocate_mixed_history_and_ties():
+    cfg = CFG["llada2_mini"]
+    rng = np.random.default_rng(5)
+    state = W.make_state(cfg, 11)
+    state["hist_len"] = rng.integers(0, 3, state["hist_len"].size).astype(np.uint8)
+    # quantised confidences force many equal scores
+    state["conf1"] = (np.round(state["conf1"] * 8) / 8).astype(np.float32)
+    state["conf2"] = (np.round(state["conf2"] * 8) / 8).astype(np.float32)
+    p = G.params_of(cfg)
+    k_gpu, ksum, status = G.gpu_allocate(state, p)
+    assert status == B.REFLEX_OK
+    assert np.array_equal(k_gpu, G.oracle_allocate(state, p))
+
+
+def test_allocate_golden_worked_case():
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden",
+                                    "paper_defaults.json")))["worked_allocation"]
+    T = g["T"]
+    state = dict(block_id=np.array(g["block_id"], np.int32),
+                 seq_offsets=np.array([0, T], np.int32),
+                 active_block=np.array([g["active_block"]], np.int32),
+                 masked=np.array(g["masked"], np.uint8),
+                 conf1=np.array(g["conf1"], np.float32),
+                 conf2=np.array(g["conf1"], np.float32),
+                 hist_len=np.full(T, g["hist_len"], np.uint8))
+    for kmax, key in ((g["k_max_unclipped"], "expected_k_unclipped"),
+                      (g["k_max_clipped"], "expected_k_clipped")):
+        p = B.make_params(k_min=g["k_min"], k_max=kmax)
+        k, ksum, status = G.gpu_allocate(state, p)
+        assert status == B.REFLEX_OK
+        assert k.tolist() == g[key]
+
+
+def test_allocate_capacity_error_is_reported():
+    T = 5000
+    state = dict(block_id=np.ones(T, np.int32), seq_offsets=np.array([0, T], np.int32),
+                 active_block=np.array([1], np.int32), masked=np.ones(T, np.uint8),
+                 conf1=np.full(T, 0.5, np.float32), conf2=np.full(T, 0.5, np.float32),
+                 hist_len=np.full(T, 2, np.uint8))
+    k, ksum, status = G.gpu_allocate(state, B.make_params())
+    assert status == B.REFLEX_ECAPACITY
+    assert np.all(k == 12) and ksum == 12 * T
+
+
+# ---------------------------------------------------------------------------
+# the MoE layer (Eq. 2)
+# ---------------------------------------------------------------------------
+def _k_for(cfg, seed=0, **override):
+    state = W.make_state(cfg, seed)
+    return G.oracle_allocate(state, G.params_of(cfg, **override))
+
+
+def test_forward_tiny_fp32_full():
+    cfg = CFG["tiny_fp32"]
+    layer = W.make_layer(cfg, 0)
+    k = _k_for(cfg)
+    gl = G.GpuLayer(cfg, layer)
+    out, rec, status = gl.forward(k)
+    assert status == B.REFLEX_OK
+    ref = G.oracle_layer(cfg, layer, k)
+    G.check_routing(rec, ref, k, cfg.E)
+    rel, mx = G.out_errors(out, ref["out"])
+    assert rel <= G.F32_REL_L2 and mx <= G.F32_MAX_ABS, (rel, mx)
+
+
+def _bf16_case(T, d, E, inter, shared, kmax, seed):
+    cfg = W.LayerConfig(name="case", dtype="bf16", d=d, E=E, inter=inter,
+                        shared_inter=shared, k_min=1, k_base=min(2, kmax),
+                        k_max=kmax, delta_role=1, delta_cur=1, w_cf=0.3, n_seq=1,
+                        prompt_len=T, gen_len=0, block=32, weight_std=0.05,
+                        conf="uniform", mask_rule="half")
+    layer = W.make_layer(cfg, seed, T=T)
+    return cfg, layer
+
+
+@pytest.mark.parametrize("T,d,E,inter,shared,kmax,kmode", [
+    (96, 256, 8, 128, 0, 4, "random"),     # one partial m-tile per expert
+    (1000, 256, 4, 128, 0, 4, "max"),      # 8 m-tiles per expert, ragged tail
+    (777, 512, 16, 256, 128, 6, "random"),  # shared expert, N > one tile
+    (1, 256, 8, 128, 0, 4, "random"),      # single token
+    (300, 256, 64, 128, 0, 2, "one"),      # many empty experts
+])
+@pytest.mark.parametrize("simt", [False, True])
+def test_forward_bf16_small(T, d, E, inter, shared, kmax, kmode, simt):
+    cfg, layer = _bf16_case(T, d, E, inter, shared, kmax, seed=T + E)
+    rng = np.random.default_rng(T)
+    if kmode == "random":
+        k = rng.integers(1, kmax + 1, T).astype(np.int32)
+    elif kmode == "max":
+        k = np.full(T, kmax, np.int32)
+    else:
+        k = np.ones(T, np.int32)
+    gl = G.GpuLayer(cfg, layer)
+    flags = B.REFLEX_FLAG_RENORM_TOPK | (B.REFLEX_FLAG_SIMT_EXPERTS if simt else 0)
+    out, rec, status = gl.forward(k, flags=flags)
+    assert status == B.REFLEX_OK
+    ref = G.oracle_layer(cfg, layer, k)
+    G.check_routing(rec, ref, k, cfg.E)
+    rel, mx = G.out_errors(out, ref["out"])
+    assert rel <= G.BF16_REL_L2 and mx <= G.BF16_MAX_ABS, (rel, mx)
+
+
+def test_forward_llada_moe_full():
+    cfg = CFG["llada_moe"]
+    layer = W.make_layer(cfg, 0)
+    k = _k_for(cfg)
+    gl = G.GpuLayer(cfg, layer)
+    out, rec, status = gl.forward(k)
+    assert status == B.REFLEX_OK
+    ref = G.oracle_layer(cfg, layer, k)          # every token
+    G.check_routing(rec, ref, k, cfg.E)
+    rel, mx = G.out_errors(out, ref["out"])
+    assert rel <= G.BF16_REL_L2 and mx <= G.BF16_MAX_ABS, (rel, mx)
+    # the SIMT expert path agrees with the tensor-core path
+    out2, rec2, status2 = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK |
+                                     B.REFLEX_FLAG_SIMT_EXPERTS)
+    assert status2 == B.REFLEX_OK
+    rel2, mx2 = G.out_errors(out2, ref["out"])
+    assert rel2 <= G.BF16_REL_L2 and mx2 <= G.BF16_MAX_ABS
+
+
+def test_forward_llada2_mini_sampled():
+    cfg = CFG["llada2_mini"]
+    layer = W.make_layer(cfg, 0)
+    state = W.make_state(cfg, 0)
+    k = G.oracle_allocate(state, G.params_of(cfg))
+    tokens = W.sample_tokens(state)
+    gl = G.GpuLayer(cfg, layer)
+    out, rec, status = gl.forward(k)
+    assert status == B.REFLEX_OK
+    ref = G.oracle_layer(cfg, layer, k, tokens=tokens)
+    G.check_routing(rec, ref, k, cfg.E)
+    rel, mx = G.out_errors(out[tokens], ref["out"])
+    assert rel <= G.BF16_REL_L2 and mx <= G.BF16_MAX_ABS, (rel, mx)
+
+
+def test_forward_fixed_counts_equal_uniform_run():
+    # delta_role = delta_cur = 0 -> uniform K_base: identical to a plain
+    # fixed top-K_base call on the same kernels, bit for bit
+    cfg = CFG["llada_moe"]
+    layer = W.make_layer(cfg, 1)
+    k_alloc = _k_for(cfg, 1, delta_role=0, delta_cur=0)
+    assert np.all(k_alloc == cfg.k_base)
+    gl = G.GpuLayer(cfg, layer)
+    a, _, _ = gl.forward(k_alloc)
+    b, _, _ = gl.forward(np.full(cfg.T, cfg.k_base, np.int32))
+    assert np.array_equal(a, b)
+
+
+def test_forward_without_renorm():
+    cfg = CFG["tiny_fp32"]
+    layer = W.make_layer(cfg, 3)
+    k = _k_for(cfg, 3)
+    gl = G.GpuLayer(cfg, layer)
+    out, rec, status = gl.forward(k, flags=0)
+    ref = G.oracle_layer(cfg, layer, k, renorm=False)
+    G.check_routing(rec, ref, k, cfg.E)
+    rel, mx = G.out_errors(out, ref["out"])
+    assert rel <= G.F32_REL_L2 and mx <= G.F32_MAX_ABS
+
+
+def test_forward_count_out_of_range_flagged():
+    cfg = CFG["tiny_fp32"]
+    layer = W.make_layer(cfg, 0)
+    gl = G.GpuLayer(cfg, layer)
+    k = np.full(cfg.T, 2, np.int32)
+    k[5] = 9                       # > k_max
+    _, rec, status = gl.forward(k)
+    assert status == B.REFLEX_EKRANGE
+    assert (rec["ids"][5] >= 0).sum() == cfg.k_max   # clamped, still routed
+
+
+def test_forward_stages_compose():
+    cfg = CFG["llada_moe"]
+    layer = W.make_layer(cfg, 2)
+    k = _k_for(cfg, 2)
+    gl = G.GpuLayer(cfg, layer)
+    full, _, _ = gl.forward(k)
+    kd = torch.from_numpy(k).cuda()
+    out = torch.empty_like(gl.dev["hidden"])
+    for st in (B.REFLEX_STAGE_ROUTE, B.REFLEX_STAGE_DISPATCH,
+               B.REFLEX_STAGE_EXPERT_UP, B.REFLEX_STAGE_EXPERT_DOWN,
+               B.REFLEX_STAGE_COMBINE):
+        gl.moe.forward(gl.dev["hidden"], kd, out=out,
+                       flags=B.REFLEX_FLAG_RENORM_TOPK | st)
+    torch.cuda.synchronize()
+    assert np.array_equal(G.to_f32(out), full)
