@@ -37,6 +37,9 @@ if ROOT not in sys.path:
 
 from paper_2608_01784_gb300 import workloads as W  # noqa: E402
 
+METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
+          "fixed top-K")
+
 # Bytes moved by the dominant kernel per launch, from an ncu capture of the
 # current kernel (profiles/); None when the kernel changed since the capture.
 NCU_TRAFFIC_BYTES = None
@@ -184,7 +187,7 @@ def run_reference(args, cfg, rank, world):
         oracle_step(cfg, layer, state, np.sort(rng.choice(T, n, replace=False)).astype(np.int32))
     dt = time.perf_counter() - t0
     value = n * args.steps / dt
-    line = dict(metric="moe_layer_tokens_per_s", value=value, unit="tokens/s",
+    line = dict(metric=METRIC, value=value, unit="tokens/s",
                 impl="reference", n_gpus=args.gpus, steps=args.steps,
                 warmup=args.warmup, ms_per_step=1e3 * dt / args.steps,
                 higher_is_better=True, scaling="weak", vs_baseline=None,
@@ -361,7 +364,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
     t_roof = max(layer_bytes / (peaks["hbm"] * 1e9), layer_flops / (peaks["bf16"] * 1e12))
     launches_per_step = 10 + (2 if S else 0)
     line = dict(
-        metric="moe_layer_tokens_per_s", value=tokens_per_s, unit="tokens/s",
+        metric=METRIC, value=tokens_per_s, unit="tokens/s",
         n_gpus=world, steps=args.steps, warmup=args.warmup, ms_per_step=ms_step,
         higher_is_better=True, scaling="weak", vs_baseline=None, dtype="bf16"
         if cfg.dtype == "bf16" else "f32", data="synthetic",
