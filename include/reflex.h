@@ -186,6 +186,35 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
                        uint32_t flags, void* workspace, size_t ws_bytes,
                        void* out, reflex_route_record* rec, void* stream);
 
+/*
+ * reflex_route_noalloc — the routing step of reflex_moe_forward (router
+ * scores, TopK(r_i, k_i), router weights) for callers that cannot allocate
+ * device memory: code inside a framework that owns the device allocator and
+ * forbids side allocations, plugins limited to the buffers they are handed,
+ * or processes where cudaMalloc is not allowed after start-up.  The paper has
+ * no counterpart; it is a deployment convenience.
+ *
+ * The one scratch buffer of this step, the fp32 score matrix [T, E], lives
+ * in a fixed array inside the library's device memory
+ * (REFLEX_NOALLOC_MAX_SCORES floats = 4 MiB, held on every GPU that uses the
+ * library until the process exits).  Nothing is allocated or freed.
+ *   ids_out    [T, k_max] int32, alpha_out [T, k_max] fp32: same meaning and
+ *              values as the ids / alpha of reflex_route_record.
+ *   dev_status nullable device error word (cleared, then OR-ed as for the
+ *              forward; read it with reflex_read_status).
+ * Returns REFLEX_EWORKSPACE when T * E > REFLEX_NOALLOC_MAX_SCORES, and
+ * REFLEX_EINVAL for the shape errors of reflex_moe_forward.  The first call
+ * on each device looks up the array's address; make it before any stream
+ * capture.  All calls share the array: calls whose GPU work overlaps in time
+ * race on it and must be serialised.
+ */
+#define REFLEX_NOALLOC_MAX_SCORES (1 << 20)
+int reflex_route_noalloc(int32_t dtype, const void* hidden,
+                         const void* w_router, const int32_t* k, int32_t T,
+                         int32_t d, int32_t E, int32_t k_max, uint32_t flags,
+                         int32_t* ids_out, float* alpha_out,
+                         int32_t* dev_status, void* stream);
+
 /* Synchronises `stream` and returns the status recorded in the workspace's
  * device error word by the last forward (REFLEX_OK if clean). */
 int reflex_moe_status(const void* workspace, void* stream);

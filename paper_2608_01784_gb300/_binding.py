@@ -36,7 +36,7 @@ EXPORTED = (
     "reflex_default_params", "reflex_allocate", "reflex_moe_workspace_size",
     "reflex_moe_forward", "reflex_moe_status", "reflex_read_status",
     "reflex_selftest_wait_timeout", "reflex_status_string",
-    "reflex_abi_version",
+    "reflex_abi_version", "reflex_route_noalloc",
 )
 
 
@@ -102,6 +102,9 @@ def load():
     lib.reflex_status_string.argtypes = [ctypes.c_int]
     lib.reflex_abi_version.restype = ctypes.c_int
     lib.reflex_abi_version.argtypes = []
+    lib.reflex_route_noalloc.restype = ctypes.c_int
+    lib.reflex_route_noalloc.argtypes = [i32, P, P, P, i32, i32, i32, i32,
+                                         ctypes.c_uint32, P, P, P, P]
     _lib = lib
     return lib
 
@@ -191,3 +194,16 @@ def reflex_read_status(dev_status, stream=None) -> int:
 def reflex_selftest_wait_timeout(dev_status, limit_us: int, stream=None) -> int:
     return int(load().reflex_selftest_wait_timeout(_ptr(dev_status), limit_us,
                                                    _stream(stream)))
+
+
+REFLEX_NOALLOC_MAX_SCORES = 1 << 20
+
+
+def reflex_route_noalloc(dtype: int, hidden, w_router, k, T: int, d: int,
+                         E: int, k_max: int, flags: int, ids_out, alpha_out,
+                         dev_status=None, stream=None) -> int:
+    """Routing step with no device allocation (scratch in the library's own
+    fixed array; see include/reflex.h)."""
+    return int(load().reflex_route_noalloc(
+        dtype, _ptr(hidden), _ptr(w_router), _ptr(k), T, d, E, k_max, flags,
+        _ptr(ids_out), _ptr(alpha_out), _ptr(dev_status), _stream(stream)))
