@@ -19,7 +19,7 @@
 namespace rx {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 1024;  // one token per thread for sequences up to 1024
 constexpr int kMaxJ = 4096;
 
 __device__ __forceinline__ float pow2i(int e) {  // e in [-126, 127]

@@ -41,10 +41,8 @@ namespace {
 constexpr int BM = kTileM;   // 128
 constexpr int BK = 64;       // 64 bf16 = 128 bytes = one swizzle row
 constexpr int UMMA_K = 16;
-constexpr int kStages = 4;
 constexpr int kThreads = 192;
-constexpr int BN_SWIGLU = 256;  // 128 gate + 128 up -> 128 activations
-constexpr int BN_DOWN = 256;
+constexpr int kRingBytes = 192 * 1024;  // TMA ring budget per CTA
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr uint64_t kDrainNs = 1000000000ull;
 
@@ -55,9 +53,11 @@ struct Cfg {
   static constexpr int kABytes = BM * BK * 2;
   static constexpr int kBBytes = BN * BK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = kRingBytes / kStageBytes;  // 4 (BN 256), 6 (BN 128)
   static constexpr int kTmemCols = 2 * BN;
   static constexpr int kBarBytes = 256;
   static constexpr int kSmemBytes = kStages * kStageBytes + kBarBytes + 1024;
+  static_assert(kStages >= 2 && kStages <= 8, "ring depth");
 };
 
 struct KParams {
@@ -211,6 +211,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const __grid_constant__ CUtensorMap map_b,
                         const KParams p) {
   using C = Cfg<BN>;
+  constexpr int kStages = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -464,15 +465,30 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
 
 }  // namespace
 
-cudaError_t launch_swiglu_tc(const TcGemmArgs& a, cudaStream_t stream) {
-  return launch_impl<BN_SWIGLU, kModeSwiGLU>(a, stream);
+cudaError_t launch_swiglu_tc(const TcGemmArgs& a, int bn, cudaStream_t stream) {
+  if (bn == 128) return launch_impl<128, kModeSwiGLU>(a, stream);
+  return launch_impl<256, kModeSwiGLU>(a, stream);
 }
-cudaError_t launch_down_tc(const TcGemmArgs& a, cudaStream_t stream) {
-  return launch_impl<BN_DOWN, kModeDown>(a, stream);
+cudaError_t launch_down_tc(const TcGemmArgs& a, int bn, cudaStream_t stream) {
+  if (bn == 128) return launch_impl<128, kModeDown>(a, stream);
+  return launch_impl<256, kModeDown>(a, stream);
 }
-int tc_swiglu_b_box_rows() { return BN_SWIGLU / 2; }
-int tc_down_b_box_rows() { return BN_DOWN; }
-int tc_swiglu_n_granule() { return BN_SWIGLU / 2; }
-int tc_down_n_granule() { return BN_DOWN; }
+// SwiGLU loads gate and up halves as two boxes of bn/2 rows; down loads one
+// box of bn rows.
+int tc_b_box_rows(bool swiglu, int bn) { return swiglu ? bn / 2 : bn; }
+// Output columns of one tile.
+int tc_n_granule(bool swiglu, int bn) { return swiglu ? bn / 2 : bn; }
+
+// Tile width: 256 when there are enough tiles to fill every SM several
+// times over (large M per expert: fewer re-reads of the A rows per output),
+// else 128 so that the persistent CTAs get more, smaller tiles and the last
+// partial wave is short (small M: the GEMM is a weight stream).
+int tc_pick_bn(bool swiglu, int n_total, int64_t mtiles_est, int num_sms) {
+  const int g256 = tc_n_granule(swiglu, 256);
+  const int g128 = tc_n_granule(swiglu, 128);
+  if (n_total % g256 != 0) return (n_total % g128 == 0) ? 128 : 0;
+  const int64_t tiles256 = static_cast<int64_t>(n_total / g256) * mtiles_est;
+  return tiles256 >= 8LL * num_sms ? 256 : 128;
+}
 
 }  // namespace rx

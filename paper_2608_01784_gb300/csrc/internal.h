@@ -90,14 +90,15 @@ struct TcGemmArgs {
   uint32_t* err;
   int num_sms;
 };
-// SwiGLU: out = silu(A Wg^T) * (A Wu^T).  Down: out = A Wd^T.
-cudaError_t launch_swiglu_tc(const TcGemmArgs& a, cudaStream_t stream);
-cudaError_t launch_down_tc(const TcGemmArgs& a, cudaStream_t stream);
-// Box rows of the B operand each kernel expects in its tensor map.
-int tc_swiglu_b_box_rows();
-int tc_down_b_box_rows();
-int tc_swiglu_n_granule();  // inter must be a multiple of this
-int tc_down_n_granule();    // d must be a multiple of this
+// SwiGLU: out = silu(A Wg^T) * (A Wu^T).  Down: out = A Wd^T.  bn = tile
+// width (128 or 256, from tc_pick_bn); the B tensor map's box must have
+// tc_b_box_rows(swiglu, bn) rows.
+cudaError_t launch_swiglu_tc(const TcGemmArgs& a, int bn, cudaStream_t stream);
+cudaError_t launch_down_tc(const TcGemmArgs& a, int bn, cudaStream_t stream);
+int tc_b_box_rows(bool swiglu, int bn);
+int tc_n_granule(bool swiglu, int bn);  // output columns per tile
+// 0 when n_total is not a multiple of the smaller granule.
+int tc_pick_bn(bool swiglu, int n_total, int64_t mtiles_est, int num_sms);
 
 // ---- combine (combine.cu) -------------------------------------------------
 // out[t] = sum_{j<k_t} alpha[t,j] * y[row_of[t,j]] (+ y_shared[t]).

@@ -235,10 +235,18 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
     return REFLEX_EINVAL;
 
   const bool simt = dtype == REFLEX_DTYPE_F32 || (flags & REFLEX_FLAG_SIMT_EXPERTS);
+  // tile widths of the tcgen05 GEMMs: the m-tile count is only known on the
+  // device, so the choice uses the expected count for pairs spread over
+  // every expert (one partial tile per expert plus T k_max / 2 rows)
+  const int sms_h = num_sms_current();
+  const int64_t mt_est = E + (static_cast<int64_t>(T) * k_max / 2 + 127) / 128;
+  const int64_t mt_dense = (T + 127) / 128;
+  const int bn_up = rx::tc_pick_bn(true, inter, mt_est, sms_h);
+  const int bn_dn = rx::tc_pick_bn(false, d, mt_est, sms_h);
+  const int bn_sup = shared_inter ? rx::tc_pick_bn(true, shared_inter, mt_dense, sms_h) : 128;
+  const int bn_sdn = shared_inter ? rx::tc_pick_bn(false, d, mt_dense, sms_h) : 128;
   if (!simt) {
-    if (d % rx::tc_down_n_granule() != 0 || inter % rx::tc_swiglu_n_granule() != 0 ||
-        (shared_inter % rx::tc_swiglu_n_granule()) != 0)
-      return REFLEX_EUNSUPPORTED;
+    if (bn_up == 0 || bn_dn == 0 || bn_sup == 0 || bn_sdn == 0) return REFLEX_EUNSUPPORTED;
     if (encode_fn() == nullptr) return REFLEX_ECUDA;
   }
   constexpr uint32_t kAllStages = REFLEX_STAGE_ROUTE | REFLEX_STAGE_DISPATCH |
@@ -247,7 +255,7 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
   uint32_t stages = flags & kAllStages;
   if (stages == 0) stages = kAllStages;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const int sms = num_sms_current();
+  const int sms = sms_h;
   const int cap = static_cast<int>(L.cap_rows);
   float* z = reinterpret_cast<float*>(ws + L.z);
   float* alpha = reinterpret_cast<float*>(ws + L.alpha);
@@ -291,10 +299,10 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
       CUtensorMap ma1, mb1, ma2, mb2;
       if (!make_map(&ma1, xperm, cap, d, rx::kTileM) ||
           !make_map(&mb1, w_gate_up, static_cast<int64_t>(E) * 2 * inter, d,
-                    rx::tc_swiglu_b_box_rows()) ||
+                    rx::tc_b_box_rows(true, bn_up)) ||
           !make_map(&ma2, amid, cap, inter, rx::kTileM) ||
           !make_map(&mb2, w_down, static_cast<int64_t>(E) * d, inter,
-                    rx::tc_down_b_box_rows()))
+                    rx::tc_b_box_rows(false, bn_dn)))
         return REFLEX_ECUDA;
       rx::TcGemmArgs g1{&ma1, &mb1, d, inter, 2 * inter, inter, grouped, amid, inter, err, sms};
       rx::TcGemmArgs g2{&ma2, &mb2, inter, d, d, 0, grouped, xperm, d, err, sms};
@@ -302,20 +310,20 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
       if (shared_inter &&
           (!make_map(&sa1, hidden, T, d, rx::kTileM) ||
            !make_map(&sb1, shared_gate_up, 2 * static_cast<int64_t>(shared_inter), d,
-                     rx::tc_swiglu_b_box_rows()) ||
+                     rx::tc_b_box_rows(true, bn_sup)) ||
            !make_map(&sa2, ash, T, shared_inter, rx::kTileM) ||
-           !make_map(&sb2, shared_down, d, shared_inter, rx::tc_down_b_box_rows())))
+           !make_map(&sb2, shared_down, d, shared_inter, rx::tc_b_box_rows(false, bn_sdn))))
         return REFLEX_ECUDA;
       rx::TcGemmArgs h1{&sa1, &sb1, d, shared_inter, 2 * shared_inter, shared_inter,
                         dense, ash, shared_inter, err, sms};
       rx::TcGemmArgs h2{&sa2, &sb2, shared_inter, d, d, 0, dense, ysh, d, err, sms};
       if (up) {
-        RX_CUDA(rx::launch_swiglu_tc(g1, s));
-        if (shared_inter) RX_CUDA(rx::launch_swiglu_tc(h1, s));
+        RX_CUDA(rx::launch_swiglu_tc(g1, bn_up, s));
+        if (shared_inter) RX_CUDA(rx::launch_swiglu_tc(h1, bn_sup, s));
       }
       if (down) {
-        RX_CUDA(rx::launch_down_tc(g2, s));
-        if (shared_inter) RX_CUDA(rx::launch_down_tc(h2, s));
+        RX_CUDA(rx::launch_down_tc(g2, bn_dn, s));
+        if (shared_inter) RX_CUDA(rx::launch_down_tc(h2, bn_sdn, s));
       }
     }
   }

@@ -6,10 +6,10 @@
 // k = 0, 1, ..., d-1 starting from +0, in fp32 (bf16 inputs are widened
 // exactly).  Fixing the summation order makes the scores — and therefore the
 // selected expert sets, an integer result — reproducible bit for bit.  The
-// kernel is a register-tiled SIMT GEMM: each thread owns TM tokens x 4
-// experts and walks k in order, so the fixed order costs no extra work; the
-// tile (8*TM tokens x 64 experts) is staged through double-buffered shared
-// memory in chunks of 32 k.
+// kernel is a register-tiled SIMT GEMM: each thread owns TM tokens x TN
+// experts and walks k in order, so the fixed order costs no extra work; raw
+// tiles stream through a cp.async ring of 32-k chunks, and each chunk is
+// widened once into a k-major fp32 buffer read with conflict-free float4s.
 //
 // Selection.  One warp per token keeps E/32 scores per lane and runs k_i
 // rounds of a warp-wide max over packed 64-bit keys
@@ -22,113 +22,173 @@
 namespace rx {
 namespace {
 
-constexpr int kKc = 32;          // k per shared-memory chunk
-constexpr int kExpPerCta = 64;   // 16 thread columns x 4 experts
-constexpr int kThreadsL = 128;   // 16 x 8 threads
+constexpr int kKc = 32;      // k per pipeline stage
+constexpr int kStagesL = 3;  // cp.async ring depth (raw input tiles)
 
-template <typename Tin, int TM>
-__global__ void __launch_bounds__(kThreadsL)
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, bool valid) {
+  const uint32_t dst = smem_addr(smem);
+  const int src_bytes = valid ? 16 : 0;  // 0: zero-fill, nothing is read
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst),
+               "l"(gmem), "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// 8 raw elements -> fp32 (exact widening).
+__device__ __forceinline__ void widen8(const uint8_t* p, float* f, const __nv_bfloat16*) {
+  const uint4 v = *reinterpret_cast<const uint4*>(p);
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = __uint_as_float(w[i] << 16);
+    f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+  }
+}
+__device__ __forceinline__ void widen8(const uint8_t* p, float* f, const float*) {
+  const float4 a = *reinterpret_cast<const float4*>(p);
+  const float4 b = *reinterpret_cast<const float4*>(p + 16);
+  f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
+  f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
+}
+
+// Tile geometry.  A warp is 8 token groups (ty) x 4 expert groups (tx);
+// thread (ty, tx) owns TM consecutive tokens and TN experts taken as TN/4
+// float4 groups spaced 16 experts apart, so each operand read of a warp is
+// one contiguous, conflict-free shared-memory wavefront.  WT x WE warps per
+// CTA: BT = 8 TM WT tokens x BE = 4 TN WE experts.
+template <typename Tin, int TM, int TN, int WT, int WE>
+struct LogitsCfg {
+  static constexpr int BT = 8 * TM * WT;
+  static constexpr int BE = 4 * TN * WE;
+  static constexpr int kRows = BT + BE;
+  static constexpr int kThreads = 32 * WT * WE;
+  static constexpr int kRowBytes = kKc * static_cast<int>(sizeof(Tin)) + 16;
+  static constexpr int kVecs = kKc * static_cast<int>(sizeof(Tin)) / 16;
+  static constexpr int kElemsPerVec = 16 / static_cast<int>(sizeof(Tin));
+  static constexpr int kRawStage = kRows * kRowBytes;
+  static constexpr int kCbuf = kKc * kRows;  // floats in one widened chunk
+  static constexpr int kSmem = kStagesL * kRawStage + 2 * kCbuf * 4;
+};
+
+// Each score is one fma chain over k = 0 .. d-1 in order.  Raw chunks of 32 k
+// stream through a cp.async ring; each chunk is widened once into a k-major
+// fp32 buffer buf[k][row] (rows: BT tokens, then BE experts) and every thread
+// then reads TM + TN operands per k for TM x TN fmas.
+template <typename Tin, int TM, int TN, int WT, int WE>
+__global__ void __launch_bounds__(LogitsCfg<Tin, TM, TN, WT, WE>::kThreads)
     logits_kernel(const Tin* __restrict__ h, const Tin* __restrict__ w, int T,
                   int d, int E, float* __restrict__ z) {
-  constexpr int BT = 8 * TM;  // tokens per CTA
-  __shared__ __align__(16) float hs[2][kKc][BT];
-  __shared__ __align__(16) float ws[2][kKc][kExpPerCta];
-  const int tx = threadIdx.x & 15;  // expert group (4 experts)
-  const int ty = threadIdx.x >> 4;  // token group (TM tokens)
+  using C = LogitsCfg<Tin, TM, TN, WT, WE>;
+  constexpr int BT = C::BT, BE = C::BE, R = C::kRows, NT = C::kThreads;
+  extern __shared__ __align__(16) uint8_t smem_l[];
+  float* cbuf = reinterpret_cast<float*>(smem_l + kStagesL * C::kRawStage);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int ty = lane >> 2, tx = lane & 3;
+  const int wt = warp / WE, we = warp % WE;
+  const int my_t = wt * (8 * TM) + ty * TM;  // first token row of this thread
+  const int my_e = we * (4 * TN) + 4 * tx;   // first expert row of group 0
   const int t0 = blockIdx.x * BT;
-  const int e0 = blockIdx.y * kExpPerCta;
-
-  // loader: h tile = BT rows x 4 vectors of 8; w tile = 64 rows x 4 vectors
-  constexpr int kHVec = BT * (kKc / 8);
-  float hv[8], wv[2][8];
+  const int e0 = blockIdx.y * BE;
   const int nchunks = d / kKc;
 
-  auto load_regs = [&](int c) {
+  auto issue = [&](int c) {
+    uint8_t* st = smem_l + (c % kStagesL) * C::kRawStage;
     const int k0 = c * kKc;
-    if (threadIdx.x < kHVec) {
-      const int r = threadIdx.x >> 2, v = threadIdx.x & 3;
-      const int t = t0 + r;
-      if (t < T) {
-        load8(h + static_cast<int64_t>(t) * d + k0 + v * 8, hv);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) hv[i] = 0.f;
-      }
-    }
-#pragma unroll
-    for (int s = 0; s < 2; ++s) {
-      const int idx = threadIdx.x + s * kThreadsL;
-      const int r = idx >> 2, v = idx & 3;
-      const int e = e0 + r;
-      if (e < E) {
-        load8(w + static_cast<int64_t>(e) * d + k0 + v * 8, wv[s]);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) wv[s][i] = 0.f;
-      }
+    for (int v = threadIdx.x; v < R * C::kVecs; v += NT) {
+      const int r = v / C::kVecs, q = v % C::kVecs;
+      const bool is_h = r < BT;
+      const int idx = is_h ? t0 + r : e0 + (r - BT);
+      const bool ok = idx < (is_h ? T : E);
+      const Tin* base = is_h ? h : w;
+      cp_async16(st + r * C::kRowBytes + q * 16,
+                 base + (ok ? static_cast<int64_t>(idx) * d + k0 + q * C::kElemsPerVec : 0),
+                 ok);
     }
   };
-  auto store_smem = [&](int buf) {
-    if (threadIdx.x < kHVec) {
-      const int r = threadIdx.x >> 2, v = threadIdx.x & 3;
+  auto widen = [&](int c, float* buf) {
+    const uint8_t* st = smem_l + (c % kStagesL) * C::kRawStage;
+    for (int v = threadIdx.x; v < R * (kKc / 8); v += NT) {
+      const int r = v % R, q = v / R;  // consecutive rows per warp
+      float f[8];
+      widen8(st + r * C::kRowBytes + q * 8 * sizeof(Tin), f, static_cast<const Tin*>(nullptr));
 #pragma unroll
-      for (int i = 0; i < 8; ++i) hs[buf][v * 8 + i][r] = hv[i];
-    }
-#pragma unroll
-    for (int s = 0; s < 2; ++s) {
-      const int idx = threadIdx.x + s * kThreadsL;
-      const int r = idx >> 2, v = idx & 3;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) ws[buf][v * 8 + i][r] = wv[s][i];
+      for (int i = 0; i < 8; ++i) buf[(q * 8 + i) * R + r] = f[i];
     }
   };
 
-  float acc[TM][4];
+  float acc[TM][TN];
 #pragma unroll
   for (int i = 0; i < TM; ++i)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+    for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
 
-  load_regs(0);
-  store_smem(0);
-  __syncthreads();
+#pragma unroll
+  for (int c = 0; c < kStagesL - 1; ++c) {
+    if (c < nchunks) issue(c);
+    cp_async_commit();
+  }
   for (int c = 0; c < nchunks; ++c) {
-    const int buf = c & 1;
-    if (c + 1 < nchunks) load_regs(c + 1);
+    cp_async_wait<kStagesL - 2>();
+    __syncthreads();  // raw chunk c visible; iteration c-1 finished everywhere
+    if (c + kStagesL - 1 < nchunks) issue(c + kStagesL - 1);
+    cp_async_commit();
+    float* buf = cbuf + (c & 1) * C::kCbuf;
+    widen(c, buf);
+    __syncthreads();
 #pragma unroll 8
     for (int kk = 0; kk < kKc; ++kk) {
-      const float4 wq = *reinterpret_cast<const float4*>(&ws[buf][kk][tx * 4]);
-      float hq[TM];
+      const float* row = buf + kk * R;
+      float hv[TM], wv[TN];
       if constexpr (TM == 4) {
-        const float4 t4 = *reinterpret_cast<const float4*>(&hs[buf][kk][ty * 4]);
-        hq[0] = t4.x; hq[1] = t4.y; hq[2] = t4.z; hq[3] = t4.w;
-      } else if constexpr (TM == 2) {
-        const float2 t2 = *reinterpret_cast<const float2*>(&hs[buf][kk][ty * 2]);
-        hq[0] = t2.x; hq[1] = t2.y;
+        const float4 q4 = *reinterpret_cast<const float4*>(row + my_t);
+        hv[0] = q4.x; hv[1] = q4.y; hv[2] = q4.z; hv[3] = q4.w;
       } else {
-        hq[0] = hs[buf][kk][ty];
+#pragma unroll
+        for (int i = 0; i < TM; ++i) hv[i] = row[my_t + i];
       }
 #pragma unroll
-      for (int i = 0; i < TM; ++i) {
-        acc[i][0] = __fmaf_rn(hq[i], wq.x, acc[i][0]);
-        acc[i][1] = __fmaf_rn(hq[i], wq.y, acc[i][1]);
-        acc[i][2] = __fmaf_rn(hq[i], wq.z, acc[i][2]);
-        acc[i][3] = __fmaf_rn(hq[i], wq.w, acc[i][3]);
+      for (int g = 0; g < TN / 4; ++g) {
+        const float4 q4 = *reinterpret_cast<const float4*>(row + BT + my_e + 16 * g);
+        wv[4 * g] = q4.x; wv[4 * g + 1] = q4.y; wv[4 * g + 2] = q4.z; wv[4 * g + 3] = q4.w;
       }
+#pragma unroll
+      for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) acc[i][j] = __fmaf_rn(hv[i], wv[j], acc[i][j]);
     }
-    if (c + 1 < nchunks) store_smem(buf ^ 1);
-    __syncthreads();
   }
+  cp_async_wait<0>();
 #pragma unroll
   for (int i = 0; i < TM; ++i) {
-    const int t = t0 + ty * TM + i;
+    const int t = t0 + my_t + i;
     if (t >= T) continue;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int e = e0 + tx * 4 + j;
+    for (int j = 0; j < TN; ++j) {
+      const int e = e0 + my_e + 16 * (j / 4) + (j % 4);
       if (e < E) z[static_cast<int64_t>(t) * E + e] = acc[i][j];
     }
   }
+}
+
+template <typename Tin, int TM, int TN, int WT, int WE>
+cudaError_t launch_logits_tile(const Tin* h, const Tin* w, int T, int d, int E,
+                               float* z, cudaStream_t s) {
+  using C = LogitsCfg<Tin, TM, TN, WT, WE>;
+  auto kern = logits_kernel<Tin, TM, TN, WT, WE>;
+  if (C::kSmem > 48 * 1024) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+    if (e != cudaSuccess) return e;
+  }
+  const dim3 g((T + C::BT - 1) / C::BT, (E + C::BE - 1) / C::BE);
+  kern<<<g, C::kThreads, C::kSmem, s>>>(h, w, T, d, E, z);
+  return cudaGetLastError();
 }
 
 __device__ __forceinline__ uint32_t order_bits(float v) {
@@ -221,23 +281,135 @@ __global__ void __launch_bounds__(kSelWarps * 32)
   }
 }
 
+// Short-batch variant: too few (token, expert) chains to fill the GPU with
+// the widened-buffer tiles, so each CTA (4 warps) keeps 8 TM tokens x 64
+// experts, one 4-stage ring of 32-k raw chunks, and widens operands at use
+// (no extra pass, one barrier per chunk).  Thread (warp w, lane l) owns
+// tokens t0 + (l >> 2) + 8 i and experts e0 + 16 w + (l & 3) + 4 j; with
+// rows padded by 16 bytes each 16-byte operand read of a warp is
+// conflict-free.
+constexpr int kStagesS = 4;
+constexpr int kThreadsS = 128;
+
+template <typename Tin>
+__device__ __forceinline__ void row8(const uint8_t* p, float* f) {
+  widen8(p, f, static_cast<const Tin*>(nullptr));
+}
+
+template <typename Tin, int TM>
+__global__ void __launch_bounds__(kThreadsS)
+    logits_short_kernel(const Tin* __restrict__ h, const Tin* __restrict__ w,
+                        int T, int d, int E, float* __restrict__ z) {
+  constexpr int BT = 8 * TM, BE = 64;
+  constexpr int kRowBytes = kKc * static_cast<int>(sizeof(Tin)) + 16;
+  constexpr int kVecs = kKc * static_cast<int>(sizeof(Tin)) / 16;
+  constexpr int kElemsPerVec = 16 / static_cast<int>(sizeof(Tin));
+  constexpr int kHBytes = BT * kRowBytes;
+  constexpr int kStageBytes = (BT + BE) * kRowBytes;
+  extern __shared__ __align__(16) uint8_t smem_s[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int ty = lane >> 2, tx = lane & 3;
+  const int t0 = blockIdx.x * BT;
+  const int e0 = blockIdx.y * BE;
+  const int nchunks = d / kKc;
+
+  auto issue = [&](int c) {
+    uint8_t* st = smem_s + (c % kStagesS) * kStageBytes;
+    const int k0 = c * kKc;
+    for (int v = threadIdx.x; v < (BT + BE) * kVecs; v += kThreadsS) {
+      const int r = v / kVecs, q = v % kVecs;
+      const bool is_h = r < BT;
+      const int idx = is_h ? t0 + r : e0 + (r - BT);
+      const bool ok = idx < (is_h ? T : E);
+      const Tin* base = is_h ? h : w;
+      cp_async16(st + r * kRowBytes + q * 16,
+                 base + (ok ? static_cast<int64_t>(idx) * d + k0 + q * kElemsPerVec : 0), ok);
+    }
+  };
+
+  float acc[TM][4];
+#pragma unroll
+  for (int i = 0; i < TM; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+
+#pragma unroll
+  for (int c = 0; c < kStagesS - 1; ++c) {
+    if (c < nchunks) issue(c);
+    cp_async_commit();
+  }
+  for (int c = 0; c < nchunks; ++c) {
+    cp_async_wait<kStagesS - 2>();
+    __syncthreads();
+    if (c + kStagesS - 1 < nchunks) issue(c + kStagesS - 1);
+    cp_async_commit();
+    const uint8_t* st = smem_s + (c % kStagesS) * kStageBytes;
+#pragma unroll
+    for (int kv = 0; kv < kKc / 8; ++kv) {
+      float hv[TM][8], wv[4][8];
+#pragma unroll
+      for (int i = 0; i < TM; ++i)
+        row8<Tin>(st + (ty + 8 * i) * kRowBytes + kv * 8 * sizeof(Tin), hv[i]);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        row8<Tin>(st + kHBytes + (16 * warp + tx + 4 * j) * kRowBytes + kv * 8 * sizeof(Tin),
+                  wv[j]);
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk)
+#pragma unroll
+        for (int i = 0; i < TM; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            acc[i][j] = __fmaf_rn(hv[i][kk], wv[j][kk], acc[i][j]);
+    }
+  }
+  cp_async_wait<0>();
+#pragma unroll
+  for (int i = 0; i < TM; ++i) {
+    const int t = t0 + ty + 8 * i;
+    if (t >= T) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int e = e0 + 16 * warp + tx + 4 * j;
+      if (e < E) z[static_cast<int64_t>(t) * E + e] = acc[i][j];
+    }
+  }
+}
+
+template <typename Tin, int TM>
+cudaError_t launch_logits_short(const Tin* h, const Tin* w, int T, int d, int E,
+                                float* z, cudaStream_t s) {
+  constexpr int kRowBytes = kKc * static_cast<int>(sizeof(Tin)) + 16;
+  constexpr int smem = kStagesS * (8 * TM + 64) * kRowBytes;
+  auto kern = logits_short_kernel<Tin, TM>;
+  if (smem > 48 * 1024) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+  }
+  const dim3 g((T + 8 * TM - 1) / (8 * TM), (E + 63) / 64);
+  kern<<<g, kThreadsS, smem, s>>>(h, w, T, d, E, z);
+  return cudaGetLastError();
+}
+
+// Tile choice: the widened-buffer tiles when they fill most SMs without
+// overhanging the expert count (more chains per thread, fewer operand reads
+// per fma); otherwise the short-batch kernel with the largest token tile
+// that still fills most SMs.
 template <typename Tin>
 cudaError_t logits_dispatch(const Tin* h, const Tin* w, int T, int d, int E,
                             float* z, int num_sms, cudaStream_t s) {
-  const int gy = (E + kExpPerCta - 1) / kExpPerCta;
-  auto grid_for = [&](int tm) { return ((T + 8 * tm - 1) / (8 * tm)) * gy; };
-  const int want = 2 * num_sms;
-  if (grid_for(4) >= want) {
-    dim3 g((T + 31) / 32, gy);
-    logits_kernel<Tin, 4><<<g, kThreadsL, 0, s>>>(h, w, T, d, E, z);
-  } else if (grid_for(2) >= want) {
-    dim3 g((T + 15) / 16, gy);
-    logits_kernel<Tin, 2><<<g, kThreadsL, 0, s>>>(h, w, T, d, E, z);
-  } else {
-    dim3 g((T + 7) / 8, gy);
-    logits_kernel<Tin, 1><<<g, kThreadsL, 0, s>>>(h, w, T, d, E, z);
-  }
-  return cudaGetLastError();
+  auto grid_for = [&](int bt, int be) {
+    return static_cast<int64_t>((T + bt - 1) / bt) * ((E + be - 1) / be);
+  };
+  const int64_t want = (num_sms * 4) / 5;
+  if (E >= 128 && grid_for(64, 128) >= want)  // TM 4, TN 8, 2 x 4 warps
+    return launch_logits_tile<Tin, 4, 8, 2, 4>(h, w, T, d, E, z, s);
+  if (E >= 64 && grid_for(64, 64) >= want)    // TM 4, TN 4, 2 x 4 warps
+    return launch_logits_tile<Tin, 4, 4, 2, 4>(h, w, T, d, E, z, s);
+  if (grid_for(32, 64) >= want) return launch_logits_short<Tin, 4>(h, w, T, d, E, z, s);
+  if (grid_for(16, 64) >= want) return launch_logits_short<Tin, 2>(h, w, T, d, E, z, s);
+  return launch_logits_short<Tin, 1>(h, w, T, d, E, z, s);
 }
 
 }  // namespace
