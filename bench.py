@@ -15,7 +15,12 @@ grouped gate/up (SwiGLU) GEMM; `e2e` times the same step from pinned host
 buffers through the C ABI with the copies inside the timed region.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reflex|reference]
-                  [--config NAME] [--no-cpu-baseline]
+                  [--config NAME] [--no-cpu-baseline] [--sweep]
+--config llada_moe_stack16: a whole denoising forward of 16 LLaDA-MoE-shaped
+layers (batch 32 x 1024 tokens, counts allocated once and shared by every
+layer, residual connection, fresh weights per layer drawn on the device).
+--sweep: LLaDA2.0-mini layer shapes, 256 .. 65536 tokens x count skew
+0 .. 1 (0 = uniform K_base, 1 = 70% K_min / 30% K_max), forward only.
 Under torchrun each rank runs its own batch on its own GPU (weak scaling, no
 data-path collective; a barrier and a max-reduce of the times only).
 """
@@ -51,7 +56,11 @@ def parse():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="reflex", choices=["reflex", "reference"])
-    ap.add_argument("--config", default="llada_moe", choices=sorted(W.CONFIGS))
+    ap.add_argument("--config", default="llada_moe",
+                    choices=sorted(W.CONFIGS) + ["llada_moe_stack16"])
+    ap.add_argument("--sweep", action="store_true",
+                    help="token-count x count-skew sweep on the LLaDA2.0-mini "
+                         "layer (one JSON line per point)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -396,9 +405,188 @@ def run_gpu(args, cfg, rank, world, local_rank):
     print(json.dumps(line), flush=True)
 
 
+# ---------------------------------------------------------------------------
+# 16-layer stack and sweep (GPU)
+# ---------------------------------------------------------------------------
+STACK_LAYERS = 16
+
+
+def _device_weights(cfg, seed, dev, std):
+    """Random-init bf16 weights of one layer drawn on the device (seeded)."""
+    import torch
+    g = torch.Generator(device=dev)
+    g.manual_seed(int(seed))
+    E, d, I = cfg.E, cfg.d, cfg.inter
+
+    def rnd(*shape):
+        return (torch.randn(*shape, generator=g, device=dev, dtype=torch.float32)
+                * std).to(torch.bfloat16)
+    return dict(w_router=rnd(E, d), w_gate_up=rnd(E, 2 * I, d), w_down=rnd(E, d, I))
+
+
+def run_stack(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    from paper_2608_01784_gb300 import _binding as B
+    from paper_2608_01784_gb300 import api, build
+
+    build.build()
+    B.load()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    cfg = W.CONFIGS["llada_moe_b32"]
+    seed = args.seed + rank
+    T, d, E, I, km = cfg.T, cfg.d, cfg.E, cfg.inter, cfg.k_max
+    state = api.state_to_device(W.make_state(cfg, seed), dev)
+    h0 = api.layer_to_device({"hidden": W.make_layer(cfg.with_(E=1, inter=64), seed)["hidden"]},
+                             cfg.dtype, dev)["hidden"]
+    layers = [_device_weights(cfg, 1000 * seed + l, dev, cfg.weight_std)
+              for l in range(STACK_LAYERS)]
+    # one workspace serves every layer (layers run one after another)
+    moe = api.MoELayer(layers[0], dtype=cfg.dtype, d=d, E=E, inter=I, shared_inter=0,
+                       k_max=km, max_tokens=T, device=dev)
+    bufs = [torch.empty_like(h0), torch.empty_like(h0)]
+    stream = torch.cuda.current_stream(dev)
+    k_buf = torch.empty(T, dtype=torch.int32, device=dev)
+    k_sum = torch.zeros(1, dtype=torch.int64, device=dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    F = B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_FLAG_RESIDUAL
+
+    def forward(params):
+        api.allocate(state, params, E, stream, k_buf, k_sum, st)
+        h = h0
+        for l, w in enumerate(layers):
+            moe.w = w
+            moe.forward(h, k_buf, bufs[l & 1], F)
+            h = bufs[l & 1]
+
+    def timed(params, steps, warmup):
+        for _ in range(warmup):
+            forward(params)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(steps):
+            forward(params)
+        b.record(stream)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+        ms = a.elapsed_time(b) / steps
+        if world > 1:
+            t = torch.tensor([ms], dtype=torch.float64, device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms = float(t.item())
+        return ms
+
+    p_reflex = B.make_params(**cfg.alloc_params())
+    p_fixed = B.make_params(**cfg.alloc_params(delta_role=0, delta_cur=0))
+    forward(p_reflex)
+    torch.cuda.synchronize(dev)
+    assert B.reflex_read_status(st) == B.REFLEX_OK and moe.status() == B.REFLEX_OK
+    pairs = int(k_sum.item())
+    forward(p_fixed)
+    torch.cuda.synchronize(dev)
+    pairs_fixed = int(k_sum.item())
+    clk = ClockSampler(local_rank)
+    clk.start()
+    ms = timed(p_reflex, args.steps, args.warmup)
+    clocks = clk.stop()
+    ms_fixed = timed(p_fixed, max(1, args.steps // 2), 2)
+    if rank != 0:
+        return
+    peaks = load_peaks()
+    L = STACK_LAYERS
+    flops = 6.0 * d * I * pairs * L
+    flops_fixed = 6.0 * d * I * pairs_fixed * L
+    line = dict(
+        metric=METRIC, value=T * world / (ms * 1e-3), unit="tokens/s", n_gpus=world,
+        steps=args.steps, warmup=args.warmup, ms_per_step=ms, higher_is_better=True,
+        scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic",
+        config=dict(workload="llada_moe_stack16",
+                    description=f"{L} LLaDA-MoE-shaped layers (d=2048, E=64, inter=1024), "
+                                f"batch 32 x 1024 tokens, counts allocated once per forward, "
+                                f"residual h <- h + MoE(h), weights drawn on the device",
+                    tokens_per_step=T, layers=L, parallelism=f"replicas{world}",
+                    l2="no flush: 12.9 GB of expert weights stream every step"),
+        expert_tflops=flops * world / (ms * 1e-3) / 1e12,
+        expert_frac_of_bf16_peak=flops / (ms * 1e-3) / 1e12 / peaks["bf16_sustained"],
+        avg_k=pairs / T, pairs_per_layer=pairs,
+        fixed_topk=dict(k=cfg.k_base, pairs_per_layer=pairs_fixed, ms_per_step=ms_fixed,
+                        value=T * world / (ms_fixed * 1e-3),
+                        expert_tflops=flops_fixed * world / (ms_fixed * 1e-3) / 1e12),
+        gpu_launches=args.steps * (1 + 10 * L),
+        clocks=dict(sm_mhz=clocks["sm_mhz"], sm_max_mhz=clocks["sm_max_mhz"],
+                    reasons=clocks["reasons"], samples=clocks["samples"]),
+        peak_source=peaks["source"] + " (sustained bf16, long step)")
+    print(json.dumps(line), flush=True)
+
+
+def run_sweep(args, rank, world, local_rank):
+    import torch
+    from paper_2608_01784_gb300 import _binding as B
+    from paper_2608_01784_gb300 import api, build
+
+    build.build()
+    B.load()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    cfg = W.CONFIGS["llada2_mini"]
+    Tmax = 65536
+    d, E, I, S, km = cfg.d, cfg.E, cfg.inter, cfg.shared_inter, cfg.k_max
+    layer = W.make_layer(cfg, args.seed, T=Tmax)
+    dl = api.layer_to_device(layer, cfg.dtype, dev)
+    moe = api.MoELayer(dl, dtype=cfg.dtype, d=d, E=E, inter=I, shared_inter=S,
+                       k_max=km, max_tokens=Tmax, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    peaks = load_peaks()
+    F = B.REFLEX_FLAG_RENORM_TOPK
+    T = 256
+    while T <= Tmax:
+        h = dl["hidden"][:T]
+        out = torch.empty((T, d), dtype=moe.tdtype, device=dev)
+        base_ms = None
+        for skew in (0.0, 0.25, 0.5, 0.75, 1.0):
+            k = torch.from_numpy(W.skewed_k(T, skew, cfg.k_min, cfg.k_base, km,
+                                            seed=args.seed)).to(dev)
+            moe.forward(h, k, out, F)
+            torch.cuda.synchronize(dev)
+            assert moe.status() == B.REFLEX_OK
+            counts = moe.record()["counts"].cpu().numpy()
+            pairs = int(counts.sum())
+            steps = max(5, min(200, int(2e5 // T) + 5))
+            for _ in range(3):
+                moe.forward(h, k, out, F)
+            torch.cuda.synchronize(dev)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(steps):
+                moe.forward(h, k, out, F)
+            b.record(stream)
+            torch.cuda.synchronize(dev)
+            ms = a.elapsed_time(b) / steps
+            if skew == 0.0:
+                base_ms = ms
+            touched = int((counts > 0).sum())
+            bytes_ = (touched * 3 * I * d + 3 * S * d + 2 * T * d + E * d) * 2
+            flops = 6.0 * d * I * pairs + 6.0 * d * S * T
+            t_roof = max(bytes_ / (peaks["hbm"] * 1e9), flops / (peaks["bf16"] * 1e12))
+            line = dict(sweep="llada2_mini", tokens=T, skew=skew, avg_k=pairs / T,
+                        pairs=pairs, ms=ms, tokens_per_s=T / (ms * 1e-3),
+                        expert_tflops=6.0 * d * I * pairs / (ms * 1e-3) / 1e12,
+                        roofline_frac=t_roof / (ms * 1e-3),
+                        bound="hbm" if bytes_ / (peaks["hbm"] * 1e9) >= flops / (peaks["bf16"] * 1e12) else "tensor",
+                        load_imbalance=float(counts.max() / max(counts.mean(), 1e-9)),
+                        vs_uniform_kbase=ms / base_ms)
+            print(json.dumps(line), flush=True)
+        T *= 2
+
+
 def main():
     args = parse()
-    cfg = W.CONFIGS[args.config]
+    cfg = W.CONFIGS.get(args.config, W.CONFIGS["llada_moe_b32"])
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
@@ -412,6 +600,11 @@ def main():
     try:
         if args.impl == "reference":
             run_reference(args, cfg, rank, world)
+        elif args.sweep:
+            if rank == 0:
+                run_sweep(args, rank, world, local_rank)
+        elif args.config == "llada_moe_stack16":
+            run_stack(args, rank, world, local_rank)
         else:
             run_gpu(args, cfg, rank, world, local_rank)
     finally:

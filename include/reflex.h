@@ -61,6 +61,9 @@ extern "C" {
 /* bf16 only: run the expert GEMMs on the SIMT kernels instead of the
  * tcgen05/TMEM kernels (cross-checking; the fp32 path always uses SIMT). */
 #define REFLEX_FLAG_SIMT_EXPERTS 0x2u
+/* Residual connection for stacked layers: out = hidden + MoE(hidden), summed
+ * in fp32 with the expert outputs and rounded once. */
+#define REFLEX_FLAG_RESIDUAL 0x4u
 /* Stage selection.  No stage bit = all five stages in order.  Stages read
  * what the previous stages left in the same workspace; running a stage whose
  * predecessors did not run on that workspace gives unspecified values (every

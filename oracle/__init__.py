@@ -15,6 +15,9 @@ file's header lists which paper passage each function follows:
 * ``select``          TopK of Eq. 2 and the normalised router weight.
 * ``permutation``     (expert, token)-ordered pair list that executes Eq. 2.
 * ``moe_tokens``      Eq. 2 with SwiGLU experts (+ shared expert), fp64.
+* ``moe_stack``       a stack of such layers with the residual update
+                      h <- bf16(h + MoE(h)), the per-token counts shared by
+                      every layer (Sec. 3.3).
 
 Parity unpinned: none of the functions above (see tests/test_oracle_pins.py);
 the paper-level AvgK / pair-reduction numbers of Table 1 need the paper's
@@ -90,6 +93,10 @@ def _load():
                                       i32, i32, i32, i32, p]
     lib.oracle_num_threads.restype = ctypes.c_int
     lib.oracle_num_threads.argtypes = []
+    lib.oracle_bf16_from_f64_n.restype = None
+    lib.oracle_bf16_from_f64_n.argtypes = [p, ctypes.c_int64, p]
+    lib.oracle_residual_bf16.restype = None
+    lib.oracle_residual_bf16.argtypes = [p, p, ctypes.c_int64, p]
     _lib = lib
     return lib
 
@@ -241,3 +248,41 @@ def moe_layer(hidden, w_router, w_gate_up, w_down, k, k_max, *, tokens=None,
                      shared_gate_up=shared_gate_up, shared_down=shared_down)
     return dict(z=z, ids=ids, alpha=alpha, offsets=offsets, perm=perm,
                 row_of=row_of, tokens=np.asarray(tokens, np.int32), out=out)
+
+
+def bf16_from_f64(x) -> np.ndarray:
+    """Round fp64 values to bf16 (nearest, ties to even); uint16 bits."""
+    x = _c(x, np.float64)
+    out = np.empty(x.shape, np.uint16)
+    _load().oracle_bf16_from_f64_n(_ptr(x), x.size, _ptr(out))
+    return out
+
+
+def residual_bf16(h_bits: np.ndarray, out: np.ndarray) -> np.ndarray:
+    """bf16(h + out) for bf16 bits h and an fp64 layer output."""
+    h_bits = _c(h_bits, np.uint16)
+    out = _c(out, np.float64)
+    assert h_bits.shape == out.shape
+    nxt = np.empty_like(h_bits)
+    _load().oracle_residual_bf16(_ptr(h_bits), _ptr(out), h_bits.size, _ptr(nxt))
+    return nxt
+
+
+def moe_stack(hidden_bits: np.ndarray, layers: list, k, k_max: int,
+              renorm: bool = True) -> list:
+    """Layer by layer: res_l = Eq. 2 on h_l with layer l's weights and the
+    shared counts k; h_{l+1} = bf16(h_l + res_l.out).  Returns one dict per
+    layer with its input h (bf16 bits), routing record and output h."""
+    h = np.ascontiguousarray(hidden_bits, np.uint16)
+    trace = []
+    for lay in layers:
+        res = moe_layer(h, lay["w_router"], lay["w_gate_up"], lay["w_down"], k,
+                        k_max, renorm=renorm,
+                        shared_gate_up=lay.get("shared_gate_up"),
+                        shared_down=lay.get("shared_down"))
+        nxt = residual_bf16(h, res["out"])
+        res["h_in"] = h
+        res["h_out"] = nxt
+        trace.append(res)
+        h = nxt
+    return trace

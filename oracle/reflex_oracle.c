@@ -409,3 +409,33 @@ void oracle_fps_n(const float* c1, const float* c2, const uint8_t* hist,
     for (int64_t i = 0; i < n; ++i)
         s[i] = oracle_fps(c1[i], c2[i], hist[i], theta, w_cf, v_ref, tau);
 }
+
+/* ------------------------------------------------------------------------ */
+/* Rounding to bf16 (8 significant bits, fp32 exponent range), nearest with  */
+/* ties to even, from fp64: x = m 2^e with m in [0.5, 1); the significand    */
+/* m 2^8 is rounded to an integer in the current (nearest-even) mode.        */
+/* ------------------------------------------------------------------------ */
+static uint16_t or_bf16_from_f64(double x) {
+    if (x != x) return 0x7FC0;
+    if (x == 0.0) return signbit(x) ? 0x8000 : 0x0000;
+    int e;
+    double m = frexp(x, &e);            /* |m| in [0.5, 1) */
+    double q = rint(ldexp(m, 8));       /* 8 significant bits */
+    double r = ldexp(q, e - 8);         /* exactly a bf16 value (normal range) */
+    float f = (float)r;                 /* exact */
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    return (uint16_t)(u >> 16);
+}
+
+void oracle_bf16_from_f64_n(const double* x, int64_t n, uint16_t* out) {
+    for (int64_t i = 0; i < n; ++i) out[i] = or_bf16_from_f64(x[i]);
+}
+
+/* Residual update of a stacked layer: next = bf16(h + out) (h bf16 bits,   */
+/* out the fp64 layer output).                                             */
+void oracle_residual_bf16(const uint16_t* h, const double* out, int64_t n,
+                          uint16_t* next) {
+    for (int64_t i = 0; i < n; ++i)
+        next[i] = or_bf16_from_f64((double)or_bf16_to_f32(h[i]) + out[i]);
+}

@@ -8,6 +8,7 @@ CPU fallback: loading fails loudly when the library is missing.
 """
 from ._binding import (  # noqa: F401
     REFLEX_DTYPE_BF16, REFLEX_DTYPE_F32, REFLEX_FLAG_RENORM_TOPK,
+    REFLEX_FLAG_RESIDUAL,
     REFLEX_FLAG_SIMT_EXPERTS, REFLEX_OK, REFLEX_STAGE_COMBINE,
     REFLEX_STAGE_DISPATCH, REFLEX_STAGE_EXPERT_DOWN, REFLEX_STAGE_EXPERT_UP,
     REFLEX_STAGE_ROUTE,

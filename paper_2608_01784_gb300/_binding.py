@@ -26,6 +26,7 @@ REFLEX_DTYPE_BF16 = 1
 
 REFLEX_FLAG_RENORM_TOPK = 0x1
 REFLEX_FLAG_SIMT_EXPERTS = 0x2
+REFLEX_FLAG_RESIDUAL = 0x4
 REFLEX_STAGE_ROUTE = 0x100
 REFLEX_STAGE_DISPATCH = 0x200
 REFLEX_STAGE_EXPERT_UP = 0x400

@@ -1,5 +1,6 @@
 // combine.cu — the weighted sum of Eq. 2 (REFLEX Sec. 3.2) back in token
-// order: out_t = sum_{j < k_t} alpha[t, j] * y[row_of[t, j]] (+ shared_t).
+// order: out_t = sum_{j < k_t} alpha[t, j] * y[row_of[t, j]] (+ shared_t)
+// (+ resid_t, the layer input, for stacked layers).
 //
 // Each thread owns 8 consecutive columns of one token (d / 8 threads per
 // token, 256 threads per CTA), so every load and store is one 16-byte (bf16)
@@ -20,7 +21,7 @@ constexpr int kMaxK = 32;
 template <typename Te>
 __global__ void __launch_bounds__(kThreads)
     combine_kernel(const Te* __restrict__ y, const Te* __restrict__ ysh,
-                   const int32_t* __restrict__ row_of,
+                   const Te* __restrict__ resid, const int32_t* __restrict__ row_of,
                    const float* __restrict__ alpha, const int32_t* __restrict__ k,
                    int T, int d, int k_max, int cap_rows, Te* __restrict__ out,
                    uint32_t* __restrict__ err) {
@@ -83,6 +84,12 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i] += v[i];
   }
+  if (resid != nullptr) {
+    float v[8];
+    load8(resid + static_cast<int64_t>(t) * d + c, v);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i] += v[i];
+  }
   store8(out + static_cast<int64_t>(t) * d + c, acc);
 }
 
@@ -90,7 +97,7 @@ __global__ void __launch_bounds__(kThreads)
 template <typename Te>
 __global__ void __launch_bounds__(kThreads)
     combine_wide_kernel(const Te* __restrict__ y, const Te* __restrict__ ysh,
-                        const int32_t* __restrict__ row_of,
+                        const Te* __restrict__ resid, const int32_t* __restrict__ row_of,
                         const float* __restrict__ alpha,
                         const int32_t* __restrict__ k, int T, int d, int k_max,
                         int cap_rows, Te* __restrict__ out,
@@ -125,23 +132,29 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
       for (int i = 0; i < 8; ++i) acc[i] += v[i];
     }
+    if (resid != nullptr) {
+      float v[8];
+      load8(resid + static_cast<int64_t>(t) * d + c, v);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] += v[i];
+    }
     store8(out + static_cast<int64_t>(t) * d + c, acc);
   }
 }
 
 template <typename Te>
-cudaError_t launch_typed(const Te* y, const Te* ysh, const int32_t* row_of,
+cudaError_t launch_typed(const Te* y, const Te* ysh, const Te* resid, const int32_t* row_of,
                          const float* alpha, const int32_t* k, int T, int d,
                          int k_max, int cap_rows, Te* out, uint32_t* err,
                          cudaStream_t stream) {
   if (d <= 2048 && kThreads % (d / 8) == 0) {
     const int tok_per_cta = kThreads / (d / 8);
     const int grid = (T + tok_per_cta - 1) / tok_per_cta;
-    combine_kernel<Te><<<grid, kThreads, 0, stream>>>(y, ysh, row_of, alpha, k, T,
+    combine_kernel<Te><<<grid, kThreads, 0, stream>>>(y, ysh, resid, row_of, alpha, k, T,
                                                       d, k_max, cap_rows, out, err);
   } else {
     combine_wide_kernel<Te><<<(T + 7) / 8, kThreads, 0, stream>>>(
-        y, ysh, row_of, alpha, k, T, d, k_max, cap_rows, out, err);
+        y, ysh, resid, row_of, alpha, k, T, d, k_max, cap_rows, out, err);
   }
   return cudaGetLastError();
 }
@@ -149,17 +162,19 @@ cudaError_t launch_typed(const Te* y, const Te* ysh, const int32_t* row_of,
 }  // namespace
 
 cudaError_t launch_combine(int dtype, const void* y, const void* y_shared,
-                           const int32_t* row_of, const float* alpha,
+                           const void* resid, const int32_t* row_of, const float* alpha,
                            const int32_t* k, int T, int d, int k_max,
                            int cap_rows, void* out, uint32_t* err, int,
                            cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
   if (dtype == 0)
     return launch_typed(static_cast<const float*>(y),
-                        static_cast<const float*>(y_shared), row_of, alpha, k, T,
+                        static_cast<const float*>(y_shared),
+                        static_cast<const float*>(resid), row_of, alpha, k, T,
                         d, k_max, cap_rows, static_cast<float*>(out), err, stream);
   return launch_typed(static_cast<const __nv_bfloat16*>(y),
-                      static_cast<const __nv_bfloat16*>(y_shared), row_of, alpha,
+                      static_cast<const __nv_bfloat16*>(y_shared),
+                      static_cast<const __nv_bfloat16*>(resid), row_of, alpha,
                       k, T, d, k_max, cap_rows, static_cast<__nv_bfloat16*>(out),
                       err, stream);
 }

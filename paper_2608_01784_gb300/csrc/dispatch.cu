@@ -12,8 +12,8 @@
 //           tile counts = tile prefix for the grouped GEMM;
 //   scatter rebuilds the block's masks; the row of pair (t, j) is
 //           offsets[e] + block prefix + popcount of lower tokens' bits.
-// A fourth launch gathers X rows into pair order (one warp per pair row,
-// 16-byte vectors).
+// A fourth launch gathers X rows into pair order (one warp per token: the
+// hidden row is read once and written to each of its pair rows).
 #include "common.cuh"
 #include "internal.h"
 
@@ -149,27 +149,49 @@ __global__ void __launch_bounds__(kBlk)
   }
 }
 
+// Token-order gather: one warp per token reads the token's hidden row once
+// (up to 8 16-byte vectors per lane in flight) and writes it to each of the
+// token's k_t pair rows, so every hidden row crosses HBM once however many
+// experts selected it.
 template <typename Te>
 __global__ void __launch_bounds__(256)
-    gather_kernel(const Te* __restrict__ x, const int32_t* __restrict__ perm,
-                  const int32_t* __restrict__ totals, int k_max, int cap_rows,
-                  int T, int d, Te* __restrict__ xp, uint32_t* __restrict__ err) {
+    gather_kernel(const Te* __restrict__ x, const int32_t* __restrict__ row_of,
+                  const int32_t* __restrict__ k, int k_max, int cap_rows, int T,
+                  int d, Te* __restrict__ xp, uint32_t* __restrict__ err) {
+  constexpr int kVecElems = 16 / sizeof(Te);  // elements per 16-byte vector
+  constexpr int kMaxVec = 8;                  // vectors per lane per pass
   const int lane = threadIdx.x & 31;
-  int n = totals[0];
-  if (n > cap_rows) {
-    if (threadIdx.x == 0 && blockIdx.x == 0) set_err(err, kErrIndex);
-    n = cap_rows;
-  }
   const int warps = gridDim.x * 8;
-  for (int p = blockIdx.x * 8 + (threadIdx.x >> 5); p < n; p += warps) {
-    const int t = perm[p] / k_max;
-    if (t < 0 || t >= T) continue;
-    const Te* src = x + static_cast<int64_t>(t) * d;
-    Te* dst = xp + static_cast<int64_t>(p) * d;
-    float v[8];
-    for (int c = lane * 8; c < d; c += 256) {
-      load8(src + c, v);
-      store8(dst + c, v);
+  const int row_vecs = d / kVecElems;
+  for (int t = blockIdx.x * 8 + (threadIdx.x >> 5); t < T; t += warps) {
+    int kt = k[t];
+    kt = kt < 1 ? 1 : (kt > k_max ? k_max : kt);
+    int my_row = -1;
+    if (lane < kt) {
+      my_row = row_of[static_cast<int64_t>(t) * k_max + lane];
+      if (my_row >= cap_rows) {
+        set_err(err, kErrIndex);
+        my_row = -1;
+      }
+    }
+    const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(t) * d);
+    for (int base = 0; base < row_vecs; base += 32 * kMaxVec) {
+      uint4 v[kMaxVec];
+#pragma unroll
+      for (int i = 0; i < kMaxVec; ++i) {
+        const int q = base + lane + 32 * i;
+        if (q < row_vecs) v[i] = __ldg(src + q);
+      }
+      for (int j = 0; j < kt; ++j) {
+        const int r = __shfl_sync(0xffffffffu, my_row, j);
+        if (r < 0) continue;
+        uint4* dst = reinterpret_cast<uint4*>(xp + static_cast<int64_t>(r) * d);
+#pragma unroll
+        for (int i = 0; i < kMaxVec; ++i) {
+          const int q = base + lane + 32 * i;
+          if (q < row_vecs) dst[q] = v[i];
+        }
+      }
     }
   }
 }
@@ -196,22 +218,21 @@ cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T, int E,
   return cudaGetLastError();
 }
 
-cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* perm,
-                               const int32_t* totals, int k_max, int cap_rows,
-                               int d, void* x_perm, int num_sms,
+cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* row_of,
+                               const int32_t* k, int T, int k_max, int cap_rows,
+                               int d, void* x_perm, uint32_t* err, int num_sms,
                                cudaStream_t stream) {
-  if (cap_rows == 0) return cudaSuccess;
-  const int T = cap_rows / k_max;
-  int grid = (cap_rows + 7) / 8;
+  if (T == 0) return cudaSuccess;
+  int grid = (T + 7) / 8;
   if (grid > 16 * num_sms) grid = 16 * num_sms;
   if (dtype == 0)
     gather_kernel<float><<<grid, 256, 0, stream>>>(
-        static_cast<const float*>(hidden), perm, totals, k_max, cap_rows, T, d,
-        static_cast<float*>(x_perm), nullptr);
+        static_cast<const float*>(hidden), row_of, k, k_max, cap_rows, T, d,
+        static_cast<float*>(x_perm), err);
   else
     gather_kernel<__nv_bfloat16><<<grid, 256, 0, stream>>>(
-        static_cast<const __nv_bfloat16*>(hidden), perm, totals, k_max,
-        cap_rows, T, d, static_cast<__nv_bfloat16*>(x_perm), nullptr);
+        static_cast<const __nv_bfloat16*>(hidden), row_of, k, k_max, cap_rows, T,
+        d, static_cast<__nv_bfloat16*>(x_perm), err);
   return cudaGetLastError();
 }
 

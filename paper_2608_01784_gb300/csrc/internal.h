@@ -52,11 +52,11 @@ constexpr int kDispatchBlock = 256;  // tokens per dispatch block
 cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T,
                             int E, int k_max, const DispatchBufs& b,
                             cudaStream_t stream);
-// X_perm[p] = X[perm[p] / k_max] for p < total_pairs.
-cudaError_t launch_gather_rows(int dtype, const void* hidden,
-                               const int32_t* perm, const int32_t* totals,
-                               int k_max, int cap_rows, int d, void* x_perm,
-                               int num_sms, cudaStream_t stream);
+// X_perm[row_of[t, j]] = X[t] for j < k_t.
+cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* row_of,
+                               const int32_t* k, int T, int k_max, int cap_rows,
+                               int d, void* x_perm, uint32_t* err, int num_sms,
+                               cudaStream_t stream);
 
 // ---- experts: SIMT grouped GEMMs (experts_simt.cu) ------------------------
 // Grouped mode: rows [offsets[e], offsets[e+1]) use expert e; dense mode
@@ -101,9 +101,9 @@ int tc_n_granule(bool swiglu, int bn);  // output columns per tile
 int tc_pick_bn(bool swiglu, int n_total, int64_t mtiles_est, int num_sms);
 
 // ---- combine (combine.cu) -------------------------------------------------
-// out[t] = sum_{j<k_t} alpha[t,j] * y[row_of[t,j]] (+ y_shared[t]).
+// out[t] = sum_{j<k_t} alpha[t,j] * y[row_of[t,j]] (+ y_shared[t]) (+ resid[t]).
 cudaError_t launch_combine(int dtype, const void* y, const void* y_shared,
-                           const int32_t* row_of, const float* alpha,
+                           const void* resid, const int32_t* row_of, const float* alpha,
                            const int32_t* k, int T, int d, int k_max,
                            int cap_rows, void* out, uint32_t* err, int num_sms,
                            cudaStream_t stream);

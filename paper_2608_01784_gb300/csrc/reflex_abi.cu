@@ -276,8 +276,8 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
                        I32(L.offsets),   I32(L.mt_prefix), I32(L.perm),
                        I32(L.row_of),    totals,          err};
     RX_CUDA(rx::launch_dispatch(I32(L.ids), k, T, E, k_max, b, s));
-    RX_CUDA(rx::launch_gather_rows(dtype, hidden, I32(L.perm), totals, k_max,
-                                   cap, d, xperm, sms, s));
+    RX_CUDA(rx::launch_gather_rows(dtype, hidden, I32(L.row_of), k, T, k_max, cap, d,
+                                   xperm, err, sms, s));
   }
   const bool up = (stages & REFLEX_STAGE_EXPERT_UP) != 0;
   const bool down = (stages & REFLEX_STAGE_EXPERT_DOWN) != 0;
@@ -312,7 +312,8 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
            !make_map(&sb1, shared_gate_up, 2 * static_cast<int64_t>(shared_inter), d,
                      rx::tc_b_box_rows(true, bn_sup)) ||
            !make_map(&sa2, ash, T, shared_inter, rx::kTileM) ||
-           !make_map(&sb2, shared_down, d, shared_inter, rx::tc_b_box_rows(false, bn_sdn))))
+           !make_map(&sb2, shared_down, d, shared_inter,
+                     rx::tc_b_box_rows(false, bn_sdn))))
         return REFLEX_ECUDA;
       rx::TcGemmArgs h1{&sa1, &sb1, d, shared_inter, 2 * shared_inter, shared_inter,
                         dense, ash, shared_inter, err, sms};
@@ -328,7 +329,8 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
     }
   }
   if (stages & REFLEX_STAGE_COMBINE) {
-    RX_CUDA(rx::launch_combine(dtype, xperm, ysh, I32(L.row_of), alpha, k, T, d,
+    const void* resid = (flags & REFLEX_FLAG_RESIDUAL) ? hidden : nullptr;
+    RX_CUDA(rx::launch_combine(dtype, xperm, ysh, resid, I32(L.row_of), alpha, k, T, d,
                                k_max, cap, out, err, sms, s));
   }
   return REFLEX_OK;

@@ -100,3 +100,32 @@ def check_routing(rec: dict, ref: dict, k: np.ndarray, E: int):
     counts = np.diff(ref["offsets"])
     assert np.array_equal(rec["counts"], counts)
     assert int(rec["totals"][1]) == int(((counts + 127) // 128).sum())
+
+
+def check_sampled_routing(rec: dict, layer: dict, k: np.ndarray, k_max: int,
+                          tokens: np.ndarray, renorm: bool = True):
+    """Routing of the listed tokens against the oracle run on those tokens
+    only (scores are per token), plus properties of the whole record."""
+    z = oracle.router_logits(layer["hidden"][tokens], layer["w_router"])
+    ids, alpha = oracle.select(z, k[tokens], k_max, renorm)
+    assert np.array_equal(rec["ids"][tokens], ids), "selected experts differ"
+    valid = ids >= 0
+    np.testing.assert_allclose(rec["alpha"][tokens][valid], alpha[valid],
+                               rtol=ALPHA_RTOL, atol=1e-7)
+    # whole record: pairs = sum k; perm is a permutation of the used slots
+    # and row_of is its inverse; rows are grouped by expert in token order
+    T = k.size
+    n = int(k.sum())
+    assert int(rec["totals"][0]) == n and rec["offsets"][-1] == n
+    perm = rec["perm"]
+    assert perm.size == n
+    used = (np.arange(k_max)[None, :] < k[:, None]).ravel()
+    assert np.array_equal(np.sort(perm), np.nonzero(used)[0])
+    row_of = rec["row_of"].ravel()
+    assert np.array_equal(row_of[perm], np.arange(n))
+    assert np.all(row_of[~used] == -1)
+    ids_all = rec["ids"].ravel()
+    for e in range(len(rec["offsets"]) - 1):
+        rows = perm[rec["offsets"][e]:rec["offsets"][e + 1]]
+        assert np.all(ids_all[rows] == e)
+        assert np.all(np.diff(rows) > 0)

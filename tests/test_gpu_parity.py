@@ -258,3 +258,91 @@ def test_forward_stages_compose():
                        flags=B.REFLEX_FLAG_RENORM_TOPK | st)
     torch.cuda.synchronize()
     assert np.array_equal(G.to_f32(out), full)
+
+
+# ---------------------------------------------------------------------------
+# stacked layers (shared counts, residual h <- bf16(h + MoE(h)))
+# ---------------------------------------------------------------------------
+def test_stack_layerwise_residual():
+    """Each GPU layer runs on the oracle's input of that layer (so routing is
+    comparable bit for bit in every layer); its bf16 output must match the
+    oracle's residual update within the bf16 tolerance."""
+    T, d, E, I, km = 256, 256, 16, 128, 4
+    cfg, lay0 = _bf16_case(T, d, E, I, 0, km, seed=21)
+    layers = [W.make_layer(cfg, 100 + l, T=T) for l in range(3)]
+    rng = np.random.default_rng(4)
+    k = rng.integers(1, km + 1, T).astype(np.int32)
+    trace = oracle.moe_stack(layers[0]["hidden"], layers, k, km)
+    for l, res in enumerate(trace):
+        lay = dict(layers[l], hidden=res["h_in"])
+        gl = G.GpuLayer(cfg, lay)
+        out, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK |
+                                      B.REFLEX_FLAG_RESIDUAL)
+        assert status == B.REFLEX_OK
+        G.check_routing(rec, res, k, E)
+        ref = W.bf16_bits_to_f32(res["h_out"]).astype(np.float64)
+        rel, mx = G.out_errors(out, ref)
+        assert rel <= G.BF16_REL_L2 and mx <= 2 * G.BF16_MAX_ABS, (l, rel, mx)
+
+
+def test_forward_llada_moe_b32_sampled():
+    """One layer of the 16-layer stack at full size (32 x 1024 tokens), with
+    the residual connection; routing on sampled tokens plus whole-record
+    properties, outputs on sampled tokens."""
+    cfg = CFG["llada_moe_b32"]
+    layer = W.make_layer(cfg, 0)
+    state = W.make_state(cfg, 0)
+    k = G.oracle_allocate(state, G.params_of(cfg))
+    tokens = W.sample_tokens(state, stride=97)
+    gl = G.GpuLayer(cfg, layer)
+    out, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK |
+                                  B.REFLEX_FLAG_RESIDUAL)
+    assert status == B.REFLEX_OK
+    G.check_sampled_routing(rec, layer, k, cfg.k_max, tokens)
+    sub = dict(layer, hidden=layer["hidden"][tokens])
+    ids, alpha = oracle.select(oracle.router_logits(sub["hidden"], layer["w_router"]),
+                               k[tokens], cfg.k_max)
+    ref = oracle.moe_tokens(sub["hidden"], layer["w_gate_up"], layer["w_down"], ids,
+                            alpha, k[tokens], np.arange(tokens.size, dtype=np.int32))
+    ref = ref + W.bf16_bits_to_f32(sub["hidden"]).astype(np.float64)
+    rel, mx = G.out_errors(out[tokens], ref)
+    assert rel <= G.BF16_REL_L2 and mx <= 2 * G.BF16_MAX_ABS, (rel, mx)
+
+
+# ---------------------------------------------------------------------------
+# token-count and count-skew sweep on the LLaDA2.0-mini layer shape
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("skew", [0.0, 0.5, 1.0])
+def test_sweep_small_batch_full(skew):
+    cfg = CFG["llada2_mini"]
+    T = 256
+    layer = W.make_layer(cfg, 7, T=T)
+    k = W.skewed_k(T, skew, cfg.k_min, cfg.k_base, cfg.k_max, seed=7)
+    gl = G.GpuLayer(cfg, layer)
+    out, rec, status = gl.forward(k)
+    assert status == B.REFLEX_OK
+    ref = G.oracle_layer(cfg, layer, k)
+    G.check_routing(rec, ref, k, cfg.E)
+    rel, mx = G.out_errors(out, ref["out"])
+    assert rel <= G.BF16_REL_L2 and mx <= G.BF16_MAX_ABS, (rel, mx)
+
+
+def test_sweep_max_batch_sampled():
+    cfg = CFG["llada2_mini"]
+    T = 65536
+    layer = W.make_layer(cfg, 8, T=T)
+    k = W.skewed_k(T, 1.0, cfg.k_min, cfg.k_base, cfg.k_max, seed=8)
+    gl = G.GpuLayer(cfg, layer)
+    out, rec, status = gl.forward(k)
+    assert status == B.REFLEX_OK
+    tokens = np.unique(np.concatenate([np.arange(0, T, 509), [T - 1]])).astype(np.int32)
+    G.check_sampled_routing(rec, layer, k, cfg.k_max, tokens)
+    ids, alpha = oracle.select(oracle.router_logits(layer["hidden"][tokens],
+                                                    layer["w_router"]),
+                               k[tokens], cfg.k_max)
+    ref = oracle.moe_tokens(layer["hidden"][tokens], layer["w_gate_up"], layer["w_down"],
+                            ids, alpha, k[tokens], np.arange(tokens.size, dtype=np.int32),
+                            shared_gate_up=layer["shared_gate_up"],
+                            shared_down=layer["shared_down"])
+    rel, mx = G.out_errors(out[tokens], ref)
+    assert rel <= G.BF16_REL_L2 and mx <= G.BF16_MAX_ABS, (rel, mx)

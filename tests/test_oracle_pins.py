@@ -517,3 +517,50 @@ def test_layer_bf16_inputs_widen_exactly():
                          W.bf16_bits_to_f32(gub), W.bf16_bits_to_f32(db), k, 4)
     for key in ("z", "ids", "alpha", "perm", "out"):
         assert np.array_equal(a[key], b[key])
+
+
+# --------------------------------------------------------------------------
+# bf16 rounding and the stacked-layer residual (reading: h <- bf16(h + out))
+# --------------------------------------------------------------------------
+def test_bf16_rounding_ties_and_library_agreement():
+    # halfway cases round to the even significand
+    one = 1.0
+    cases = [(one, 0x3F80), (one + 2.0 ** -8, 0x3F80), (one + 3 * 2.0 ** -8, 0x3F82),
+             (one + 2.0 ** -7, 0x3F81), (-(one + 2.0 ** -8), 0xBF80), (0.0, 0x0000),
+             (-0.0, 0x8000), (3.0, 0x4040)]
+    got = oracle.bf16_from_f64(np.array([c[0] for c in cases]))
+    assert got.tolist() == [c[1] for c in cases]
+    # fp32-representable values: agrees with torch's float -> bfloat16
+    x = np.random.default_rng(0).standard_normal(100000).astype(np.float32)
+    x = np.concatenate([x, x * 1e-20, x * 1e20])
+    assert np.array_equal(oracle.bf16_from_f64(x.astype(np.float64)), W.to_bf16_bits(x))
+
+
+def test_residual_update_closed_form():
+    h = W.to_bf16_bits(np.array([1.0, -2.0, 0.5, 3.0], np.float32))
+    out = np.array([0.25, 2.0, -0.5, 2.0 ** -9], np.float64)
+    nxt = W.bf16_bits_to_f32(oracle.residual_bf16(h, out))
+    assert nxt.tolist() == [1.25, 0.0, 0.0, 3.0]
+
+
+def test_stack_shares_counts_and_chains_inputs():
+    rng = np.random.default_rng(9)
+    T, d, E, I = 16, 32, 4, 16
+    h0 = W.to_bf16_bits(rng.standard_normal((T, d)).astype(np.float32))
+    layers = []
+    for _ in range(3):
+        layers.append(dict(
+            w_router=W.to_bf16_bits((0.3 * rng.standard_normal((E, d))).astype(np.float32)),
+            w_gate_up=W.to_bf16_bits((0.2 * rng.standard_normal((E, 2 * I, d))).astype(np.float32)),
+            w_down=W.to_bf16_bits((0.2 * rng.standard_normal((E, d, I))).astype(np.float32))))
+    k = rng.integers(1, 3, T).astype(np.int32)
+    tr = oracle.moe_stack(h0, layers, k, 2)
+    assert np.array_equal(tr[0]["h_in"], h0)
+    for a, b in zip(tr[:-1], tr[1:]):
+        assert np.array_equal(a["h_out"], b["h_in"])
+    for res in tr:
+        assert res["perm"].size == int(k.sum())          # same counts per layer
+    # a layer with zero down-projection leaves the stream unchanged
+    zero = dict(layers[0], w_down=np.zeros_like(layers[0]["w_down"]))
+    tr0 = oracle.moe_stack(h0, [zero], k, 2)
+    assert np.array_equal(tr0[0]["h_out"], h0)
