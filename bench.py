@@ -45,9 +45,11 @@ from paper_2608_01784_gb300 import workloads as W  # noqa: E402
 METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
           "fixed top-K")
 
-# Bytes moved by the dominant kernel per launch, from an ncu capture of the
-# current kernel (profiles/); None when the kernel changed since the capture.
-NCU_TRAFFIC_BYTES = None
+# DRAM bytes (read + write) moved per launch by the dominant kernel, from an
+# ncu capture of the current kernel on the same workload
+# (profiles/grouped_gemm_llada_moe_T1024.md); workloads without a capture of
+# the current kernel report null.
+NCU_TRAFFIC_BYTES = {"llada_moe": 568417024}
 
 
 def parse():
@@ -361,8 +363,8 @@ def run_gpu(args, cfg, rank, world, local_rank):
         tf = up_flops / (up_ms * 1e-3) / 1e12
         roof = dict(bound="tensor", achieved=tf, peak=peaks["bf16"],
                     unit="TFLOP/s", frac=tf / peaks["bf16"])
-    roof.update(kernel="grouped_gemm_kernel<256, SwiGLU> (gate/up + SwiGLU)",
-                traffic=NCU_TRAFFIC_BYTES, algorithmic_bytes=up_bytes,
+    roof.update(kernel="grouped_gemm_kernel, gate/up + SwiGLU (tcgen05)",
+                traffic=NCU_TRAFFIC_BYTES.get(cfg.name), algorithmic_bytes=up_bytes,
                 algorithmic_flops=up_flops, avg_launch_ms=up_ms,
                 peak_source=peaks["source"] + " (burst)")
     # layer roofline: all expert weights touched + hidden in/out vs Eq. 10 flops
