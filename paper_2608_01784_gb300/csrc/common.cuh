@@ -21,7 +21,8 @@ struct WsHeader {
   uint32_t err;          // device error word
   int32_t total_pairs;   // sum_i k_i after dispatch
   int32_t total_mtiles;  // sum_e ceil(count_e / 128) after dispatch
-  int32_t pad[61];
+  int32_t total_mtiles2; // sum_e ceil(count_e / 256) after dispatch
+  int32_t pad[60];
 };
 static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 

@@ -8,8 +8,8 @@
 //           (bit = token of the block selected the expert; a token selects
 //           an expert at most once) and its popcount per expert;
 //   scan    per expert, exclusive prefix over blocks; per-expert totals;
-//           exclusive prefix over experts = offsets, and over the 128-row
-//           tile counts = tile prefix for the grouped GEMM;
+//           exclusive prefix over experts = offsets, and over the 128- and
+//           256-row tile counts = tile prefixes for the grouped GEMMs;
 //   scatter rebuilds the block's masks; the row of pair (t, j) is
 //           offsets[e] + block prefix + popcount of lower tokens' bits.
 // A fourth launch gathers X rows into pair order (one warp per token: the
@@ -91,7 +91,7 @@ __global__ void __launch_bounds__(1024)
     scan_kernel(const int32_t* __restrict__ blk_count, int nblk, int E,
                 int32_t* __restrict__ blk_off, int32_t* __restrict__ counts,
                 int32_t* __restrict__ offsets, int32_t* __restrict__ mt_prefix,
-                int32_t* __restrict__ totals) {
+                int32_t* __restrict__ mt2_prefix, int32_t* __restrict__ totals) {
   __shared__ int s_warp[32];
   const int e = threadIdx.x;  // E <= 1024
   int run = 0;
@@ -107,15 +107,21 @@ __global__ void __launch_bounds__(1024)
   const int off = block_exclusive_scan(e < E ? run : 0, s_warp, &total_pairs);
   const int tiles = e < E ? (run + kTileM - 1) / kTileM : 0;
   const int toff = block_exclusive_scan(tiles, s_warp, &total_tiles);
+  int total_tiles2;  // 256-row tiles of the CTA-pair GEMM
+  const int tiles2 = e < E ? (run + 2 * kTileM - 1) / (2 * kTileM) : 0;
+  const int toff2 = block_exclusive_scan(tiles2, s_warp, &total_tiles2);
   if (e < E) {
     offsets[e] = off;
     mt_prefix[e] = toff;
+    mt2_prefix[e] = toff2;
   }
   if (e == 0) {
     offsets[E] = total_pairs;
     mt_prefix[E] = total_tiles;
+    mt2_prefix[E] = total_tiles2;
     totals[0] = total_pairs;
     totals[1] = total_tiles;
+    totals[2] = total_tiles2;
   }
 }
 
@@ -212,7 +218,7 @@ cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T, int E,
   }
   count_kernel<<<nblk, kBlk, smem, stream>>>(ids, k, T, E, k_max, b.blk_count, b.err);
   scan_kernel<<<1, 1024, 0, stream>>>(b.blk_count, nblk, E, b.blk_off, b.counts,
-                                      b.offsets, b.mt_prefix, b.totals);
+                                      b.offsets, b.mt_prefix, b.mt2_prefix, b.totals);
   scatter_kernel<<<nblk, kBlk, smem, stream>>>(ids, k, T, E, k_max, b.blk_off,
                                                b.offsets, b.perm, b.row_of, b.err);
   return cudaGetLastError();

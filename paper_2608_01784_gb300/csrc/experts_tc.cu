@@ -66,8 +66,9 @@ struct KParams {
   int b_rows_per_group;
   int b_up_offset;
   GroupRows g;
-  const int32_t* mt_prefix;  // [E+1] (grouped mode)
+  const int32_t* mt_prefix;  // [E+1] prefix of tile counts (grouped mode)
   int max_mtiles;            // host upper bound of m-tiles
+  int tile_rows;             // rows per tile: 128 (1-SM) or 256 (CTA pair)
   __nv_bfloat16* out;
   int ldo;
   uint32_t* err;
@@ -170,7 +171,7 @@ struct Tile {
 __device__ __forceinline__ int total_tiles(const KParams& p) {
   int mt;
   if (p.g.offsets == nullptr) {
-    mt = (p.g.dense_rows + BM - 1) / BM;
+    mt = (p.g.dense_rows + p.tile_rows - 1) / p.tile_rows;
   } else {
     mt = p.mt_prefix[p.g.E];
     if (mt < 0) mt = 0;
@@ -182,11 +183,11 @@ __device__ __forceinline__ int total_tiles(const KParams& p) {
 // Tile t -> (expert, n-tile, rows); false when the workspace is inconsistent.
 __device__ __forceinline__ bool decode_tile(const KParams& p, int t, Tile& o) {
   if (p.g.offsets == nullptr) {
-    const int mt = (p.g.dense_rows + BM - 1) / BM;
+    const int mt = (p.g.dense_rows + p.tile_rows - 1) / p.tile_rows;
     o.e = 0;
     o.n = t / mt;
-    o.row0 = (t % mt) * BM;
-    o.rows = min(BM, p.g.dense_rows - o.row0);
+    o.row0 = (t % mt) * p.tile_rows;
+    o.rows = min(p.tile_rows, p.g.dense_rows - o.row0);
     return true;
   }
   int lo = 0, hi = p.g.E;  // n_tiles*prefix[lo] <= t < n_tiles*prefix[hi]
@@ -199,8 +200,8 @@ __device__ __forceinline__ bool decode_tile(const KParams& p, int t, Tile& o) {
   const int l = t - p.n_tiles * p.mt_prefix[lo];
   o.e = lo;
   o.n = l / mt_e;
-  o.row0 = p.g.offsets[lo] + (l % mt_e) * BM;
-  o.rows = min(BM, p.g.offsets[lo + 1] - o.row0);
+  o.row0 = p.g.offsets[lo] + (l % mt_e) * p.tile_rows;
+  o.rows = min(p.tile_rows, p.g.offsets[lo + 1] - o.row0);
   return o.n < p.n_tiles && o.row0 >= 0 && o.rows > 0 &&
          o.row0 + o.rows <= p.g.cap_rows;
 }
@@ -456,11 +457,385 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.ldo = a.ldo;
   p.err = a.err;
   p.mt_prefix = a.g.mt_prefix;
+  p.tile_rows = BM;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);
   kernel<<<grid, kThreads, C::kSmemBytes, stream>>>(*a.map_a, *a.map_b, p);
   return cudaGetLastError();
+}
+
+// ===========================================================================
+// 2-SM variant (cta_group::2) for groups of many rows.
+//
+// A cluster of two CTAs on one TPC computes a 256 x 256 tile: CTA rank r
+// holds rows [row0 + 128 r, +128) of A and one half of the weight tile
+// (SwiGLU: rank 0 the 128 gate rows, rank 1 the 128 matching up rows; down:
+// rows n*256 + 128 r of W_down), so each SM streams 32 KB per 64-k stage
+// instead of 48 KB, and the 192 KB ring holds 6 stages.  One thread of the
+// leader CTA (rank 0) issues tcgen05.mma.cta_group::2 (M = 256, N = 256);
+// each CTA's TMEM receives its 128 rows x 256 fp32 columns (two buffers of
+// 256 columns, allocated collectively by one warp per CTA).
+// Barriers: both producers arrive (with their byte counts) on the leader's
+// "full" barrier and their TMA loads complete on it; MMA completion is
+// multicast to both CTAs' "empty" and "accumulator full" barriers; both
+// CTAs' epilogue warps arrive on the leader's "accumulator empty" barrier.
+// Every barrier wait is bounded, as in the 1-SM kernel.
+// ===========================================================================
+constexpr int kThreads2 = 192;
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// shared::cta address -> the same variable's shared::cluster address in CTA `rank`
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+// Byte-count announcement on the leader's barrier from the peer CTA: no
+// release needed (the bytes themselves arrive by TMA complete_tx).
+__device__ __forceinline__ void mbar_expect_tx_cluster(uint32_t cl_bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.relaxed.cluster.shared::cluster.b64 _, [%0], %1;" ::"r"(cl_bar),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cl_bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cl_bar)
+               : "memory");
+}
+// TMA tile load whose completion is counted on a barrier in either CTA of the pair.
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int c0,
+                                                 int c1, uint32_t cl_bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(cl_bar)
+      : "memory");
+}
+__device__ __forceinline__ void mma_bf16_pair(uint32_t tmem_d, uint64_t da, uint64_t db,
+                                              uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(tmem_d),
+      "l"(da), "l"(db), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on the barrier at this shared-memory offset in both CTAs of the pair
+// once all prior MMAs of this thread have completed.
+__device__ __forceinline__ void mma_commit_pair(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(bar),
+      "h"(static_cast<uint16_t>(0x3))
+      : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+
+struct Cfg2 {
+  static constexpr int BN = 256;                 // output tile width of the pair
+  static constexpr int kABytes = BM * BK * 2;    // 16 KB: this CTA's 128 rows
+  static constexpr int kBBytes = (BN / 2) * BK * 2;  // 16 KB: this CTA's half
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = kRingBytes / kStageBytes;  // 6
+  static constexpr int kTmemCols = 2 * BN;       // two accumulators
+  static constexpr int kSmemBytes = kStages * kStageBytes + 256 + 1024;
+};
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads2, 1)
+    grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap map_a,
+                             const __grid_constant__ CUtensorMap map_b, const KParams p) {
+  using C = Cfg2;
+  constexpr int kStages = C::kStages;
+  constexpr int BN = C::BN;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* sa = smem;
+  uint8_t* sb = smem + kStages * C::kABytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * C::kStageBytes);
+  uint64_t* full = bars;                        // leader's is the one used
+  uint64_t* empty = bars + kStages;             // per CTA
+  uint64_t* acc_full = bars + 2 * kStages;      // per CTA
+  uint64_t* acc_empty = bars + 2 * kStages + 2; // leader's is the one used
+  uint64_t* drain = bars + 2 * kStages + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+  const int pair = blockIdx.x >> 1;
+  const int npairs = gridDim.x >> 1;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 2);  // one expect_tx arrival per CTA of the pair
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 8);  // 4 epilogue warps x 2 CTAs
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_map(&map_a);
+    prefetch_map(&map_b);
+  }
+  cluster_sync_all();  // barriers of both CTAs initialised; the peer is running
+  if (warp == 1) tmem_alloc_pair(smem_addr(tmem_slot), C::kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  // tiles are 256 rows (both CTAs) x 256 columns; mt_prefix counts 256-row tiles
+  const int ntiles = total_tiles(p);
+  const int nk = p.K / BK;
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer (each CTA: its A rows, its B half) -------
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t issued_mask = 0, issued_phase = 0;
+    bool ok = true;
+    for (int t = pair; t < ntiles && ok; t += npairs) {
+      Tile tl;
+      if (!decode_tile(p, t, tl)) {
+        set_err(p.err, kErrIndex);
+        *abort_flag = 1;
+        break;
+      }
+      for (int kb = 0; kb < nk; ++kb) {
+        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitNs)) {
+          ok = false;
+          break;
+        }
+        const uint32_t fb = map_to_rank(smem_addr(&full[stage]), 0);
+        if (leader)
+          mbar_expect_tx(smem_addr(&full[stage]), C::kStageBytes);
+        else
+          mbar_expect_tx_cluster(fb, C::kStageBytes);
+        const int k0 = kb * BK;
+        tma_load_2d_pair(smem_addr(sa + stage * C::kABytes), &map_a, k0,
+                         tl.row0 + static_cast<int>(rank) * BM, fb);
+        int brow;
+        if (MODE == kModeSwiGLU)
+          brow = tl.e * p.b_rows_per_group + (rank ? p.b_up_offset : 0) + tl.n * (BN / 2);
+        else
+          brow = tl.e * p.b_rows_per_group + tl.n * BN + static_cast<int>(rank) * (BN / 2);
+        tma_load_2d_pair(smem_addr(sb + stage * C::kBBytes), &map_b, k0, brow, fb);
+        issued_mask |= 1u << stage;
+        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    if (!ok) {
+      set_err(p.err, kErrTimeout);
+      *abort_flag = 1;
+    }
+    if (*abort_flag && leader) {
+      for (int s = 0; s < kStages; ++s)
+        if (issued_mask & (1u << s))
+          mbar_wait(&full[s], (issued_phase >> s) & 1u, nullptr, kDrainNs);
+    }
+  } else if (warp == 1 && lane == 0 && leader) {
+    // ---------------- MMA issuer (leader CTA only) ----------------
+    constexpr uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) |
+                               (static_cast<uint32_t>(BN >> 3) << 17) |
+                               (static_cast<uint32_t>((2 * BM) >> 4) << 24);
+    int stage = 0;
+    uint32_t phase = 0;
+    int lt = 0;
+    bool ok = true, issued_any = false;
+    for (int t = pair; t < ntiles && ok; t += npairs, ++lt) {
+      const int ab = lt & 1;
+      const uint32_t acc_phase = (lt >> 1) & 1;
+      if (!mbar_wait(&acc_empty[ab], acc_phase ^ 1u, abort_flag, kWaitNs)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(ab * BN);
+      for (int kb = 0; kb < nk; ++kb) {
+        if (!mbar_wait(&full[stage], phase, abort_flag, kWaitNs)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a0 = smem_addr(sa + stage * C::kABytes);
+        const uint32_t b0 = smem_addr(sb + stage * C::kBBytes);
+#pragma unroll
+        for (int k = 0; k < BK / UMMA_K; ++k)
+          mma_bf16_pair(d_tmem, desc_sw128(a0 + k * UMMA_K * 2), desc_sw128(b0 + k * UMMA_K * 2),
+                        idesc, (kb > 0 || k > 0) ? 1u : 0u);
+        issued_any = true;
+        mma_commit_pair(smem_addr(&empty[stage]));
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (!ok) break;
+      mma_commit_pair(smem_addr(&acc_full[ab]));
+    }
+    if (!ok) {
+      set_err(p.err, kErrTimeout);
+      *abort_flag = 1;
+    }
+    if (*abort_flag && issued_any) {
+      mma_commit_pair(smem_addr(drain));
+      mbar_wait(drain, 0, nullptr, kDrainNs);
+    }
+  } else if (warp >= 2) {
+    // ---------------- epilogue (each CTA: its 128 rows) ----------------
+    const int quarter = warp & 3;
+    const int row = static_cast<int>(rank) * BM + quarter * 32 + lane;  // row within the 256
+    const uint32_t acc_empty_leader0 = map_to_rank(smem_addr(&acc_empty[0]), 0);
+    const uint32_t acc_empty_leader1 = map_to_rank(smem_addr(&acc_empty[1]), 0);
+    int lt = 0;
+    for (int t = pair; t < ntiles; t += npairs, ++lt) {
+      Tile tl;
+      const bool tile_ok = decode_tile(p, t, tl);
+      const int ab = lt & 1;
+      const uint32_t acc_phase = (lt >> 1) & 1;
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&acc_full[ab], acc_phase, abort_flag, kWaitNs) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) {
+        if (lane == 0) {
+          if (!*abort_flag) set_err(p.err, kErrTimeout);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                             static_cast<uint32_t>(ab * BN);
+      const bool store = tile_ok && row < tl.rows;
+      __nv_bfloat16* orow = p.out + static_cast<int64_t>(tl.row0 + (store ? row : 0)) * p.ldo;
+      if (MODE == kModeSwiGLU) {
+#pragma unroll 1
+        for (int c = 0; c < BN / 2; c += 32) {
+          uint32_t g[32], u[32];
+          tmem_ld32(tbase + c, g);
+          tmem_ld32(tbase + BN / 2 + c, u);
+          tmem_ld_wait();
+          if (store) {
+            uint32_t packed[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+              const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+              const float a0 = g0 / (1.0f + __expf(-g0)) * u0;
+              const float a1 = g1 / (1.0f + __expf(-g1)) * u1;
+              __nv_bfloat162 h2 = __floats2bfloat162_rn(a0, a1);
+              packed[i] = *reinterpret_cast<uint32_t*>(&h2);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(orow + tl.n * (BN / 2) + c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              dst[v] = make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
+                                  packed[4 * v + 3]);
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t v32[32];
+          tmem_ld32(tbase + c, v32);
+          tmem_ld_wait();
+          if (store) {
+            uint32_t packed[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              __nv_bfloat162 h2 = __floats2bfloat162_rn(__uint_as_float(v32[2 * i]),
+                                                        __uint_as_float(v32[2 * i + 1]));
+              packed[i] = *reinterpret_cast<uint32_t*>(&h2);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(orow + tl.n * BN + c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              dst[v] = make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
+                                  packed[4 * v + 3]);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(ab ? acc_empty_leader1 : acc_empty_leader0);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // the pair's MMAs and TMEM reads are done in both CTAs
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc_pair(tmem_base, C::kTmemCols);
+  }
+}
+
+template <int MODE>
+cudaError_t launch_pair_impl(const TcGemmArgs& a, cudaStream_t stream) {
+  using C = Cfg2;
+  auto kernel = grouped_gemm_pair_kernel<MODE>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       C::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  KParams p;
+  p.K = a.K;
+  p.n_tiles = MODE == kModeSwiGLU ? a.n_total / (C::BN / 2) : a.n_total / C::BN;
+  p.b_rows_per_group = a.b_rows_per_group;
+  p.b_up_offset = a.b_up_offset;
+  p.g = a.g;
+  p.mt_prefix = a.g.mt2_prefix;
+  p.tile_rows = 2 * BM;
+  p.max_mtiles = a.g.offsets ? (a.g.cap_rows + p.tile_rows - 1) / p.tile_rows + a.g.E
+                             : (a.g.dense_rows + p.tile_rows - 1) / p.tile_rows;
+  p.out = static_cast<__nv_bfloat16*>(a.out);
+  p.ldo = a.ldo;
+  p.err = a.err;
+  const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
+  if (max_tiles == 0) return cudaSuccess;
+  int pairs = a.num_sms / 2;
+  if (pairs > max_tiles) pairs = static_cast<int>(max_tiles);
+  if (pairs < 1) pairs = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * pairs);
+  cfg.blockDim = dim3(kThreads2);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, *a.map_a, *a.map_b, p);
 }
 
 }  // namespace
@@ -476,6 +851,13 @@ cudaError_t launch_down_tc(const TcGemmArgs& a, int bn, cudaStream_t stream) {
 // SwiGLU loads gate and up halves as two boxes of bn/2 rows; down loads one
 // box of bn rows.
 int tc_b_box_rows(bool swiglu, int bn) { return swiglu ? bn / 2 : bn; }
+
+cudaError_t launch_swiglu_tc_pair(const TcGemmArgs& a, cudaStream_t stream) {
+  return launch_pair_impl<kModeSwiGLU>(a, stream);
+}
+cudaError_t launch_down_tc_pair(const TcGemmArgs& a, cudaStream_t stream) {
+  return launch_pair_impl<kModeDown>(a, stream);
+}
 // Output columns of one tile.
 int tc_n_granule(bool swiglu, int bn) { return swiglu ? bn / 2 : bn; }
 

@@ -42,10 +42,11 @@ struct DispatchBufs {
   int32_t* blk_off;    // [nblk, E]
   int32_t* counts;     // [E]
   int32_t* offsets;    // [E+1]
-  int32_t* mt_prefix;  // [E+1]
+  int32_t* mt_prefix;  // [E+1] 128-row tiles
+  int32_t* mt2_prefix; // [E+1] 256-row tiles
   int32_t* perm;       // [T*k_max]
   int32_t* row_of;     // [T*k_max]
-  int32_t* totals;     // header: total_pairs, total_mtiles
+  int32_t* totals;     // header: total_pairs, total_mtiles, total_mtiles2
   uint32_t* err;
 };
 constexpr int kDispatchBlock = 256;  // tokens per dispatch block
@@ -64,6 +65,7 @@ cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* row
 struct GroupRows {
   const int32_t* offsets;    // [E+1] or nullptr
   const int32_t* mt_prefix;  // [E+1] prefix of 128-row tile counts
+  const int32_t* mt2_prefix; // [E+1] prefix of 256-row tile counts
   const int32_t* totals;     // device total rows (grouped mode)
   int E;
   int dense_rows;
@@ -96,6 +98,12 @@ struct TcGemmArgs {
 cudaError_t launch_swiglu_tc(const TcGemmArgs& a, int bn, cudaStream_t stream);
 cudaError_t launch_down_tc(const TcGemmArgs& a, int bn, cudaStream_t stream);
 int tc_b_box_rows(bool swiglu, int bn);
+// CTA-pair (2-SM, cta_group::2) variants: 256 x 256 tiles, cluster of two
+// CTAs; A and B tensor maps both with boxes of 128 rows; needs
+// GroupRows::mt2_prefix in grouped mode.  n_total must be a multiple of 128
+// (SwiGLU) or 256 (down).
+cudaError_t launch_swiglu_tc_pair(const TcGemmArgs& a, cudaStream_t stream);
+cudaError_t launch_down_tc_pair(const TcGemmArgs& a, cudaStream_t stream);
 int tc_n_granule(bool swiglu, int bn);  // output columns per tile
 // 0 when n_total is not a multiple of the smaller granule.
 int tc_pick_bn(bool swiglu, int n_total, int64_t mtiles_est, int num_sms);

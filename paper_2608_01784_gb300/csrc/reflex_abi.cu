@@ -21,7 +21,7 @@ size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 // Byte offsets of every workspace region (all 256-byte aligned).
 struct Layout {
   size_t hdr, z, ids, alpha, blk_count, blk_off, counts, offsets, mt_prefix,
-      perm, row_of, xperm, amid, ash, ysh, total;
+      mt2_prefix, perm, row_of, xperm, amid, ash, ysh, total;
   int64_t cap_rows;
   int nblk;
 };
@@ -58,6 +58,7 @@ Layout make_layout(int32_t dtype, int32_t T, int32_t d, int32_t E,
   L.counts = take(static_cast<size_t>(E) * 4);
   L.offsets = take(static_cast<size_t>(E + 1) * 4);
   L.mt_prefix = take(static_cast<size_t>(E + 1) * 4);
+  L.mt2_prefix = take(static_cast<size_t>(E + 1) * 4);
   L.perm = take(cap * 4);
   L.row_of = take(cap * 4);
   L.xperm = take(cap * d * es);  // later reused for the expert outputs y
@@ -245,6 +246,10 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
   const int bn_dn = rx::tc_pick_bn(false, d, mt_est, sms_h);
   const int bn_sup = shared_inter ? rx::tc_pick_bn(true, shared_inter, mt_dense, sms_h) : 128;
   const int bn_sdn = shared_inter ? rx::tc_pick_bn(false, d, mt_dense, sms_h) : 128;
+  // CTA-pair (2-SM) GEMMs once the groups are expected to hold several
+  // 256-row tiles (compute-bound regime): half the operand bytes per SM
+  const int64_t rows_per_group_est = static_cast<int64_t>(T) * k_max / 2 / E;
+  const bool pair_routed = rows_per_group_est >= 512 && inter % 128 == 0 && d % 256 == 0;
   if (!simt) {
     if (bn_up == 0 || bn_dn == 0 || bn_sup == 0 || bn_sdn == 0) return REFLEX_EUNSUPPORTED;
     if (encode_fn() == nullptr) return REFLEX_ECUDA;
@@ -272,9 +277,10 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
                                      I32(L.ids), alpha, err, s));
   }
   if (stages & REFLEX_STAGE_DISPATCH) {
-    rx::DispatchBufs b{I32(L.blk_count), I32(L.blk_off), I32(L.counts),
-                       I32(L.offsets),   I32(L.mt_prefix), I32(L.perm),
-                       I32(L.row_of),    totals,          err};
+    rx::DispatchBufs b{I32(L.blk_count), I32(L.blk_off),   I32(L.counts),
+                       I32(L.offsets),   I32(L.mt_prefix), I32(L.mt2_prefix),
+                       I32(L.perm),      I32(L.row_of),    totals,
+                       err};
     RX_CUDA(rx::launch_dispatch(I32(L.ids), k, T, E, k_max, b, s));
     RX_CUDA(rx::launch_gather_rows(dtype, hidden, I32(L.row_of), k, T, k_max, cap, d,
                                    xperm, err, sms, s));
@@ -282,8 +288,9 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
   const bool up = (stages & REFLEX_STAGE_EXPERT_UP) != 0;
   const bool down = (stages & REFLEX_STAGE_EXPERT_DOWN) != 0;
   if (up || down) {
-    rx::GroupRows grouped{I32(L.offsets), I32(L.mt_prefix), totals, E, 0, cap};
-    rx::GroupRows dense{nullptr, nullptr, nullptr, 1, T, T};
+    rx::GroupRows grouped{I32(L.offsets), I32(L.mt_prefix), I32(L.mt2_prefix), totals,
+                          E, 0, cap};
+    rx::GroupRows dense{nullptr, nullptr, nullptr, nullptr, 1, T, T};
     if (simt) {
       if (up) {
         RX_CUDA(rx::launch_swiglu_simt(dtype, xperm, w_gate_up, d, inter, grouped, amid, err, s));
@@ -299,10 +306,10 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
       CUtensorMap ma1, mb1, ma2, mb2;
       if (!make_map(&ma1, xperm, cap, d, rx::kTileM) ||
           !make_map(&mb1, w_gate_up, static_cast<int64_t>(E) * 2 * inter, d,
-                    rx::tc_b_box_rows(true, bn_up)) ||
+                    pair_routed ? 128 : rx::tc_b_box_rows(true, bn_up)) ||
           !make_map(&ma2, amid, cap, inter, rx::kTileM) ||
           !make_map(&mb2, w_down, static_cast<int64_t>(E) * d, inter,
-                    rx::tc_b_box_rows(false, bn_dn)))
+                    pair_routed ? 128 : rx::tc_b_box_rows(false, bn_dn)))
         return REFLEX_ECUDA;
       rx::TcGemmArgs g1{&ma1, &mb1, d, inter, 2 * inter, inter, grouped, amid, inter, err, sms};
       rx::TcGemmArgs g2{&ma2, &mb2, inter, d, d, 0, grouped, xperm, d, err, sms};
@@ -319,11 +326,17 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
                         dense, ash, shared_inter, err, sms};
       rx::TcGemmArgs h2{&sa2, &sb2, shared_inter, d, d, 0, dense, ysh, d, err, sms};
       if (up) {
-        RX_CUDA(rx::launch_swiglu_tc(g1, bn_up, s));
+        if (pair_routed)
+          RX_CUDA(rx::launch_swiglu_tc_pair(g1, s));
+        else
+          RX_CUDA(rx::launch_swiglu_tc(g1, bn_up, s));
         if (shared_inter) RX_CUDA(rx::launch_swiglu_tc(h1, bn_sup, s));
       }
       if (down) {
-        RX_CUDA(rx::launch_down_tc(g2, bn_dn, s));
+        if (pair_routed)
+          RX_CUDA(rx::launch_down_tc_pair(g2, s));
+        else
+          RX_CUDA(rx::launch_down_tc(g2, bn_dn, s));
         if (shared_inter) RX_CUDA(rx::launch_down_tc(h2, bn_sdn, s));
       }
     }

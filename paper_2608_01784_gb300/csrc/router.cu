@@ -281,6 +281,139 @@ __global__ void __launch_bounds__(kSelWarps * 32)
   }
 }
 
+// Large-batch variant, SGEMM-style register blocking.  Thread tile 8 tokens
+// x 8 experts (64 chains); a warp is 8 token rows (ty) x 4 expert columns
+// (tx); WT x WE warps per CTA.  Each 16-k stage is loaded into registers one
+// stage ahead (16-byte vectors), widened, and stored k-major into a
+// double-buffered fp32 tile; per k a thread reads its 8 token and 8 expert
+// values with four 16-byte shared loads and issues 64 fmas, every chain
+// still advancing over k = 0 .. d-1 in order.
+constexpr int kKcB = 16;
+
+template <typename Tin, int WT, int WE>
+struct BlockCfg {
+  static constexpr int BT = 64 * WT;   // tokens per CTA
+  static constexpr int BE = 32 * WE;   // experts per CTA
+  static constexpr int NT = 32 * WT * WE;
+  static constexpr int kVecPerRow = kKcB * static_cast<int>(sizeof(Tin)) / 16;
+  static constexpr int kElemsPerVec = 16 / static_cast<int>(sizeof(Tin));
+  static constexpr int kVecs = (BT + BE) * kVecPerRow;
+  static constexpr int kVecsPerThread = (kVecs + NT - 1) / NT;
+};
+
+template <typename Tin, int WT, int WE>
+__global__ void __launch_bounds__(BlockCfg<Tin, WT, WE>::NT)
+    logits_block_kernel(const Tin* __restrict__ h, const Tin* __restrict__ w,
+                        int T, int d, int E, float* __restrict__ z) {
+  using C = BlockCfg<Tin, WT, WE>;
+  constexpr int BT = C::BT, BE = C::BE, NT = C::NT, VPT = C::kVecsPerThread;
+  constexpr int EV = C::kElemsPerVec;
+  __shared__ __align__(16) float As[2][kKcB][BT];
+  __shared__ __align__(16) float Bs[2][kKcB][BE];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int ty = lane >> 2, tx = lane & 3;
+  const int wt = warp / WE, we = warp % WE;
+  const int my_t = wt * 64 + ty * 8;
+  const int my_e = we * 32 + tx * 8;
+  const int t0 = blockIdx.x * BT;
+  const int e0 = blockIdx.y * BE;
+  const int nst = d / kKcB;
+
+  uint4 raw[VPT];
+  auto load_regs = [&](int st) {
+    const int k0 = st * kKcB;
+#pragma unroll
+    for (int u = 0; u < VPT; ++u) {
+      const int v = threadIdx.x + u * NT;
+      raw[u] = make_uint4(0u, 0u, 0u, 0u);
+      if (v < C::kVecs) {
+        const int r = v % (BT + BE), q = v / (BT + BE);
+        const bool is_h = r < BT;
+        const int idx = is_h ? t0 + r : e0 + (r - BT);
+        if (idx < (is_h ? T : E)) {
+          const Tin* src = (is_h ? h : w) + static_cast<int64_t>(idx) * d + k0 + q * EV;
+          raw[u] = __ldg(reinterpret_cast<const uint4*>(src));
+        }
+      }
+    }
+  };
+  auto store_smem = [&](int buf) {
+#pragma unroll
+    for (int u = 0; u < VPT; ++u) {
+      const int v = threadIdx.x + u * NT;
+      if (v < C::kVecs) {
+        const int r = v % (BT + BE), q = v / (BT + BE);
+        float f[8];
+        if constexpr (EV == 8) {
+          widen8(reinterpret_cast<const uint8_t*>(&raw[u]), f, static_cast<const Tin*>(nullptr));
+        } else {
+          f[0] = __uint_as_float(raw[u].x); f[1] = __uint_as_float(raw[u].y);
+          f[2] = __uint_as_float(raw[u].z); f[3] = __uint_as_float(raw[u].w);
+        }
+#pragma unroll
+        for (int i = 0; i < EV; ++i) {
+          if (r < BT) As[buf][q * EV + i][r] = f[i];
+          else Bs[buf][q * EV + i][r - BT] = f[i];
+        }
+      }
+    }
+  };
+
+  float acc[8][8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+
+  load_regs(0);
+  store_smem(0);
+  __syncthreads();
+  for (int st = 0; st < nst; ++st) {
+    const int buf = st & 1;
+    if (st + 1 < nst) load_regs(st + 1);
+#pragma unroll 4
+    for (int kk = 0; kk < kKcB; ++kk) {
+      const float4 a0 = *reinterpret_cast<const float4*>(&As[buf][kk][my_t]);
+      const float4 a1 = *reinterpret_cast<const float4*>(&As[buf][kk][my_t + 4]);
+      const float4 b0 = *reinterpret_cast<const float4*>(&Bs[buf][kk][my_e]);
+      const float4 b1 = *reinterpret_cast<const float4*>(&Bs[buf][kk][my_e + 4]);
+      const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = __fmaf_rn(a[i], b[j], acc[i][j]);
+    }
+    if (st + 1 < nst) store_smem(buf ^ 1);
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int t = t0 + my_t + i;
+    if (t >= T) continue;
+    float* zr = z + static_cast<int64_t>(t) * E;
+    const int e = e0 + my_e;
+    if (e + 8 <= E && (E % 4) == 0) {
+      *reinterpret_cast<float4*>(zr + e) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+      *reinterpret_cast<float4*>(zr + e + 4) =
+          make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (e + j < E) zr[e + j] = acc[i][j];
+    }
+  }
+}
+
+template <typename Tin, int WT, int WE>
+cudaError_t launch_logits_block(const Tin* h, const Tin* w, int T, int d, int E,
+                                float* z, cudaStream_t s) {
+  using C = BlockCfg<Tin, WT, WE>;
+  const dim3 g((T + C::BT - 1) / C::BT, (E + C::BE - 1) / C::BE);
+  logits_block_kernel<Tin, WT, WE><<<g, C::NT, 0, s>>>(h, w, T, d, E, z);
+  return cudaGetLastError();
+}
+
 // Short-batch variant: too few (token, expert) chains to fill the GPU with
 // the widened-buffer tiles, so each CTA (4 warps) keeps 8 TM tokens x 64
 // experts, one 4-stage ring of 32-k raw chunks, and widens operands at use
@@ -403,10 +536,12 @@ cudaError_t logits_dispatch(const Tin* h, const Tin* w, int T, int d, int E,
     return static_cast<int64_t>((T + bt - 1) / bt) * ((E + be - 1) / be);
   };
   const int64_t want = (num_sms * 4) / 5;
+  // measured on GB300: E >= 128 -> widened-buffer tiles (TM 4, TN 8); E = 64
+  // with a large batch -> 8 x 8 register blocking
   if (E >= 128 && grid_for(64, 128) >= want)  // TM 4, TN 8, 2 x 4 warps
     return launch_logits_tile<Tin, 4, 8, 2, 4>(h, w, T, d, E, z, s);
-  if (E >= 64 && grid_for(64, 64) >= want)    // TM 4, TN 4, 2 x 4 warps
-    return launch_logits_tile<Tin, 4, 4, 2, 4>(h, w, T, d, E, z, s);
+  if (E >= 64 && grid_for(128, 64) >= want)   // 8 x 8 blocking, 2 x 2 warps
+    return launch_logits_block<Tin, 2, 2>(h, w, T, d, E, z, s);
   if (grid_for(32, 64) >= want) return launch_logits_short<Tin, 4>(h, w, T, d, E, z, s);
   if (grid_for(16, 64) >= want) return launch_logits_short<Tin, 2>(h, w, T, d, E, z, s);
   return launch_logits_short<Tin, 1>(h, w, T, d, E, z, s);
