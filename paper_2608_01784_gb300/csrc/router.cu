@@ -6,10 +6,10 @@
 // k = 0, 1, ..., d-1 starting from +0, in fp32 (bf16 inputs are widened
 // exactly).  Fixing the summation order makes the scores — and therefore the
 // selected expert sets, an integer result — reproducible bit for bit.  The
-// kernel is a register-tiled SIMT GEMM: each thread owns TM tokens x TN
-// experts and walks k in order, so the fixed order costs no extra work; raw
-// tiles stream through a cp.async ring of 32-k chunks, and each chunk is
-// widened once into a k-major fp32 buffer read with conflict-free float4s.
+// kernels are register-tiled SIMT GEMMs: each thread owns TM tokens x TN
+// experts and walks k in order, so the fixed order costs no extra work.  Raw
+// tiles stream through a cp.async ring; bf16 operands are read straight from
+// it into mixed-precision fmas, fp32 operands through a k-major buffer.
 //
 // Selection.  One warp per token keeps E/32 scores per lane and runs k_i
 // rounds of a warp-wide max over packed 64-bit keys
@@ -281,139 +281,6 @@ __global__ void __launch_bounds__(kSelWarps * 32)
   }
 }
 
-// Large-batch variant, SGEMM-style register blocking.  Thread tile 8 tokens
-// x 8 experts (64 chains); a warp is 8 token rows (ty) x 4 expert columns
-// (tx); WT x WE warps per CTA.  Each 16-k stage is loaded into registers one
-// stage ahead (16-byte vectors), widened, and stored k-major into a
-// double-buffered fp32 tile; per k a thread reads its 8 token and 8 expert
-// values with four 16-byte shared loads and issues 64 fmas, every chain
-// still advancing over k = 0 .. d-1 in order.
-constexpr int kKcB = 16;
-
-template <typename Tin, int WT, int WE>
-struct BlockCfg {
-  static constexpr int BT = 64 * WT;   // tokens per CTA
-  static constexpr int BE = 32 * WE;   // experts per CTA
-  static constexpr int NT = 32 * WT * WE;
-  static constexpr int kVecPerRow = kKcB * static_cast<int>(sizeof(Tin)) / 16;
-  static constexpr int kElemsPerVec = 16 / static_cast<int>(sizeof(Tin));
-  static constexpr int kVecs = (BT + BE) * kVecPerRow;
-  static constexpr int kVecsPerThread = (kVecs + NT - 1) / NT;
-};
-
-template <typename Tin, int WT, int WE>
-__global__ void __launch_bounds__(BlockCfg<Tin, WT, WE>::NT)
-    logits_block_kernel(const Tin* __restrict__ h, const Tin* __restrict__ w,
-                        int T, int d, int E, float* __restrict__ z) {
-  using C = BlockCfg<Tin, WT, WE>;
-  constexpr int BT = C::BT, BE = C::BE, NT = C::NT, VPT = C::kVecsPerThread;
-  constexpr int EV = C::kElemsPerVec;
-  __shared__ __align__(16) float As[2][kKcB][BT];
-  __shared__ __align__(16) float Bs[2][kKcB][BE];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int ty = lane >> 2, tx = lane & 3;
-  const int wt = warp / WE, we = warp % WE;
-  const int my_t = wt * 64 + ty * 8;
-  const int my_e = we * 32 + tx * 8;
-  const int t0 = blockIdx.x * BT;
-  const int e0 = blockIdx.y * BE;
-  const int nst = d / kKcB;
-
-  uint4 raw[VPT];
-  auto load_regs = [&](int st) {
-    const int k0 = st * kKcB;
-#pragma unroll
-    for (int u = 0; u < VPT; ++u) {
-      const int v = threadIdx.x + u * NT;
-      raw[u] = make_uint4(0u, 0u, 0u, 0u);
-      if (v < C::kVecs) {
-        const int r = v % (BT + BE), q = v / (BT + BE);
-        const bool is_h = r < BT;
-        const int idx = is_h ? t0 + r : e0 + (r - BT);
-        if (idx < (is_h ? T : E)) {
-          const Tin* src = (is_h ? h : w) + static_cast<int64_t>(idx) * d + k0 + q * EV;
-          raw[u] = __ldg(reinterpret_cast<const uint4*>(src));
-        }
-      }
-    }
-  };
-  auto store_smem = [&](int buf) {
-#pragma unroll
-    for (int u = 0; u < VPT; ++u) {
-      const int v = threadIdx.x + u * NT;
-      if (v < C::kVecs) {
-        const int r = v % (BT + BE), q = v / (BT + BE);
-        float f[8];
-        if constexpr (EV == 8) {
-          widen8(reinterpret_cast<const uint8_t*>(&raw[u]), f, static_cast<const Tin*>(nullptr));
-        } else {
-          f[0] = __uint_as_float(raw[u].x); f[1] = __uint_as_float(raw[u].y);
-          f[2] = __uint_as_float(raw[u].z); f[3] = __uint_as_float(raw[u].w);
-        }
-#pragma unroll
-        for (int i = 0; i < EV; ++i) {
-          if (r < BT) As[buf][q * EV + i][r] = f[i];
-          else Bs[buf][q * EV + i][r - BT] = f[i];
-        }
-      }
-    }
-  };
-
-  float acc[8][8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
-
-  load_regs(0);
-  store_smem(0);
-  __syncthreads();
-  for (int st = 0; st < nst; ++st) {
-    const int buf = st & 1;
-    if (st + 1 < nst) load_regs(st + 1);
-#pragma unroll 4
-    for (int kk = 0; kk < kKcB; ++kk) {
-      const float4 a0 = *reinterpret_cast<const float4*>(&As[buf][kk][my_t]);
-      const float4 a1 = *reinterpret_cast<const float4*>(&As[buf][kk][my_t + 4]);
-      const float4 b0 = *reinterpret_cast<const float4*>(&Bs[buf][kk][my_e]);
-      const float4 b1 = *reinterpret_cast<const float4*>(&Bs[buf][kk][my_e + 4]);
-      const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-      const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = __fmaf_rn(a[i], b[j], acc[i][j]);
-    }
-    if (st + 1 < nst) store_smem(buf ^ 1);
-    __syncthreads();
-  }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int t = t0 + my_t + i;
-    if (t >= T) continue;
-    float* zr = z + static_cast<int64_t>(t) * E;
-    const int e = e0 + my_e;
-    if (e + 8 <= E && (E % 4) == 0) {
-      *reinterpret_cast<float4*>(zr + e) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-      *reinterpret_cast<float4*>(zr + e + 4) =
-          make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
-    } else {
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        if (e + j < E) zr[e + j] = acc[i][j];
-    }
-  }
-}
-
-template <typename Tin, int WT, int WE>
-cudaError_t launch_logits_block(const Tin* h, const Tin* w, int T, int d, int E,
-                                float* z, cudaStream_t s) {
-  using C = BlockCfg<Tin, WT, WE>;
-  const dim3 g((T + C::BT - 1) / C::BT, (E + C::BE - 1) / C::BE);
-  logits_block_kernel<Tin, WT, WE><<<g, C::NT, 0, s>>>(h, w, T, d, E, z);
-  return cudaGetLastError();
-}
-
 // Short-batch variant: too few (token, expert) chains to fill the GPU with
 // the widened-buffer tiles, so each CTA (4 warps) keeps 8 TM tokens x 64
 // experts, one 4-stage ring of 32-k raw chunks, and widens operands at use
@@ -525,26 +392,190 @@ cudaError_t launch_logits_short(const Tin* h, const Tin* w, int T, int d, int E,
   return cudaGetLastError();
 }
 
-// Tile choice: the widened-buffer tiles when they fill most SMs without
-// overhanging the expert count (more chains per thread, fewer operand reads
-// per fma); otherwise the short-batch kernel with the largest token tile
-// that still fills most SMs.
-template <typename Tin>
-cudaError_t logits_dispatch(const Tin* h, const Tin* w, int T, int d, int E,
+// ---- bf16 scores with mixed-precision fma ----------------------------------
+// fma.rn.f32.bf16 d, a, b, c rounds a*b + c once to fp32 with bf16 a, b and
+// fp32 c, d.  A bf16 x bf16 product is exact in fp32, so every step equals
+// fma(widen(a), widen(b), c) bit for bit and the chain needs no widening
+// instructions: operands go from shared memory straight into the fma.
+__device__ __forceinline__ void fma_lo(float& acc, uint32_t a2, uint32_t b2) {
+  asm("{\n\t.reg .b16 al, ah, bl, bh;\n\t"
+      "mov.b32 {al, ah}, %1;\n\t"
+      "mov.b32 {bl, bh}, %2;\n\t"
+      "fma.rn.f32.bf16 %0, al, bl, %0;\n\t}"
+      : "+f"(acc)
+      : "r"(a2), "r"(b2));
+}
+__device__ __forceinline__ void fma_hi(float& acc, uint32_t a2, uint32_t b2) {
+  asm("{\n\t.reg .b16 al, ah, bl, bh;\n\t"
+      "mov.b32 {al, ah}, %1;\n\t"
+      "mov.b32 {bl, bh}, %2;\n\t"
+      "fma.rn.f32.bf16 %0, ah, bh, %0;\n\t}"
+      : "+f"(acc)
+      : "r"(a2), "r"(b2));
+}
+
+// Tile geometry.  A warp is LY token lanes x LX expert lanes (LY LX = 32);
+// lane (ty, tx) owns tokens ty + LY i (i < TM) and experts tx + LX j
+// (j < TN) of the warp tile, so for fixed (i, j) the warp reads LY (resp.
+// LX) consecutive rows; with rows padded to 80 bytes any 8 consecutive rows
+// start in distinct 16-byte bank groups and each 16-byte operand read is one
+// shared-memory wavefront.  WT x WE warps per CTA.
+template <int LY, int TM, int TN, int WT, int WE, int S, int KC>
+struct MxCfg {
+  static constexpr int LX = 32 / LY;
+  static constexpr int BT = LY * TM * WT;   // tokens per CTA
+  static constexpr int BE = LX * TN * WE;   // experts per CTA
+  static constexpr int NT = 32 * WT * WE;
+  static constexpr int kRowBytes = KC * 2 + 16;
+  static constexpr int kStage = (BT + BE) * kRowBytes;
+  static constexpr int kSmem = S * kStage;
+};
+
+// Each thread keeps TM x TN chains; per 8-k step it reads TM token and TN
+// expert vectors of 8 bf16 and issues 8 TM TN fmas, every chain advancing
+// over k = 0 .. d-1 in order (within a 32-bit word: even k, then odd k).
+// Raw KC-k chunks stream through an S-stage cp.async ring.
+template <int LY, int TM, int TN, int WT, int WE, int S, int KC>
+__global__ void __launch_bounds__(MxCfg<LY, TM, TN, WT, WE, S, KC>::NT)
+    logits_mx_kernel(const __nv_bfloat16* __restrict__ h,
+                     const __nv_bfloat16* __restrict__ w, int T, int d, int E,
+                     float* __restrict__ z) {
+  using C = MxCfg<LY, TM, TN, WT, WE, S, KC>;
+  constexpr int LX = C::LX, BT = C::BT, BE = C::BE, NT = C::NT;
+  constexpr int kRB = C::kRowBytes;
+  constexpr int kVecs = KC / 8;  // 16-byte vectors per row per chunk
+  extern __shared__ __align__(16) uint8_t smem_m[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int ty = lane / LX, tx = lane % LX;
+  const int wt = warp / WE, we = warp % WE;
+  const int rt = wt * (LY * TM) + ty;       // first token row of this thread
+  const int re = we * (LX * TN) + tx;       // first expert row
+  const int t0 = blockIdx.x * BT;
+  const int e0 = blockIdx.y * BE;
+  const int nchunks = d / KC;
+
+  auto issue = [&](int c) {
+    uint8_t* st = smem_m + (c % S) * C::kStage;
+    const int k0 = c * KC;
+    for (int v = threadIdx.x; v < (BT + BE) * kVecs; v += NT) {
+      const int r = v / kVecs, q = v % kVecs;
+      const bool is_h = r < BT;
+      const int idx = is_h ? t0 + r : e0 + (r - BT);
+      const bool ok = idx < (is_h ? T : E);
+      const __nv_bfloat16* base = is_h ? h : w;
+      cp_async16(st + r * kRB + q * 16,
+                 base + (ok ? static_cast<int64_t>(idx) * d + k0 + q * 8 : 0), ok);
+    }
+  };
+
+  float acc[TM][TN];
+#pragma unroll
+  for (int i = 0; i < TM; ++i)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
+
+#pragma unroll
+  for (int c = 0; c < S - 1; ++c) {
+    if (c < nchunks) issue(c);
+    cp_async_commit();
+  }
+  for (int c = 0; c < nchunks; ++c) {
+    cp_async_wait<S - 2>();
+    __syncthreads();  // chunk c visible; chunk c-1's slot free everywhere
+    if (c + S - 1 < nchunks) issue(c + S - 1);
+    cp_async_commit();
+    const uint8_t* st = smem_m + (c % S) * C::kStage;
+    const uint8_t* hrow = st + rt * kRB;
+    const uint8_t* wrow = st + (BT + re) * kRB;
+#pragma unroll
+    for (int kv = 0; kv < kVecs; ++kv) {
+      uint4 hv[TM], wv[TN];
+#pragma unroll
+      for (int i = 0; i < TM; ++i)
+        hv[i] = *reinterpret_cast<const uint4*>(hrow + (LY * i) * kRB + kv * 16);
+#pragma unroll
+      for (int j = 0; j < TN; ++j)
+        wv[j] = *reinterpret_cast<const uint4*>(wrow + (LX * j) * kRB + kv * 16);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+#pragma unroll
+        for (int i = 0; i < TM; ++i) {
+          const uint32_t a2 = q == 0 ? hv[i].x : q == 1 ? hv[i].y : q == 2 ? hv[i].z : hv[i].w;
+#pragma unroll
+          for (int j = 0; j < TN; ++j) {
+            const uint32_t b2 = q == 0 ? wv[j].x : q == 1 ? wv[j].y : q == 2 ? wv[j].z : wv[j].w;
+            fma_lo(acc[i][j], a2, b2);
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < TM; ++i) {
+          const uint32_t a2 = q == 0 ? hv[i].x : q == 1 ? hv[i].y : q == 2 ? hv[i].z : hv[i].w;
+#pragma unroll
+          for (int j = 0; j < TN; ++j) {
+            const uint32_t b2 = q == 0 ? wv[j].x : q == 1 ? wv[j].y : q == 2 ? wv[j].z : wv[j].w;
+            fma_hi(acc[i][j], a2, b2);
+          }
+        }
+      }
+    }
+  }
+  cp_async_wait<0>();
+#pragma unroll
+  for (int i = 0; i < TM; ++i) {
+    const int t = t0 + rt + LY * i;
+    if (t >= T) continue;
+#pragma unroll
+    for (int j = 0; j < TN; ++j) {
+      const int e = e0 + re + LX * j;
+      if (e < E) z[static_cast<int64_t>(t) * E + e] = acc[i][j];
+    }
+  }
+}
+
+template <int LY, int TM, int TN, int WT, int WE, int S, int KC = 32>
+cudaError_t launch_logits_mx(const __nv_bfloat16* h, const __nv_bfloat16* w, int T,
+                             int d, int E, float* z, cudaStream_t s) {
+  using C = MxCfg<LY, TM, TN, WT, WE, S, KC>;
+  auto kern = logits_mx_kernel<LY, TM, TN, WT, WE, S, KC>;
+  if (C::kSmem > 48 * 1024) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+    if (e != cudaSuccess) return e;
+  }
+  const dim3 g((T + C::BT - 1) / C::BT, (E + C::BE - 1) / C::BE);
+  kern<<<g, C::NT, C::kSmem, s>>>(h, w, T, d, E, z);
+  return cudaGetLastError();
+}
+
+// fp32 inputs: the widened-buffer tiles when they fill most SMs without
+// overhanging the expert count; otherwise the short-batch kernel with the
+// largest token tile that still fills most SMs.
+cudaError_t logits_dispatch(const float* h, const float* w, int T, int d, int E,
                             float* z, int num_sms, cudaStream_t s) {
   auto grid_for = [&](int bt, int be) {
     return static_cast<int64_t>((T + bt - 1) / bt) * ((E + be - 1) / be);
   };
   const int64_t want = (num_sms * 4) / 5;
-  // measured on GB300: E >= 128 -> widened-buffer tiles (TM 4, TN 8); E = 64
-  // with a large batch -> 8 x 8 register blocking
   if (E >= 128 && grid_for(64, 128) >= want)  // TM 4, TN 8, 2 x 4 warps
-    return launch_logits_tile<Tin, 4, 8, 2, 4>(h, w, T, d, E, z, s);
-  if (E >= 64 && grid_for(128, 64) >= want)   // 8 x 8 blocking, 2 x 2 warps
-    return launch_logits_block<Tin, 2, 2>(h, w, T, d, E, z, s);
-  if (grid_for(32, 64) >= want) return launch_logits_short<Tin, 4>(h, w, T, d, E, z, s);
-  if (grid_for(16, 64) >= want) return launch_logits_short<Tin, 2>(h, w, T, d, E, z, s);
-  return launch_logits_short<Tin, 1>(h, w, T, d, E, z, s);
+    return launch_logits_tile<float, 4, 8, 2, 4>(h, w, T, d, E, z, s);
+  if (grid_for(32, 64) >= want) return launch_logits_short<float, 4>(h, w, T, d, E, z, s);
+  if (grid_for(16, 64) >= want) return launch_logits_short<float, 2>(h, w, T, d, E, z, s);
+  return launch_logits_short<float, 1>(h, w, T, d, E, z, s);
+}
+
+// bf16 inputs: mixed-precision fma tiles, chosen by the number of chains
+// T x E per SM (measured on GB300 over T = 256 .. 65536, E = 64 and 256).
+// Few chains: small thread tiles so every SM gets warps; many chains: 4 x 8
+// or 4 x 4 thread tiles, which need fewer operand reads per fma.
+cudaError_t logits_dispatch(const __nv_bfloat16* h, const __nv_bfloat16* w, int T,
+                            int d, int E, float* z, int num_sms, cudaStream_t s) {
+  const int64_t per_sm = static_cast<int64_t>(T) * E / (num_sms > 0 ? num_sms : 1);
+  if (per_sm <= 216) return launch_logits_mx<4, 1, 1, 4, 1, 8>(h, w, T, d, E, z, s);
+  if (per_sm <= 1080) return launch_logits_mx<4, 1, 2, 4, 1, 8>(h, w, T, d, E, z, s);
+  if (per_sm <= 4300) return launch_logits_mx<4, 2, 2, 2, 2, 4, 64>(h, w, T, d, E, z, s);
+  if (per_sm <= 10000) return launch_logits_mx<8, 4, 8, 2, 2, 3, 64>(h, w, T, d, E, z, s);
+  if (per_sm <= 20000) return launch_logits_mx<8, 4, 4, 2, 2, 3, 64>(h, w, T, d, E, z, s);
+  return launch_logits_mx<8, 4, 8, 2, 2, 4>(h, w, T, d, E, z, s);
 }
 
 }  // namespace
