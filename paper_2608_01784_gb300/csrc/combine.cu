@@ -32,6 +32,8 @@ __global__ void __launch_bounds__(kThreads)
   __shared__ int32_t s_row[kThreads / 8][kMaxK];
   __shared__ float s_a[kThreads / 8][kMaxK];
   __shared__ int s_k[kThreads / 8];
+  grid_dep_wait();
+  grid_dep_launch();
   const int t = blockIdx.x * tok_per_cta + sub;
   const bool active = sub < tok_per_cta && t < T;
   if (active && threadIdx.x % tpt == 0) {
@@ -102,6 +104,8 @@ __global__ void __launch_bounds__(kThreads)
                         const int32_t* __restrict__ k, int T, int d, int k_max,
                         int cap_rows, Te* __restrict__ out,
                         uint32_t* __restrict__ err) {
+  grid_dep_wait();
+  grid_dep_launch();
   const int lane = threadIdx.x & 31;
   const int t = blockIdx.x * 8 + (threadIdx.x >> 5);
   if (t >= T) return;
@@ -150,13 +154,11 @@ cudaError_t launch_typed(const Te* y, const Te* ysh, const Te* resid, const int3
   if (d <= 2048 && kThreads % (d / 8) == 0) {
     const int tok_per_cta = kThreads / (d / 8);
     const int grid = (T + tok_per_cta - 1) / tok_per_cta;
-    combine_kernel<Te><<<grid, kThreads, 0, stream>>>(y, ysh, resid, row_of, alpha, k, T,
-                                                      d, k_max, cap_rows, out, err);
-  } else {
-    combine_wide_kernel<Te><<<(T + 7) / 8, kThreads, 0, stream>>>(
-        y, ysh, resid, row_of, alpha, k, T, d, k_max, cap_rows, out, err);
+    return launch_pdl(combine_kernel<Te>, dim3(grid), dim3(kThreads), 0, stream, y, ysh, resid,
+                      row_of, alpha, k, T, d, k_max, cap_rows, out, err);
   }
-  return cudaGetLastError();
+  return launch_pdl(combine_wide_kernel<Te>, dim3((T + 7) / 8), dim3(kThreads), 0, stream, y,
+                    ysh, resid, row_of, alpha, k, T, d, k_max, cap_rows, out, err);
 }
 
 }  // namespace

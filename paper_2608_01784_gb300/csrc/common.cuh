@@ -28,6 +28,37 @@ static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 
 constexpr int kTileM = 128;  // rows per grouped-GEMM tile (M of tcgen05.mma)
 
+// ---- programmatic dependent launch -----------------------------------------
+// The kernels after the first of a call are launched with programmatic stream
+// serialization: the next kernel in the stream may be scheduled while the
+// current one drains and runs its prologue (barrier setup, TMEM allocation)
+// early.  grid_dep_wait() returns once the preceding kernel has completed and
+// its writes are visible; every kernel calls it before its first global
+// memory access, so stream order is kept exactly.  grid_dep_launch() allows
+// the following kernel to be scheduled.  Both are no-ops for plain launches.
+__device__ __forceinline__ void grid_dep_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dep_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t stream, Args... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 __device__ __forceinline__ void set_err(uint32_t* err, uint32_t bit) {
   if (err) atomicOr(err, bit);
 }

@@ -51,6 +51,8 @@ __global__ void __launch_bounds__(kBlk)
                  int T, int E, int k_max, int32_t* __restrict__ blk_count,
                  uint32_t* __restrict__ err) {
   extern __shared__ uint32_t mask[];
+  grid_dep_wait();
+  grid_dep_launch();
   build_masks(mask, ids, k, T, E, k_max, err);
   for (int e = threadIdx.x; e < E; e += kBlk) {
     int c = 0;
@@ -93,6 +95,8 @@ __global__ void __launch_bounds__(1024)
                 int32_t* __restrict__ offsets, int32_t* __restrict__ mt_prefix,
                 int32_t* __restrict__ mt2_prefix, int32_t* __restrict__ totals) {
   __shared__ int s_warp[32];
+  grid_dep_wait();
+  grid_dep_launch();
   const int e = threadIdx.x;  // E <= 1024
   int run = 0;
   if (e < E) {
@@ -133,6 +137,8 @@ __global__ void __launch_bounds__(kBlk)
                    int32_t* __restrict__ perm, int32_t* __restrict__ row_of,
                    uint32_t* __restrict__ err) {
   extern __shared__ uint32_t mask[];
+  grid_dep_wait();
+  grid_dep_launch();
   build_masks(mask, ids, k, T, E, k_max, nullptr);
   const int t = blockIdx.x * kBlk + threadIdx.x;
   if (t >= T) return;
@@ -166,6 +172,8 @@ __global__ void __launch_bounds__(256)
                   int d, Te* __restrict__ xp, uint32_t* __restrict__ err) {
   constexpr int kVecElems = 16 / sizeof(Te);  // elements per 16-byte vector
   constexpr int kMaxVec = 8;                  // vectors per lane per pass
+  grid_dep_wait();
+  grid_dep_launch();
   const int lane = threadIdx.x & 31;
   const int warps = gridDim.x * 8;
   const int row_vecs = d / kVecElems;
@@ -216,12 +224,14 @@ cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T, int E,
     if (e1 != cudaSuccess) return e1;
     if (e2 != cudaSuccess) return e2;
   }
-  count_kernel<<<nblk, kBlk, smem, stream>>>(ids, k, T, E, k_max, b.blk_count, b.err);
-  scan_kernel<<<1, 1024, 0, stream>>>(b.blk_count, nblk, E, b.blk_off, b.counts,
-                                      b.offsets, b.mt_prefix, b.mt2_prefix, b.totals);
-  scatter_kernel<<<nblk, kBlk, smem, stream>>>(ids, k, T, E, k_max, b.blk_off,
-                                               b.offsets, b.perm, b.row_of, b.err);
-  return cudaGetLastError();
+  cudaError_t e = launch_pdl(count_kernel, dim3(nblk), dim3(kBlk), smem, stream, ids, k, T,
+                             E, k_max, b.blk_count, b.err);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(scan_kernel, dim3(1), dim3(1024), 0, stream, b.blk_count, nblk, E, b.blk_off,
+                 b.counts, b.offsets, b.mt_prefix, b.mt2_prefix, b.totals);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(scatter_kernel, dim3(nblk), dim3(kBlk), smem, stream, ids, k, T, E, k_max,
+                    b.blk_off, b.offsets, b.perm, b.row_of, b.err);
 }
 
 cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* row_of,
@@ -232,14 +242,12 @@ cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* row
   int grid = (T + 7) / 8;
   if (grid > 16 * num_sms) grid = 16 * num_sms;
   if (dtype == 0)
-    gather_kernel<float><<<grid, 256, 0, stream>>>(
-        static_cast<const float*>(hidden), row_of, k, k_max, cap_rows, T, d,
-        static_cast<float*>(x_perm), err);
-  else
-    gather_kernel<__nv_bfloat16><<<grid, 256, 0, stream>>>(
-        static_cast<const __nv_bfloat16*>(hidden), row_of, k, k_max, cap_rows, T,
-        d, static_cast<__nv_bfloat16*>(x_perm), err);
-  return cudaGetLastError();
+    return launch_pdl(gather_kernel<float>, dim3(grid), dim3(256), 0, stream,
+                      static_cast<const float*>(hidden), row_of, k, k_max, cap_rows, T, d,
+                      static_cast<float*>(x_perm), err);
+  return launch_pdl(gather_kernel<__nv_bfloat16>, dim3(grid), dim3(256), 0, stream,
+                    static_cast<const __nv_bfloat16*>(hidden), row_of, k, k_max, cap_rows, T,
+                    d, static_cast<__nv_bfloat16*>(x_perm), err);
 }
 
 }  // namespace rx

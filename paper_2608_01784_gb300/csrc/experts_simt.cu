@@ -43,6 +43,8 @@ template <typename Te>
 __global__ void __launch_bounds__(kRowsPerCta * 32)
     swiglu_simt_kernel(const Te* __restrict__ x, const Te* __restrict__ wgu,
                        int d, int inter, GroupRows g, Te* __restrict__ act) {
+  grid_dep_wait();
+  grid_dep_launch();
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * kRowsPerCta + (threadIdx.x >> 5);
   if (r >= rows_of(g)) return;
@@ -79,6 +81,8 @@ template <typename Te>
 __global__ void __launch_bounds__(kRowsPerCta * 32)
     down_simt_kernel(const Te* __restrict__ act, const Te* __restrict__ wd,
                      int d, int inter, GroupRows g, Te* __restrict__ y) {
+  grid_dep_wait();
+  grid_dep_launch();
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * kRowsPerCta + (threadIdx.x >> 5);
   if (r >= rows_of(g)) return;
@@ -116,15 +120,13 @@ cudaError_t launch_swiglu_simt(int dtype, const void* x, const void* w_gate_up,
   const dim3 grid((rows + kRowsPerCta - 1) / kRowsPerCta,
                   (inter + kColsPerCta - 1) / kColsPerCta);
   if (dtype == 0)
-    swiglu_simt_kernel<float><<<grid, kRowsPerCta * 32, 0, stream>>>(
-        static_cast<const float*>(x), static_cast<const float*>(w_gate_up), d,
-        inter, g, static_cast<float*>(act));
-  else
-    swiglu_simt_kernel<__nv_bfloat16><<<grid, kRowsPerCta * 32, 0, stream>>>(
-        static_cast<const __nv_bfloat16*>(x),
-        static_cast<const __nv_bfloat16*>(w_gate_up), d, inter, g,
-        static_cast<__nv_bfloat16*>(act));
-  return cudaGetLastError();
+    return launch_pdl(swiglu_simt_kernel<float>, grid, dim3(kRowsPerCta * 32), 0, stream,
+                      static_cast<const float*>(x), static_cast<const float*>(w_gate_up), d,
+                      inter, g, static_cast<float*>(act));
+  return launch_pdl(swiglu_simt_kernel<__nv_bfloat16>, grid, dim3(kRowsPerCta * 32), 0, stream,
+                    static_cast<const __nv_bfloat16*>(x),
+                    static_cast<const __nv_bfloat16*>(w_gate_up), d, inter, g,
+                    static_cast<__nv_bfloat16*>(act));
 }
 
 cudaError_t launch_down_simt(int dtype, const void* act, const void* w_down,
@@ -135,15 +137,13 @@ cudaError_t launch_down_simt(int dtype, const void* act, const void* w_down,
   const dim3 grid((rows + kRowsPerCta - 1) / kRowsPerCta,
                   (d + kColsPerCta - 1) / kColsPerCta);
   if (dtype == 0)
-    down_simt_kernel<float><<<grid, kRowsPerCta * 32, 0, stream>>>(
-        static_cast<const float*>(act), static_cast<const float*>(w_down), d,
-        inter, g, static_cast<float*>(y));
-  else
-    down_simt_kernel<__nv_bfloat16><<<grid, kRowsPerCta * 32, 0, stream>>>(
-        static_cast<const __nv_bfloat16*>(act),
-        static_cast<const __nv_bfloat16*>(w_down), d, inter, g,
-        static_cast<__nv_bfloat16*>(y));
-  return cudaGetLastError();
+    return launch_pdl(down_simt_kernel<float>, grid, dim3(kRowsPerCta * 32), 0, stream,
+                      static_cast<const float*>(act), static_cast<const float*>(w_down), d,
+                      inter, g, static_cast<float*>(y));
+  return launch_pdl(down_simt_kernel<__nv_bfloat16>, grid, dim3(kRowsPerCta * 32), 0, stream,
+                    static_cast<const __nv_bfloat16*>(act),
+                    static_cast<const __nv_bfloat16*>(w_down), d, inter, g,
+                    static_cast<__nv_bfloat16*>(y));
 }
 
 }  // namespace rx

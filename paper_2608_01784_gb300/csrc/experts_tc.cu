@@ -250,6 +250,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  grid_dep_wait();  // the tile count and every operand come from earlier kernels
+  grid_dep_launch();
   const int ntiles = total_tiles(p);
   const int nk = p.K / BK;
 
@@ -461,8 +463,8 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);
-  kernel<<<grid, kThreads, C::kSmemBytes, stream>>>(*a.map_a, *a.map_b, p);
-  return cudaGetLastError();
+  return launch_pdl(kernel, dim3(grid), dim3(kThreads), C::kSmemBytes, stream, *a.map_a,
+                    *a.map_b, p);
 }
 
 // ===========================================================================
@@ -607,6 +609,8 @@ __global__ void __launch_bounds__(kThreads2, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  grid_dep_wait();
+  grid_dep_launch();
   // tiles are 256 rows (both CTAs) x 256 columns; mt_prefix counts 256-row tiles
   const int ntiles = total_tiles(p);
   const int nk = p.K / BK;
@@ -828,13 +832,15 @@ cudaError_t launch_pair_impl(const TcGemmArgs& a, cudaStream_t stream) {
   cfg.blockDim = dim3(kThreads2);
   cfg.dynamicSmemBytes = C::kSmemBytes;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kernel, *a.map_a, *a.map_b, p);
 }
 

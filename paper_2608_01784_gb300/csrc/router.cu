@@ -87,6 +87,8 @@ __global__ void __launch_bounds__(LogitsCfg<Tin, TM, TN, WT, WE>::kThreads)
   using C = LogitsCfg<Tin, TM, TN, WT, WE>;
   constexpr int BT = C::BT, BE = C::BE, R = C::kRows, NT = C::kThreads;
   extern __shared__ __align__(16) uint8_t smem_l[];
+  grid_dep_wait();
+  grid_dep_launch();
   float* cbuf = reinterpret_cast<float*>(smem_l + kStagesL * C::kRawStage);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ty = lane >> 2, tx = lane & 3;
@@ -209,6 +211,8 @@ __global__ void __launch_bounds__(kSelWarps * 32)
                   uint32_t* __restrict__ err) {
   __shared__ float s_z[kSelWarps][32];
   __shared__ int32_t s_e[kSelWarps][32];
+  grid_dep_wait();
+  grid_dep_launch();
   const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t = blockIdx.x * kSelWarps + wid;
   if (t >= T) return;
@@ -307,6 +311,8 @@ __global__ void __launch_bounds__(kThreadsS)
   constexpr int kHBytes = BT * kRowBytes;
   constexpr int kStageBytes = (BT + BE) * kRowBytes;
   extern __shared__ __align__(16) uint8_t smem_s[];
+  grid_dep_wait();
+  grid_dep_launch();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ty = lane >> 2, tx = lane & 3;
   const int t0 = blockIdx.x * BT;
@@ -445,6 +451,8 @@ __global__ void __launch_bounds__(MxCfg<LY, TM, TN, WT, WE, S, KC>::NT)
   constexpr int kRB = C::kRowBytes;
   constexpr int kVecs = KC / 8;  // 16-byte vectors per row per chunk
   extern __shared__ __align__(16) uint8_t smem_m[];
+  grid_dep_wait();
+  grid_dep_launch();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ty = lane / LX, tx = lane % LX;
   const int wt = warp / WE, we = warp % WE;
@@ -601,19 +609,20 @@ cudaError_t launch_router_select(const float* z, const int32_t* k, int T,
   const dim3 grid((T + kSelWarps - 1) / kSelWarps);
   const dim3 block(kSelWarps * 32);
   const int r = renorm ? 1 : 0;
+  cudaError_t e;
   if (E <= 32)
-    select_kernel<1><<<grid, block, 0, stream>>>(z, k, T, E, k_max, r, ids, alpha, err);
+    e = launch_pdl(select_kernel<1>, grid, block, 0, stream, z, k, T, E, k_max, r, ids, alpha, err);
   else if (E <= 64)
-    select_kernel<2><<<grid, block, 0, stream>>>(z, k, T, E, k_max, r, ids, alpha, err);
+    e = launch_pdl(select_kernel<2>, grid, block, 0, stream, z, k, T, E, k_max, r, ids, alpha, err);
   else if (E <= 128)
-    select_kernel<4><<<grid, block, 0, stream>>>(z, k, T, E, k_max, r, ids, alpha, err);
+    e = launch_pdl(select_kernel<4>, grid, block, 0, stream, z, k, T, E, k_max, r, ids, alpha, err);
   else if (E <= 256)
-    select_kernel<8><<<grid, block, 0, stream>>>(z, k, T, E, k_max, r, ids, alpha, err);
+    e = launch_pdl(select_kernel<8>, grid, block, 0, stream, z, k, T, E, k_max, r, ids, alpha, err);
   else if (E <= 512)
-    select_kernel<16><<<grid, block, 0, stream>>>(z, k, T, E, k_max, r, ids, alpha, err);
+    e = launch_pdl(select_kernel<16>, grid, block, 0, stream, z, k, T, E, k_max, r, ids, alpha, err);
   else
-    select_kernel<32><<<grid, block, 0, stream>>>(z, k, T, E, k_max, r, ids, alpha, err);
-  return cudaGetLastError();
+    e = launch_pdl(select_kernel<32>, grid, block, 0, stream, z, k, T, E, k_max, r, ids, alpha, err);
+  return e;
 }
 
 }  // namespace rx
