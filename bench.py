@@ -40,6 +40,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
+from paper_2608_01784_gb300 import replicas as R  # noqa: E402
 from paper_2608_01784_gb300 import workloads as W  # noqa: E402
 
 METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
@@ -49,13 +50,13 @@ METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
 # ncu capture of the current kernel on the same workload
 # (profiles/grouped_gemm_llada_moe_T1024.md); workloads without a capture of
 # the current kernel report null.
-NCU_TRAFFIC_BYTES = {"llada_moe": 568417024}
+NCU_TRAFFIC_BYTES = {"llada_moe": 568977664}
 
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="reflex", choices=["reflex", "reference"])
     ap.add_argument("--config", default="llada_moe",
@@ -220,7 +221,6 @@ def run_reference(args, cfg, rank, world):
 # ---------------------------------------------------------------------------
 def run_gpu(args, cfg, rank, world, local_rank):
     import torch
-    import torch.distributed as dist
     from paper_2608_01784_gb300 import _binding as B
     from paper_2608_01784_gb300 import api, build
 
@@ -228,7 +228,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
     B.load()
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    seed = args.seed + rank
+    seed = R.rank_seed(args.seed, rank)
     layer = W.make_layer(cfg, seed)
     state = W.make_state(cfg, seed)
     T, d, E, I, S, km = cfg.T, cfg.d, cfg.E, cfg.inter, cfg.shared_inter, cfg.k_max
@@ -258,9 +258,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
         moe.forward(h, k_buf, out, F | B.REFLEX_STAGE_EXPERT_DOWN | B.REFLEX_STAGE_COMBINE)
 
     def barrier():
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize(dev)
+        R.barrier(world, dev)
 
     def timed(params, steps, warmup, up_times=None):
         for _ in range(warmup):
@@ -280,11 +278,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
         return ms
 
     def max_over_ranks(x: float) -> float:
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return R.max_over_ranks(x, world, dev)
 
     # correctness gate before timing: counts and routing status clean
     step(p_reflex)
@@ -342,7 +336,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
     if rank != 0:
         return
     peaks = load_peaks()
-    tokens_per_s = T * world / (ms_step * 1e-3)
+    tokens_per_s = R.whole_job_rate(T, world, ms_step)
     flops_step = 6.0 * d * I * pairs          # Eq. 10, routed experts
     # dominant kernel: grouped gate/up GEMM; algorithmic bytes per launch =
     # gate/up weights of the experts that received pairs + gathered rows read
@@ -386,10 +380,10 @@ def run_gpu(args, cfg, rank, world, local_rank):
         layer_roofline_frac=t_roof / (ms_step * 1e-3),
         avg_k=pairs / T, pairs=pairs,
         fixed_topk=dict(k=cfg.k_base, pairs=pairs_fixed, ms_per_step=ms_fixed,
-                        value=T * world / (ms_fixed * 1e-3),
+                        value=R.whole_job_rate(T, world, ms_fixed),
                         expert_tflops=6.0 * d * I * pairs_fixed * world / (ms_fixed * 1e-3) / 1e12),
         roofline=roof,
-        e2e=dict(value=T * world / (ms_e2e * 1e-3), unit="tokens/s",
+        e2e=dict(value=R.whole_job_rate(T, world, ms_e2e), unit="tokens/s",
                  h2d_bytes_per_step=h2d, d2h_bytes_per_step=d2h,
                  ms_per_step=ms_e2e),
         gpu_launches=launches_per_step * args.steps,
@@ -428,7 +422,6 @@ def _device_weights(cfg, seed, dev, std):
 
 def run_stack(args, rank, world, local_rank):
     import torch
-    import torch.distributed as dist
     from paper_2608_01784_gb300 import _binding as B
     from paper_2608_01784_gb300 import api, build
 
@@ -437,7 +430,7 @@ def run_stack(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     cfg = W.CONFIGS["llada_moe_b32"]
-    seed = args.seed + rank
+    seed = R.rank_seed(args.seed, rank)
     T, d, E, I, km = cfg.T, cfg.d, cfg.E, cfg.inter, cfg.k_max
     state = api.state_to_device(W.make_state(cfg, seed), dev)
     h0 = api.layer_to_device({"hidden": W.make_layer(cfg.with_(E=1, inter=64), seed)["hidden"]},
@@ -465,23 +458,14 @@ def run_stack(args, rank, world, local_rank):
     def timed(params, steps, warmup):
         for _ in range(warmup):
             forward(params)
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize(dev)
+        R.barrier(world, dev)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         for _ in range(steps):
             forward(params)
         b.record(stream)
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize(dev)
-        ms = a.elapsed_time(b) / steps
-        if world > 1:
-            t = torch.tensor([ms], dtype=torch.float64, device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
-        return ms
+        R.barrier(world, dev)
+        return R.max_over_ranks(a.elapsed_time(b) / steps, world, dev)
 
     p_reflex = B.make_params(**cfg.alloc_params())
     p_fixed = B.make_params(**cfg.alloc_params(delta_role=0, delta_cur=0))
@@ -504,7 +488,7 @@ def run_stack(args, rank, world, local_rank):
     flops = 6.0 * d * I * pairs * L
     flops_fixed = 6.0 * d * I * pairs_fixed * L
     line = dict(
-        metric=METRIC, value=T * world / (ms * 1e-3), unit="tokens/s", n_gpus=world,
+        metric=METRIC, value=R.whole_job_rate(T, world, ms), unit="tokens/s", n_gpus=world,
         steps=args.steps, warmup=args.warmup, ms_per_step=ms, higher_is_better=True,
         scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic",
         config=dict(workload="llada_moe_stack16",
@@ -517,7 +501,7 @@ def run_stack(args, rank, world, local_rank):
         expert_frac_of_bf16_peak=flops / (ms * 1e-3) / 1e12 / peaks["bf16_sustained"],
         avg_k=pairs / T, pairs_per_layer=pairs,
         fixed_topk=dict(k=cfg.k_base, pairs_per_layer=pairs_fixed, ms_per_step=ms_fixed,
-                        value=T * world / (ms_fixed * 1e-3),
+                        value=R.whole_job_rate(T, world, ms_fixed),
                         expert_tflops=flops_fixed * world / (ms_fixed * 1e-3) / 1e12),
         gpu_launches=args.steps * (1 + 10 * L),
         clocks=dict(sm_mhz=clocks["sm_mhz"], sm_max_mhz=clocks["sm_max_mhz"],
@@ -589,16 +573,10 @@ def run_sweep(args, rank, world, local_rank):
 def main():
     args = parse()
     cfg = W.CONFIGS.get(args.config, W.CONFIGS["llada_moe_b32"])
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
-    if world > 1:
-        import torch
-        import torch.distributed as dist
-        backend = "nccl" if args.impl == "reflex" else "gloo"
-        if backend == "nccl":
-            torch.cuda.set_device(local_rank)
-        dist.init_process_group(backend=backend)
+    ri = R.rank_info()
+    world, rank, local_rank = ri.world, ri.rank, ri.local_rank
+    # the GPU arm reduces on the GPUs (NCCL); the reference arm is host-only
+    R.init(world, "nccl" if args.impl == "reflex" else "gloo", local_rank)
     try:
         if args.impl == "reference":
             run_reference(args, cfg, rank, world)
@@ -610,9 +588,7 @@ def main():
         else:
             run_gpu(args, cfg, rank, world, local_rank)
     finally:
-        if world > 1:
-            import torch.distributed as dist
-            dist.destroy_process_group()
+        R.finalize(world)
 
 
 if __name__ == "__main__":
