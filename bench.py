@@ -64,6 +64,8 @@ def parse():
     ap.add_argument("--sweep", action="store_true",
                     help="token-count x count-skew sweep on the LLaDA2.0-mini "
                          "layer (one JSON line per point)")
+    ap.add_argument("--ablation", action="store_true",
+                    help="REFLEX and its App. C allocation ablations on one layer")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -246,36 +248,42 @@ def run_gpu(args, cfg, rank, world, local_rank):
     F = B.REFLEX_FLAG_RENORM_TOPK
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
 
-    def step(params, up_events=None, hidden=None):
-        api.allocate(ds, params, E, stream, k_buf, k_sum, st)
-        h = dl["hidden"] if hidden is None else hidden
+    # every call takes the current stream, so the steps can be captured into
+    # CUDA graphs (the library never synchronises with the host)
+    def step(params, hidden=None):
+        api.allocate(ds, params, E, None, k_buf, k_sum, st)
+        moe.forward(dl["hidden"] if hidden is None else hidden, k_buf, out, F)
+
+    def staged_step(params, up_events):
+        # the same work as step(), split so that events bracket the gate/up GEMM
+        api.allocate(ds, params, E, None, k_buf, k_sum, st)
+        h = dl["hidden"]
         moe.forward(h, k_buf, out, F | B.REFLEX_STAGE_ROUTE | B.REFLEX_STAGE_DISPATCH)
-        if up_events is not None:
-            up_events[0].record(stream)
+        up_events[0].record()
         moe.forward(h, k_buf, out, F | B.REFLEX_STAGE_EXPERT_UP)
-        if up_events is not None:
-            up_events[1].record(stream)
+        up_events[1].record()
         moe.forward(h, k_buf, out, F | B.REFLEX_STAGE_EXPERT_DOWN | B.REFLEX_STAGE_COMBINE)
+
+    def graph_of(fn):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="relaxed"):
+            fn()
+        return g
 
     def barrier():
         R.barrier(world, dev)
 
-    def timed(params, steps, warmup, up_times=None):
+    def timed(graph, replays, warmup):
         for _ in range(warmup):
-            step(params)
+            graph.replay()
         barrier()
         start, stop = (torch.cuda.Event(enable_timing=True) for _ in range(2))
-        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)]
-               for _ in range(steps)] if up_times is not None else None
         start.record(stream)
-        for i in range(steps):
-            step(params, evs[i] if evs else None)
+        for _ in range(replays):
+            graph.replay()
         stop.record(stream)
         barrier()
-        ms = start.elapsed_time(stop)
-        if up_times is not None:
-            up_times.extend(e[0].elapsed_time(e[1]) for e in evs)
-        return ms
+        return start.elapsed_time(stop)
 
     def max_over_ranks(x: float) -> float:
         return R.max_over_ranks(x, world, dev)
@@ -292,46 +300,94 @@ def run_gpu(args, cfg, rank, world, local_rank):
     torch.cuda.synchronize(dev)
     pairs_fixed = int(k_sum.item())
 
-    # ---- timed region: REFLEX counts ----
+    # ---- timed region: REFLEX counts, one step per graph replay ----
+    g_reflex = graph_of(lambda: step(p_reflex))
     clk = ClockSampler(local_rank)
     clk.start()
-    up_times: list[float] = []
-    ms = timed(p_reflex, args.steps, args.warmup, up_times)
+    ms = timed(g_reflex, args.steps, args.warmup)
     clocks = clk.stop()
     ms = max_over_ranks(ms)
     ms_step = ms / args.steps
-    # ---- same kernels at fixed top-K_base ----
-    ms_fixed = max_over_ranks(timed(p_fixed, max(1, args.steps // 2), 2)) / max(1, args.steps // 2)
+    # ---- gate/up GEMM launches: the same step with events around the GEMM,
+    # 16 steps per graph; the durations of the last replay are averaged ----
+    NS = 16
+    try:   # timestamps recorded by graph nodes need external event records
+        up_evs = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+                  for _ in range(NS)]
 
-    # ---- end to end from pinned host buffers ----
+        def staged_block():
+            for e in up_evs:
+                staged_step(p_reflex, e)
+        timed(graph_of(staged_block), max(1, min(args.steps, 400) // NS), 1)
+    except TypeError:  # older torch: the same staged steps, launched eagerly
+        up_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(NS)]
+        for _ in range(2):
+            for e in up_evs:
+                staged_step(p_reflex, e)
+        barrier()
+    up_times = [e[0].elapsed_time(e[1]) for e in up_evs]
+    # ---- same kernels at fixed top-K_base ----
+    g_fixed = graph_of(lambda: step(p_fixed))
+    n_fixed = max(1, args.steps // 2)
+    ms_fixed = max_over_ranks(timed(g_fixed, n_fixed, 2)) / n_fixed
+
+    # ---- end to end from pinned host buffers: every step uploads its inputs
+    # (hidden states and per-token state) and reads its output back.  Copies
+    # run on a copy stream with two buffer sets, so the upload of step i+1 and
+    # the read-back of step i-1 overlap the kernels of step i ----
     host_in = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
                for k, v in state.items()}
     host_h = torch.from_numpy(np.ascontiguousarray(layer["hidden"]).view(
         np.int16 if cfg.dtype == "bf16" else np.float32)).pin_memory()
-    host_out = torch.empty((T, d), dtype=moe.tdtype).pin_memory()
-    dev_h = torch.empty_like(dl["hidden"])
+    host_out = [torch.empty((T, d), dtype=moe.tdtype).pin_memory() for _ in range(2)]
+    dev_state = [{k: torch.empty_like(v) for k, v in ds.items()} for _ in range(2)]
+    dev_h = [torch.empty_like(dl["hidden"]) for _ in range(2)]
+    dev_out = [torch.empty_like(out) for _ in range(2)]
     h2d = sum(int(v.numel() * v.element_size()) for v in host_in.values()) + \
         int(host_h.numel() * host_h.element_size())
-    d2h = int(host_out.numel() * host_out.element_size())
+    d2h = int(host_out[0].numel() * host_out[0].element_size())
+    copy_s = torch.cuda.Stream(dev)
+    ev_up = [torch.cuda.Event() for _ in range(2)]
+    ev_done = [torch.cuda.Event() for _ in range(2)]
+    ev_read = [torch.cuda.Event() for _ in range(2)]
 
-    def e2e_step():
-        for k, v in host_in.items():
-            ds[k].copy_(v, non_blocking=True)
-        dev_h.view(host_h.dtype).copy_(host_h, non_blocking=True)
-        step(p_reflex, hidden=dev_h)
-        host_out.copy_(out, non_blocking=True)
+    def e2e_run(n: int):
+        for i in range(n + 1):
+            b = i & 1
+            if i < n:
+                with torch.cuda.stream(copy_s):   # upload step i
+                    copy_s.wait_event(ev_done[b])  # step i-2 finished with buffer b
+                    for k, v in host_in.items():
+                        dev_state[b][k].copy_(v, non_blocking=True)
+                    dev_h[b].view(host_h.dtype).copy_(host_h, non_blocking=True)
+                    ev_up[b].record(copy_s)
+                stream.wait_event(ev_up[b])
+                stream.wait_event(ev_read[b])      # read-back of step i-2 done
+                api.allocate(dev_state[b], p_reflex, E, None, k_buf, k_sum, st)
+                moe.forward(dev_h[b], k_buf, dev_out[b], F)
+                ev_done[b].record(stream)
+            if i > 0:
+                pb = (i - 1) & 1
+                with torch.cuda.stream(copy_s):   # read back step i-1
+                    copy_s.wait_event(ev_done[pb])
+                    host_out[pb].copy_(dev_out[pb], non_blocking=True)
+                    ev_read[pb].record(copy_s)
+        stream.wait_event(ev_read[(n - 1) & 1])
 
-    for _ in range(max(3, args.warmup // 2)):
-        e2e_step()
+    e2e_run(max(3, args.warmup // 2))
     barrier()
     n_e2e = max(3, args.steps // 2)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(n_e2e):
-        e2e_step()
+    copy_s.wait_event(e0)
+    e2e_run(n_e2e)
     e1.record(stream)
     barrier()
     ms_e2e = max_over_ranks(e0.elapsed_time(e1)) / n_e2e
+    # the end-to-end outputs are those of the resident-input step, bit for bit
+    g_reflex.replay()
+    torch.cuda.synchronize(dev)
+    assert torch.equal(host_out[(n_e2e - 1) & 1], out.cpu())
 
     if rank != 0:
         return
@@ -375,7 +431,11 @@ def run_gpu(args, cfg, rank, world, local_rank):
         if cfg.dtype == "bf16" else "f32", data="synthetic",
         config=dict(workload=cfg.name, description=cfg.description,
                     tokens_per_step=T, parallelism=f"replicas{world}",
-                    l2="no flush: expert weights > 129 MB L2 stream from HBM every step"),
+                    l2="no flush: expert weights > 129 MB L2 stream from HBM every step",
+                    timing="CUDA-graph replay of one step (allocation + forward) per "
+                           "timed iteration; e2e: eager API calls, each step's upload "
+                           "and read-back from pinned host memory on a copy stream, "
+                           "double-buffered so they overlap the neighbouring steps"),
         expert_tflops=flops_step * world / (ms_step * 1e-3) / 1e12,
         layer_roofline_frac=t_roof / (ms_step * 1e-3),
         avg_k=pairs / T, pairs=pairs,
@@ -570,6 +630,83 @@ def run_sweep(args, rank, world, local_rank):
         T *= 2
 
 
+ABLATIONS = [  # (name, allocation overrides): REFLEX and its App. C ablations
+    ("reflex", {}),
+    ("rrb_only", dict(delta_cur=0)),
+    ("fger_only", dict(delta_role=0)),
+    ("role_shuffled_rrb", dict(delta_cur=0, role_shuffle=1)),
+    ("frontier_only", dict(signal=1)),
+    ("progress_only", dict(signal=2)),
+    ("confidence_only", dict(signal=3)),
+    ("uncertainty_only", dict(signal=4)),
+    ("fixed_topk", dict(delta_role=0, delta_cur=0)),
+]
+
+
+def run_ablation(args, rank, world, local_rank):
+    """One JSON line per allocation variant on the same layer and state:
+    realised counts (avg k, pairs), the allocation kernel's own time and the
+    whole step (allocation + layer).  The role shuffle draws a new seed every
+    step (one permutation per denoising forward)."""
+    import torch
+    from paper_2608_01784_gb300 import _binding as B
+    from paper_2608_01784_gb300 import api, build
+
+    build.build()
+    B.load()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    cfg = W.CONFIGS.get(args.config, W.CONFIGS["llada_moe"])
+    T, d, E, I, S, km = cfg.T, cfg.d, cfg.E, cfg.inter, cfg.shared_inter, cfg.k_max
+    dl = api.layer_to_device(W.make_layer(cfg, args.seed), cfg.dtype, dev)
+    ds = api.state_to_device(W.make_state(cfg, args.seed), dev)
+    moe = api.MoELayer(dl, dtype=cfg.dtype, d=d, E=E, inter=I, shared_inter=S,
+                       k_max=km, max_tokens=T, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    k_buf = torch.empty(T, dtype=torch.int32, device=dev)
+    k_sum = torch.zeros(1, dtype=torch.int64, device=dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    out = torch.empty((T, d), dtype=moe.tdtype, device=dev)
+    F = B.REFLEX_FLAG_RENORM_TOPK
+    steps = max(20, min(args.steps, 500))
+
+    def timed(fn):
+        for i in range(3):
+            fn(i)
+        torch.cuda.synchronize(dev)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(steps):
+            fn(i)
+        b.record(stream)
+        torch.cuda.synchronize(dev)
+        return a.elapsed_time(b) / steps
+
+    for name, over in ABLATIONS:
+        params = [B.make_params(**cfg.alloc_params(**over, shuffle_seed=args.seed + i))
+                  for i in range(steps)]
+
+        def alloc(i):
+            api.allocate(ds, params[i % steps], E, stream, k_buf, k_sum, st)
+
+        def step(i):
+            alloc(i)
+            moe.forward(dl["hidden"], k_buf, out, F)
+
+        alloc(0)
+        moe.forward(dl["hidden"], k_buf, out, F)
+        torch.cuda.synchronize(dev)
+        assert B.reflex_read_status(st) == B.REFLEX_OK and moe.status() == B.REFLEX_OK
+        pairs = int(k_sum.item())
+        ms_alloc = timed(alloc)
+        ms = timed(step)
+        line = dict(ablation=name, workload=cfg.name, tokens=T, avg_k=pairs / T,
+                    pairs=pairs, alloc_us=1e3 * ms_alloc, ms_per_step=ms,
+                    tokens_per_s=T / (ms * 1e-3),
+                    expert_tflops=6.0 * d * I * pairs / (ms * 1e-3) / 1e12)
+        print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     cfg = W.CONFIGS.get(args.config, W.CONFIGS["llada_moe_b32"])
@@ -583,6 +720,9 @@ def main():
         elif args.sweep:
             if rank == 0:
                 run_sweep(args, rank, world, local_rank)
+        elif args.ablation:
+            if rank == 0:
+                run_ablation(args, rank, world, local_rank)
         elif args.config == "llada_moe_stack16":
             run_stack(args, rank, world, local_rank)
         else:

@@ -88,11 +88,42 @@ typedef struct {
                            velocity clip, > 0                               */
     float v_ref;        /* velocity reference of Eq. 7                      */
     float tau;          /* gate temperature of Eq. 6-7, > 0                 */
+    int32_t signal;     /* rank key of the Eq. 9 groups: REFLEX_SIGNAL_*    */
+    int32_t role_shuffle; /* 1: permute each sequence's final counts among
+                           its positions (Role-Shuffled RRB, App. C); the
+                           multiset and sum of the counts are unchanged.
+                           Sequences longer than 4096 tokens are left as
+                           they are and flag REFLEX_ECAPACITY.              */
+    uint64_t shuffle_seed; /* seed of the shuffle's splitmix64 stream       */
 } reflex_alloc_params;
+
+/* Rank keys for the FGER groups (Sec. 4.3; signal ablation of App. C).  The
+ * top floor(q |J_h|) tokens by (key desc, position asc) gain delta_cur, the
+ * bottom ones lose it.
+ *   FPS          S = F * P (Eq. 8), the REFLEX default
+ *   FRONTIER     F alone (Eq. 6)
+ *   PROGRESS     P alone (Eq. 7; 1 with fewer than two observations)
+ *   CONFIDENCE   c^{t-1}
+ *   UNCERTAINTY  1 - c^{t-1} (fp32)
+ * RRB Only and FGER Only (Sec. 5.3) are parameter settings: delta_cur = 0 and
+ * delta_role = 0 respectively. */
+#define REFLEX_SIGNAL_FPS 0
+#define REFLEX_SIGNAL_FRONTIER 1
+#define REFLEX_SIGNAL_PROGRESS 2
+#define REFLEX_SIGNAL_CONFIDENCE 3
+#define REFLEX_SIGNAL_UNCERTAINTY 4
+
+/* Role shuffle.  Token i of a sequence gets the key
+ *   key_i = high 32 bits of splitmix64 output number i + 1 for shuffle_seed
+ * (splitmix64: state_n = seed + n * 0x9e3779b97f4a7c15, output = the
+ * Stafford "mix13" finaliser of state_n, Steele, Lea and Flood 2014), i the
+ * token's index in the batch; with r_i the rank of (key_i, i) in ascending
+ * order within the sequence, token i receives the count the unshuffled
+ * allocation gives to the sequence's r_i-th position. */
 
 /* Fills the Sec. 5.1 defaults: k_base 8, delta_role 4, delta_cur 2, q 0.25,
  * theta 0.9, w_cf 0.30 (LLaDA-MoE; 0.25 for LLaDA2.0-mini), v_ref 0.01,
- * tau 0.05, and the clip [k_min, k_max] = [2, 12]. */
+ * tau 0.05, the clip [k_min, k_max] = [2, 12], signal FPS, no shuffle. */
 void reflex_default_params(reflex_alloc_params* p);
 
 /*

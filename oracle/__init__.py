@@ -82,6 +82,15 @@ def _load():
     lib.oracle_allocate.argtypes = [p, p, p, p, p, p, p, i32, i32,
                                     i32, i32, i32, i32, i32,
                                     f32, f32, f32, f32, f32, p, p]
+    lib.oracle_allocate_ex.restype = ctypes.c_int
+    lib.oracle_allocate_ex.argtypes = [p, p, p, p, p, p, p, i32, i32,
+                                       i32, i32, i32, i32, i32,
+                                       f32, f32, f32, f32, f32,
+                                       i32, i32, ctypes.c_uint64, p, p]
+    lib.oracle_rank_key.restype = f32
+    lib.oracle_rank_key.argtypes = [i32, f32, f32, i32, f32, f32, f32, f32]
+    lib.oracle_splitmix64.restype = ctypes.c_uint64
+    lib.oracle_splitmix64.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
     lib.oracle_router_logits.restype = None
     lib.oracle_router_logits.argtypes = [i32, p, p, i32, i32, i32, p]
     lib.oracle_select.restype = ctypes.c_int
@@ -135,8 +144,11 @@ def fps(c1, c2, hist, theta, w_cf, v_ref, tau) -> np.ndarray:
 
 def allocate(conf1, conf2, hist_len, masked, block_id, seq_offsets,
              active_block, *, k_min, k_base, k_max, delta_role, delta_cur,
-             q, theta, w_cf, v_ref, tau, return_scores: bool = False):
-    """Per-token expert counts of REFLEX (Eq. 5, Eq. 9, clip); int32 [T]."""
+             q, theta, w_cf, v_ref, tau, signal: int = 0, role_shuffle: int = 0,
+             shuffle_seed: int = 0, return_scores: bool = False):
+    """Per-token expert counts of REFLEX (Eq. 5, Eq. 9, clip); int32 [T].
+    signal / role_shuffle / shuffle_seed select the App. C ablations (rank
+    key of the Eq. 9 groups; Role-Shuffled RRB)."""
     conf1 = _c(conf1, np.float32)
     conf2 = _c(conf2, np.float32)
     hist_len = _c(hist_len, np.uint8)
@@ -148,14 +160,27 @@ def allocate(conf1, conf2, hist_len, masked, block_id, seq_offsets,
     B = active_block.size
     k = np.empty(T, np.int32)
     s = np.empty(T, np.float32)
-    rc = _load().oracle_allocate(
+    rc = _load().oracle_allocate_ex(
         _ptr(conf1), _ptr(conf2), _ptr(hist_len), _ptr(masked),
         _ptr(block_id), _ptr(seq_offsets), _ptr(active_block), T, B,
         k_min, k_base, k_max, delta_role, delta_cur, q, theta, w_cf, v_ref,
-        tau, _ptr(k), _ptr(s))
+        tau, int(signal), int(role_shuffle), int(shuffle_seed) & (2**64 - 1),
+        _ptr(k), _ptr(s))
     if rc != 0:
         raise ValueError("oracle_allocate: invalid input")
     return (k, s) if return_scores else k
+
+
+def rank_key(signal: int, c1: float, c2: float, hist: int, theta: float,
+             w_cf: float, v_ref: float, tau: float) -> float:
+    """Rank key of one J_h member under an App. C signal (0 FPS, 1 F, 2 P,
+    3 c^{t-1}, 4 1 - c^{t-1})."""
+    return float(_load().oracle_rank_key(signal, c1, c2, hist, theta, w_cf, v_ref, tau))
+
+
+def splitmix64(seed: int, n: int) -> int:
+    """Output number n (n >= 1) of the splitmix64 stream seeded with seed."""
+    return int(_load().oracle_splitmix64(seed & (2**64 - 1), n & (2**64 - 1)))
 
 
 def _dtype_code(a: np.ndarray) -> int:

@@ -14,6 +14,11 @@
  *                        Frontier-Guided Expert Reallocation (Sec. 4.3,
  *                        forecast, Eq. 6-8 and Eq. 9), then the clip of every
  *                        count to [K_min, K_max] required by Eq. 3.
+ *   oracle_allocate_ex   the same with the ablations of App. C: the rank key
+ *                        of the Eq. 9 groups (FPS, F only, P only, c^{t-1},
+ *                        1 - c^{t-1}) and Role-Shuffled RRB (a seeded
+ *                        permutation of each sequence's counts; its keys come
+ *                        from splitmix64, Steele, Lea and Flood 2014).
  *   oracle_router_logits router scores r = h . W_r (Sec. 3.2) as a sequential
  *                        fp32 fused-multiply-add chain over the hidden index,
  *                        k = 0 .. d-1, starting from +0 (the summation-order
@@ -119,17 +124,47 @@ static float or_sigmoid(float x) {
 /*   P    = hist>=2 ? sig((v_ref - vbar) / tau) : 1                   Eq.7 */
 /*   S    = F * P                                                     Eq.8 */
 /* ------------------------------------------------------------------------ */
-float oracle_fps(float c1, float c2, int32_t hist, float theta, float w_cf,
-                 float v_ref, float tau) {
+static void or_frontier_progress(float c1, float c2, int32_t hist, float theta,
+                                 float w_cf, float v_ref, float tau,
+                                 float* F_out, float* P_out) {
     float v = (hist >= 2) ? (c1 - c2) : 0.0f;
     float half_w = w_cf * 0.5f;
     float vbar = fminf(fmaxf(v, -half_w), half_w);
     float chat = fminf(fmaxf(c1 + vbar, 0.0f), 1.0f);
     float x1 = ((chat - theta) + w_cf) / tau;
     float x2 = (theta - chat) / tau;
-    float F = or_sigmoid(x1) * or_sigmoid(x2);
-    float P = (hist >= 2) ? or_sigmoid((v_ref - vbar) / tau) : 1.0f;
+    *F_out = or_sigmoid(x1) * or_sigmoid(x2);
+    *P_out = (hist >= 2) ? or_sigmoid((v_ref - vbar) / tau) : 1.0f;
+}
+
+float oracle_fps(float c1, float c2, int32_t hist, float theta, float w_cf,
+                 float v_ref, float tau) {
+    float F, P;
+    or_frontier_progress(c1, c2, hist, theta, w_cf, v_ref, tau, &F, &P);
     return F * P;
+}
+
+/* Rank key of a J_h member under each signal of the App. C ablation:      */
+/*   0 FPS: F * P     1 Frontier: F     2 Progress: P                      */
+/*   3 Confidence: c^{t-1}     4 Uncertainty: 1 - c^{t-1} (fp32)           */
+float oracle_rank_key(int32_t signal, float c1, float c2, int32_t hist,
+                      float theta, float w_cf, float v_ref, float tau) {
+    float F, P;
+    if (signal == 3) return c1;
+    if (signal == 4) return 1.0f - c1;
+    or_frontier_progress(c1, c2, hist, theta, w_cf, v_ref, tau, &F, &P);
+    if (signal == 1) return F;
+    if (signal == 2) return P;
+    return F * P;
+}
+
+/* splitmix64 output number n (n >= 1) of the stream seeded with seed: the  */
+/* state is seed + n * golden gamma, the output its "mix13" finaliser.      */
+uint64_t oracle_splitmix64(uint64_t seed, uint64_t n) {
+    uint64_t z = seed + n * 0x9e3779b97f4a7c15ULL;
+    z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ULL;
+    z = (z ^ (z >> 27)) * 0x94d049bb133111ebULL;
+    return z ^ (z >> 31);
 }
 
 /* ------------------------------------------------------------------------ */
@@ -150,14 +185,27 @@ static int32_t or_role_count(int32_t dist, int32_t k_base, int32_t d_role) {
     return k_base - d_role;
 }
 
-int oracle_allocate(const float* conf1, const float* conf2,
-                    const uint8_t* hist_len, const uint8_t* masked,
-                    const int32_t* block_id, const int32_t* seq_off,
-                    const int32_t* active_block, int32_t T, int32_t B,
-                    int32_t k_min, int32_t k_base, int32_t k_max,
-                    int32_t delta_role, int32_t delta_cur, float q,
-                    float theta, float w_cf, float v_ref, float tau,
-                    int32_t* k_out, float* s_out) {
+typedef struct {
+    uint32_t key;
+    int32_t pos;
+} or_key_pos;
+
+static int or_cmp_key_pos(const void* a, const void* b) {
+    const or_key_pos* x = (const or_key_pos*)a;
+    const or_key_pos* y = (const or_key_pos*)b;
+    if (x->key != y->key) return x->key < y->key ? -1 : 1;
+    return x->pos < y->pos ? -1 : (x->pos > y->pos ? 1 : 0);
+}
+
+int oracle_allocate_ex(const float* conf1, const float* conf2,
+                       const uint8_t* hist_len, const uint8_t* masked,
+                       const int32_t* block_id, const int32_t* seq_off,
+                       const int32_t* active_block, int32_t T, int32_t B,
+                       int32_t k_min, int32_t k_base, int32_t k_max,
+                       int32_t delta_role, int32_t delta_cur, float q,
+                       float theta, float w_cf, float v_ref, float tau,
+                       int32_t signal, int32_t role_shuffle, uint64_t shuffle_seed,
+                       int32_t* k_out, float* s_out) {
     if (T < 0 || B < 0) return OR_EINVAL;
     if (T > 0 && seq_off[B] != T) return OR_EINVAL;
     for (int32_t i = 0; i < T; ++i) {
@@ -180,8 +228,8 @@ int oracle_allocate(const float* conf1, const float* conf2,
         for (int32_t i = lo; i < hi; ++i) {
             if (block_id[i] == a && masked[i] && hist_len[i] >= 1) {
                 idx[nj] = i;
-                sc[nj] = oracle_fps(conf1[i], conf2[i], hist_len[i], theta,
-                                    w_cf, v_ref, tau);
+                sc[nj] = oracle_rank_key(signal, conf1[i], conf2[i], hist_len[i],
+                                         theta, w_cf, v_ref, tau);
                 if (s_out) s_out[i] = sc[nj];
                 ++nj;
             }
@@ -216,8 +264,39 @@ int oracle_allocate(const float* conf1, const float* conf2,
             if (k > k_max) k = k_max;
             k_out[i] = k;
         }
+        /* step 5 (Role-Shuffled RRB): sort the positions by (key, position);
+           the token in sorted place r receives the count of position lo + r */
+        if (role_shuffle && hi > lo) {
+            int32_t len = hi - lo;
+            or_key_pos* kp = (or_key_pos*)malloc(sizeof(or_key_pos) * (size_t)len);
+            int32_t* old = (int32_t*)malloc(sizeof(int32_t) * (size_t)len);
+            for (int32_t r = 0; r < len; ++r) {
+                kp[r].key = (uint32_t)(oracle_splitmix64(shuffle_seed,
+                                                         (uint64_t)(lo + r) + 1) >> 32);
+                kp[r].pos = lo + r;
+                old[r] = k_out[lo + r];
+            }
+            qsort(kp, (size_t)len, sizeof(or_key_pos), or_cmp_key_pos);
+            for (int32_t r = 0; r < len; ++r) k_out[kp[r].pos] = old[r];
+            free(kp);
+            free(old);
+        }
     }
     return OR_OK;
+}
+
+int oracle_allocate(const float* conf1, const float* conf2,
+                    const uint8_t* hist_len, const uint8_t* masked,
+                    const int32_t* block_id, const int32_t* seq_off,
+                    const int32_t* active_block, int32_t T, int32_t B,
+                    int32_t k_min, int32_t k_base, int32_t k_max,
+                    int32_t delta_role, int32_t delta_cur, float q,
+                    float theta, float w_cf, float v_ref, float tau,
+                    int32_t* k_out, float* s_out) {
+    return oracle_allocate_ex(conf1, conf2, hist_len, masked, block_id, seq_off,
+                              active_block, T, B, k_min, k_base, k_max, delta_role,
+                              delta_cur, q, theta, w_cf, v_ref, tau, 0, 0, 0,
+                              k_out, s_out);
 }
 
 /* ------------------------------------------------------------------------ */

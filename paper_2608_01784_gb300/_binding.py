@@ -27,6 +27,11 @@ REFLEX_DTYPE_BF16 = 1
 REFLEX_FLAG_RENORM_TOPK = 0x1
 REFLEX_FLAG_SIMT_EXPERTS = 0x2
 REFLEX_FLAG_RESIDUAL = 0x4
+REFLEX_SIGNAL_FPS = 0
+REFLEX_SIGNAL_FRONTIER = 1
+REFLEX_SIGNAL_PROGRESS = 2
+REFLEX_SIGNAL_CONFIDENCE = 3
+REFLEX_SIGNAL_UNCERTAINTY = 4
 REFLEX_STAGE_ROUTE = 0x100
 REFLEX_STAGE_DISPATCH = 0x200
 REFLEX_STAGE_EXPERT_UP = 0x400
@@ -46,7 +51,9 @@ class reflex_alloc_params(ctypes.Structure):
                 ("k_max", ctypes.c_int32), ("delta_role", ctypes.c_int32),
                 ("delta_cur", ctypes.c_int32), ("q", ctypes.c_float),
                 ("theta", ctypes.c_float), ("w_cf", ctypes.c_float),
-                ("v_ref", ctypes.c_float), ("tau", ctypes.c_float)]
+                ("v_ref", ctypes.c_float), ("tau", ctypes.c_float),
+                ("signal", ctypes.c_int32), ("role_shuffle", ctypes.c_int32),
+                ("shuffle_seed", ctypes.c_uint64)]
 
 
 class reflex_route_record(ctypes.Structure):

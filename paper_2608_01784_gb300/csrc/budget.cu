@@ -12,9 +12,12 @@
 // The score is computed in fp32 with one rounding per operation, in a fixed
 // order, and with an exp written here from Cody & Waite's argument reduction
 // and a degree-7 Taylor polynomial, so that the ranking (an integer result)
-// is reproducible bit for bit.
+// is reproducible bit for bit.  The ablations of App. C are options: other
+// rank keys (F, P, c^{t-1}, 1 - c^{t-1}) and a seeded permutation of each
+// sequence's final counts (Role-Shuffled RRB).
 #include "common.cuh"
 #include "internal.h"
+#include "reflex.h"
 
 namespace rx {
 namespace {
@@ -59,20 +62,37 @@ __device__ __forceinline__ float sigmoid_cw(float x) {
   return __fdiv_rn(1.0f, __fadd_rn(1.0f, exp_cw(-x)));
 }
 
-// Frontier-Progress Score S = F * P (Eq. 6-8) from the two latest
-// confidences; hist = number of observations available.
-__device__ float fps(float c1, float c2, int hist, float theta, float w,
-                     float v_ref, float tau) {
+// Rank key of a member of J_h from the two latest confidences (hist =
+// number of observations available).  REFLEX_SIGNAL_FPS is the
+// Frontier-Progress Score S = F * P (Eq. 6-8); the other keys are the
+// single-signal ablations: F, P, c^{t-1}, 1 - c^{t-1}.
+__device__ float rank_key(int signal, float c1, float c2, int hist, float theta, float w,
+                          float v_ref, float tau) {
+  if (signal == REFLEX_SIGNAL_CONFIDENCE) return c1;
+  if (signal == REFLEX_SIGNAL_UNCERTAINTY) return __fsub_rn(1.0f, c1);
   const float v = hist >= 2 ? __fsub_rn(c1, c2) : 0.0f;
   const float half_w = __fmul_rn(w, 0.5f);
   const float vbar = fminf(fmaxf(v, -half_w), half_w);
+  const float P =
+      hist >= 2 ? sigmoid_cw(__fdiv_rn(__fsub_rn(v_ref, vbar), tau)) : 1.0f;
+  if (signal == REFLEX_SIGNAL_PROGRESS) return P;
   const float chat = fminf(fmaxf(__fadd_rn(c1, vbar), 0.0f), 1.0f);
   const float x1 = __fdiv_rn(__fadd_rn(__fsub_rn(chat, theta), w), tau);
   const float x2 = __fdiv_rn(__fsub_rn(theta, chat), tau);
   const float F = __fmul_rn(sigmoid_cw(x1), sigmoid_cw(x2));
-  const float P =
-      hist >= 2 ? sigmoid_cw(__fdiv_rn(__fsub_rn(v_ref, vbar), tau)) : 1.0f;
+  if (signal == REFLEX_SIGNAL_FRONTIER) return F;
   return __fmul_rn(F, P);
+}
+
+// Role-shuffle key of the token at batch index pos: the high 32 bits of
+// splitmix64 output number pos + 1 for the seed (Steele, Lea and Flood 2014:
+// state advances by the golden gamma, output is Stafford's mix13 of it).
+__device__ __forceinline__ uint32_t shuffle_key(uint64_t seed, int pos) {
+  uint64_t z = seed + static_cast<uint64_t>(pos + 1) * 0x9e3779b97f4a7c15ull;
+  z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ull;
+  z = (z ^ (z >> 27)) * 0x94d049bb133111ebull;
+  z ^= z >> 31;
+  return static_cast<uint32_t>(z >> 32);
 }
 
 __device__ __forceinline__ int role_count(int dist, int k_base, int d_role) {
@@ -94,21 +114,38 @@ __global__ void __launch_bounds__(kThreads)
                   int32_t* __restrict__ k_out,
                   unsigned long long* __restrict__ k_sum,
                   uint32_t* __restrict__ err) {
-  __shared__ float s_score[kMaxJ];
-  __shared__ int32_t s_tok[kMaxJ];
+  // J_h scores and positions; the role shuffle reuses the same 32 KB as
+  // kMaxJ 64-bit sort words
+  __shared__ __align__(16) uint64_t s_raw[kMaxJ];
+  float* s_score = reinterpret_cast<float*>(s_raw);
+  int32_t* s_tok = reinterpret_cast<int32_t*>(s_raw) + kMaxJ;
   __shared__ int s_nj;
   __shared__ unsigned long long s_sum;
+  __shared__ uint32_t s_err;
+  grid_dep_wait();
+  grid_dep_launch();
+  // With one sequence (one CTA) the sum and the error word are stored
+  // outright at the end, so the caller needs no clearing; with several,
+  // the host clears them and each CTA adds its share.
+  const bool sole = gridDim.x == 1;
   const int s = blockIdx.x;
   const int lo = seq_off[s], hi = seq_off[s + 1];
-  if (lo < 0 || hi > T || lo > hi) {  // malformed offsets: touch nothing
-    if (threadIdx.x == 0) set_err(err, kErrIndex);
+  if (lo < 0 || hi > T || lo > hi) {  // malformed offsets: touch no count
+    if (threadIdx.x == 0) {
+      if (sole) {
+        if (err) *err = kErrIndex;
+        if (k_sum) *k_sum = 0ull;
+      } else {
+        set_err(err, kErrIndex);
+      }
+    }
     return;
   }
   int act = active_block[s];
   if (threadIdx.x == 0) {
     s_nj = 0;
     s_sum = 0ull;
-    if (act < 1) set_err(err, kErrActive);
+    s_err = act < 1 ? kErrActive : 0u;
   }
   __syncthreads();
   const int k_cur = a.k_base + a.delta_role;
@@ -123,8 +160,8 @@ __global__ void __launch_bounds__(kThreads)
       const int slot = atomicAdd(&s_nj, 1);
       if (slot < kMaxJ) {
         s_tok[slot] = i;
-        s_score[slot] = fps(conf1[i], conf2[i], hist_len[i], a.theta, a.w_cf,
-                            a.v_ref, a.tau);
+        s_score[slot] = rank_key(a.signal, conf1[i], conf2[i], hist_len[i], a.theta,
+                                 a.w_cf, a.v_ref, a.tau);
         continue;  // written in pass 2
       }
       k = k_cur;  // over capacity: keeps K_cur (error flagged below)
@@ -138,7 +175,7 @@ __global__ void __launch_bounds__(kThreads)
   const int nj = nj_all < kMaxJ ? nj_all : kMaxJ;
   if (nj_all > kMaxJ) {
     // too many to rank: every stored member keeps K_cur too
-    if (threadIdx.x == 0) set_err(err, kErrCapacity);
+    if (threadIdx.x == 0) atomicOr(&s_err, kErrCapacity);
     for (int m = threadIdx.x; m < nj; m += kThreads) {
       const int k = clip(k_cur, a.k_min, a.k_max);
       k_out[s_tok[m]] = k;
@@ -165,12 +202,67 @@ __global__ void __launch_bounds__(kThreads)
       my_sum += static_cast<unsigned long long>(k);
     }
   }
-  if (k_sum != nullptr) {
-    // warp sums, then one shared atomic per warp and one global per block
-    for (int o = 16; o > 0; o >>= 1) my_sum += __shfl_xor_sync(0xffffffffu, my_sum, o);
-    if ((threadIdx.x & 31) == 0) atomicAdd(&s_sum, my_sum);
-    __syncthreads();
-    if (threadIdx.x == 0) atomicAdd(k_sum, s_sum);
+  if (a.role_shuffle) {
+    // Role shuffle: token i takes the count of the sequence's r_i-th
+    // position, r_i the rank of (key_i, i); a permutation, so my_sum holds.
+    // The ranks come from a bitonic sort of the words key << 32 | offset.
+    const int len = hi - lo;
+    if (len > kMaxJ) {
+      if (threadIdx.x == 0) atomicOr(&s_err, kErrCapacity);
+    } else {
+      constexpr int kPer = kMaxJ / kThreads;
+      int n2 = 1;
+      while (n2 < len) n2 <<= 1;
+      __syncthreads();  // every count of the sequence written, s_raw free
+      for (int m = threadIdx.x; m < n2; m += kThreads)
+        s_raw[m] = m < len ? (static_cast<uint64_t>(shuffle_key(a.shuffle_seed, lo + m)) << 32) |
+                                 static_cast<uint32_t>(m)
+                           : ~0ull;  // padding sorts last
+      __syncthreads();
+      for (int size = 2; size <= n2; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+          for (int m = threadIdx.x; m < n2; m += kThreads) {
+            const int o = m ^ stride;
+            if (o > m) {
+              const uint64_t x = s_raw[m], y = s_raw[o];
+              const bool up = (m & size) == 0;
+              if ((x > y) == up) {
+                s_raw[m] = y;
+                s_raw[o] = x;
+              }
+            }
+          }
+          __syncthreads();
+        }
+      }
+      int take[kPer], dest[kPer];
+#pragma unroll
+      for (int u = 0; u < kPer; ++u) {
+        const int r = threadIdx.x + u * kThreads;
+        dest[u] = -1;
+        if (r < len) {
+          take[u] = k_out[lo + r];  // count of place r goes to the r-th smallest key
+          dest[u] = lo + static_cast<int>(s_raw[r] & 0xffffffffu);
+        }
+      }
+      __syncthreads();  // all old counts read before any is replaced
+#pragma unroll
+      for (int u = 0; u < kPer; ++u)
+        if (dest[u] >= 0) k_out[dest[u]] = take[u];
+    }
+  }
+  // warp sums, then one shared atomic per warp; one store or atomic per CTA
+  for (int o = 16; o > 0; o >>= 1) my_sum += __shfl_xor_sync(0xffffffffu, my_sum, o);
+  if ((threadIdx.x & 31) == 0) atomicAdd(&s_sum, my_sum);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (sole) {
+      if (err) *err = s_err;
+      if (k_sum) *k_sum = s_sum;
+    } else {
+      if (err && s_err) atomicOr(err, s_err);
+      if (k_sum) atomicAdd(k_sum, s_sum);
+    }
   }
 }
 
@@ -198,6 +290,10 @@ cudaError_t launch_budget(const float* conf1, const float* conf2,
                           unsigned long long* k_sum, uint32_t* err,
                           cudaStream_t stream) {
   if (B <= 0) return cudaSuccess;
+  if (B == 1)  // nothing to clear first: programmatic launch after the previous kernel
+    return launch_pdl(budget_kernel, dim3(1), dim3(kThreads), 0, stream, conf1, conf2,
+                      hist_len, masked, block_id, seq_off, active_block, T, a, k_out,
+                      k_sum, err);
   budget_kernel<<<B, kThreads, 0, stream>>>(conf1, conf2, hist_len, masked,
                                             block_id, seq_off, active_block, T, a,
                                             k_out, k_sum, err);

@@ -12,6 +12,9 @@ namespace rx {
 struct AllocArgs {
   int k_min, k_base, k_max, delta_role, delta_cur;
   float q, theta, w_cf, v_ref, tau;
+  int signal;             // rank key of the Eq. 9 groups (REFLEX_SIGNAL_*)
+  int role_shuffle;       // permute each sequence's final counts
+  uint64_t shuffle_seed;  // splitmix64 seed of the permutation keys
 };
 
 // ---- allocation (budget.cu) -----------------------------------------------
@@ -27,9 +30,12 @@ cudaError_t launch_wait_selftest(uint32_t* err, uint64_t limit_ns,
 
 // ---- routing (router.cu) --------------------------------------------------
 // z[T, E] = router scores (sequential fp32 fma chain over the hidden index).
+// The first CTA also clears zero_words[0, n_zero) (nullable): the call's
+// header or error word, so no memset precedes the first kernel.
 cudaError_t launch_router_logits(int dtype, const void* hidden,
                                  const void* w_router, int T, int d, int E,
-                                 float* z, int num_sms, cudaStream_t stream);
+                                 float* z, uint32_t* zero_words, int n_zero,
+                                 int num_sms, cudaStream_t stream);
 // ids/alpha [T, k_max] from z and the counts k.
 cudaError_t launch_router_select(const float* z, const int32_t* k, int T,
                                  int E, int k_max, bool renorm, int32_t* ids,

@@ -132,7 +132,7 @@ int map_err_bits(uint32_t bits) {
 
 extern "C" {
 
-int reflex_abi_version(void) { return 100; }
+int reflex_abi_version(void) { return 110; }
 
 const char* reflex_status_string(int s) {
   switch (s) {
@@ -160,6 +160,9 @@ void reflex_default_params(reflex_alloc_params* p) {
   p->w_cf = 0.30f;
   p->v_ref = 0.01f;
   p->tau = 0.05f;
+  p->signal = REFLEX_SIGNAL_FPS;
+  p->role_shuffle = 0;
+  p->shuffle_seed = 0;
 }
 
 int reflex_allocate(const float* router_scores, const float* conf_prev1,
@@ -182,12 +185,18 @@ int reflex_allocate(const float* router_scores, const float* conf_prev1,
     return REFLEX_EINVAL;
   if (!(p->q > 0.0f && p->q <= 0.5f) || !(p->w_cf > 0.0f) || !(p->tau > 0.0f))
     return REFLEX_EINVAL;
+  if (p->signal < REFLEX_SIGNAL_FPS || p->signal > REFLEX_SIGNAL_UNCERTAINTY ||
+      (p->role_shuffle != 0 && p->role_shuffle != 1))
+    return REFLEX_EINVAL;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint32_t* err = reinterpret_cast<uint32_t*>(dev_status);
-  if (err) RX_CUDA(cudaMemsetAsync(err, 0, sizeof(int32_t), s));
-  if (k_sum_out) RX_CUDA(cudaMemsetAsync(k_sum_out, 0, sizeof(int64_t), s));
+  if (B > 1) {  // a single-sequence call stores both from its one CTA
+    if (err) RX_CUDA(cudaMemsetAsync(err, 0, sizeof(int32_t), s));
+    if (k_sum_out) RX_CUDA(cudaMemsetAsync(k_sum_out, 0, sizeof(int64_t), s));
+  }
   rx::AllocArgs a{p->k_min, p->k_base,  p->k_max, p->delta_role, p->delta_cur,
-                  p->q,     p->theta,   p->w_cf,  p->v_ref,      p->tau};
+                  p->q,     p->theta,   p->w_cf,  p->v_ref,      p->tau,
+                  p->signal, p->role_shuffle, p->shuffle_seed};
   RX_CUDA(rx::launch_budget(conf_prev1, conf_prev2, hist_len, masked, block_id,
                             seq_offsets, active_block, T, B, a, k_out,
                             reinterpret_cast<unsigned long long*>(k_sum_out),
@@ -270,8 +279,11 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
   void* ysh = shared_inter ? ws + L.ysh : nullptr;
 
   if (stages & REFLEX_STAGE_ROUTE) {
-    RX_CUDA(cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s));
-    RX_CUDA(rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z, sms, s));
+    // the router's first CTA clears the header (error word, totals): no
+    // kernel before the router reads it
+    RX_CUDA(rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z,
+                                     reinterpret_cast<uint32_t*>(hdr),
+                                     static_cast<int>(sizeof(WsHeader) / 4), sms, s));
     RX_CUDA(rx::launch_router_select(z, k, T, E, k_max,
                                      (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
                                      I32(L.ids), alpha, err, s));

@@ -76,9 +76,9 @@ extern "C" int reflex_route_noalloc(int32_t dtype, const void* hidden,
   if (!device_setup(&z, &sms)) return REFLEX_ECUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint32_t* err = reinterpret_cast<uint32_t*>(dev_status);
-  if (err != nullptr && cudaMemsetAsync(err, 0, sizeof(int32_t), s) != cudaSuccess)
-    return REFLEX_ECUDA;
-  if (rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z, sms, s) != cudaSuccess)
+  // the router clears the error word before select may set bits in it
+  if (rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z, err, err ? 1 : 0, sms,
+                               s) != cudaSuccess)
     return REFLEX_ECUDA;
   if (rx::launch_router_select(z, k, T, E, k_max, (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
                                ids_out, alpha_out, err, s) != cudaSuccess)

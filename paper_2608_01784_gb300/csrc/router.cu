@@ -83,12 +83,14 @@ struct LogitsCfg {
 template <typename Tin, int TM, int TN, int WT, int WE>
 __global__ void __launch_bounds__(LogitsCfg<Tin, TM, TN, WT, WE>::kThreads)
     logits_kernel(const Tin* __restrict__ h, const Tin* __restrict__ w, int T,
-                  int d, int E, float* __restrict__ z) {
+                  int d, int E, float* __restrict__ z, uint32_t* __restrict__ zw, int nz) {
   using C = LogitsCfg<Tin, TM, TN, WT, WE>;
   constexpr int BT = C::BT, BE = C::BE, R = C::kRows, NT = C::kThreads;
   extern __shared__ __align__(16) uint8_t smem_l[];
   grid_dep_wait();
   grid_dep_launch();
+  if (zw != nullptr && blockIdx.x == 0 && blockIdx.y == 0)
+    for (int i = threadIdx.x; i < nz; i += blockDim.x) zw[i] = 0u;
   float* cbuf = reinterpret_cast<float*>(smem_l + kStagesL * C::kRawStage);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ty = lane >> 2, tx = lane & 3;
@@ -180,7 +182,7 @@ __global__ void __launch_bounds__(LogitsCfg<Tin, TM, TN, WT, WE>::kThreads)
 
 template <typename Tin, int TM, int TN, int WT, int WE>
 cudaError_t launch_logits_tile(const Tin* h, const Tin* w, int T, int d, int E,
-                               float* z, cudaStream_t s) {
+                               float* z, uint32_t* zw, int nz, cudaStream_t s) {
   using C = LogitsCfg<Tin, TM, TN, WT, WE>;
   auto kern = logits_kernel<Tin, TM, TN, WT, WE>;
   if (C::kSmem > 48 * 1024) {
@@ -189,8 +191,7 @@ cudaError_t launch_logits_tile(const Tin* h, const Tin* w, int T, int d, int E,
     if (e != cudaSuccess) return e;
   }
   const dim3 g((T + C::BT - 1) / C::BT, (E + C::BE - 1) / C::BE);
-  kern<<<g, C::kThreads, C::kSmem, s>>>(h, w, T, d, E, z);
-  return cudaGetLastError();
+  return launch_pdl(kern, g, dim3(C::kThreads), C::kSmem, s, h, w, T, d, E, z, zw, nz);
 }
 
 __device__ __forceinline__ uint32_t order_bits(float v) {
@@ -303,7 +304,8 @@ __device__ __forceinline__ void row8(const uint8_t* p, float* f) {
 template <typename Tin, int TM>
 __global__ void __launch_bounds__(kThreadsS)
     logits_short_kernel(const Tin* __restrict__ h, const Tin* __restrict__ w,
-                        int T, int d, int E, float* __restrict__ z) {
+                        int T, int d, int E, float* __restrict__ z,
+                        uint32_t* __restrict__ zw, int nz) {
   constexpr int BT = 8 * TM, BE = 64;
   constexpr int kRowBytes = kKc * static_cast<int>(sizeof(Tin)) + 16;
   constexpr int kVecs = kKc * static_cast<int>(sizeof(Tin)) / 16;
@@ -313,6 +315,8 @@ __global__ void __launch_bounds__(kThreadsS)
   extern __shared__ __align__(16) uint8_t smem_s[];
   grid_dep_wait();
   grid_dep_launch();
+  if (zw != nullptr && blockIdx.x == 0 && blockIdx.y == 0)
+    for (int i = threadIdx.x; i < nz; i += blockDim.x) zw[i] = 0u;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ty = lane >> 2, tx = lane & 3;
   const int t0 = blockIdx.x * BT;
@@ -384,7 +388,7 @@ __global__ void __launch_bounds__(kThreadsS)
 
 template <typename Tin, int TM>
 cudaError_t launch_logits_short(const Tin* h, const Tin* w, int T, int d, int E,
-                                float* z, cudaStream_t s) {
+                                float* z, uint32_t* zw, int nz, cudaStream_t s) {
   constexpr int kRowBytes = kKc * static_cast<int>(sizeof(Tin)) + 16;
   constexpr int smem = kStagesS * (8 * TM + 64) * kRowBytes;
   auto kern = logits_short_kernel<Tin, TM>;
@@ -394,8 +398,7 @@ cudaError_t launch_logits_short(const Tin* h, const Tin* w, int T, int d, int E,
     if (e != cudaSuccess) return e;
   }
   const dim3 g((T + 8 * TM - 1) / (8 * TM), (E + 63) / 64);
-  kern<<<g, kThreadsS, smem, s>>>(h, w, T, d, E, z);
-  return cudaGetLastError();
+  return launch_pdl(kern, g, dim3(kThreadsS), smem, s, h, w, T, d, E, z, zw, nz);
 }
 
 // ---- bf16 scores with mixed-precision fma ----------------------------------
@@ -445,7 +448,7 @@ template <int LY, int TM, int TN, int WT, int WE, int S, int KC>
 __global__ void __launch_bounds__(MxCfg<LY, TM, TN, WT, WE, S, KC>::NT)
     logits_mx_kernel(const __nv_bfloat16* __restrict__ h,
                      const __nv_bfloat16* __restrict__ w, int T, int d, int E,
-                     float* __restrict__ z) {
+                     float* __restrict__ z, uint32_t* __restrict__ zw, int nz) {
   using C = MxCfg<LY, TM, TN, WT, WE, S, KC>;
   constexpr int LX = C::LX, BT = C::BT, BE = C::BE, NT = C::NT;
   constexpr int kRB = C::kRowBytes;
@@ -453,6 +456,8 @@ __global__ void __launch_bounds__(MxCfg<LY, TM, TN, WT, WE, S, KC>::NT)
   extern __shared__ __align__(16) uint8_t smem_m[];
   grid_dep_wait();
   grid_dep_launch();
+  if (zw != nullptr && blockIdx.x == 0 && blockIdx.y == 0)
+    for (int i = threadIdx.x; i < nz; i += blockDim.x) zw[i] = 0u;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ty = lane / LX, tx = lane % LX;
   const int wt = warp / WE, we = warp % WE;
@@ -542,7 +547,7 @@ __global__ void __launch_bounds__(MxCfg<LY, TM, TN, WT, WE, S, KC>::NT)
 
 template <int LY, int TM, int TN, int WT, int WE, int S, int KC = 32>
 cudaError_t launch_logits_mx(const __nv_bfloat16* h, const __nv_bfloat16* w, int T,
-                             int d, int E, float* z, cudaStream_t s) {
+                             int d, int E, float* z, uint32_t* zw, int nz, cudaStream_t s) {
   using C = MxCfg<LY, TM, TN, WT, WE, S, KC>;
   auto kern = logits_mx_kernel<LY, TM, TN, WT, WE, S, KC>;
   if (C::kSmem > 48 * 1024) {
@@ -551,24 +556,23 @@ cudaError_t launch_logits_mx(const __nv_bfloat16* h, const __nv_bfloat16* w, int
     if (e != cudaSuccess) return e;
   }
   const dim3 g((T + C::BT - 1) / C::BT, (E + C::BE - 1) / C::BE);
-  kern<<<g, C::NT, C::kSmem, s>>>(h, w, T, d, E, z);
-  return cudaGetLastError();
+  return launch_pdl(kern, g, dim3(C::NT), C::kSmem, s, h, w, T, d, E, z, zw, nz);
 }
 
 // fp32 inputs: the widened-buffer tiles when they fill most SMs without
 // overhanging the expert count; otherwise the short-batch kernel with the
 // largest token tile that still fills most SMs.
 cudaError_t logits_dispatch(const float* h, const float* w, int T, int d, int E,
-                            float* z, int num_sms, cudaStream_t s) {
+                            float* z, uint32_t* zw, int nz, int num_sms, cudaStream_t s) {
   auto grid_for = [&](int bt, int be) {
     return static_cast<int64_t>((T + bt - 1) / bt) * ((E + be - 1) / be);
   };
   const int64_t want = (num_sms * 4) / 5;
   if (E >= 128 && grid_for(64, 128) >= want)  // TM 4, TN 8, 2 x 4 warps
-    return launch_logits_tile<float, 4, 8, 2, 4>(h, w, T, d, E, z, s);
-  if (grid_for(32, 64) >= want) return launch_logits_short<float, 4>(h, w, T, d, E, z, s);
-  if (grid_for(16, 64) >= want) return launch_logits_short<float, 2>(h, w, T, d, E, z, s);
-  return launch_logits_short<float, 1>(h, w, T, d, E, z, s);
+    return launch_logits_tile<float, 4, 8, 2, 4>(h, w, T, d, E, z, zw, nz, s);
+  if (grid_for(32, 64) >= want) return launch_logits_short<float, 4>(h, w, T, d, E, z, zw, nz, s);
+  if (grid_for(16, 64) >= want) return launch_logits_short<float, 2>(h, w, T, d, E, z, zw, nz, s);
+  return launch_logits_short<float, 1>(h, w, T, d, E, z, zw, nz, s);
 }
 
 // bf16 inputs: mixed-precision fma tiles, chosen by the number of chains
@@ -576,29 +580,31 @@ cudaError_t logits_dispatch(const float* h, const float* w, int T, int d, int E,
 // Few chains: small thread tiles so every SM gets warps; many chains: 4 x 8
 // or 4 x 4 thread tiles, which need fewer operand reads per fma.
 cudaError_t logits_dispatch(const __nv_bfloat16* h, const __nv_bfloat16* w, int T,
-                            int d, int E, float* z, int num_sms, cudaStream_t s) {
+                            int d, int E, float* z, uint32_t* zw, int nz, int num_sms,
+                            cudaStream_t s) {
   const int64_t per_sm = static_cast<int64_t>(T) * E / (num_sms > 0 ? num_sms : 1);
-  if (per_sm <= 216) return launch_logits_mx<4, 1, 1, 4, 1, 8>(h, w, T, d, E, z, s);
-  if (per_sm <= 1080) return launch_logits_mx<4, 1, 2, 4, 1, 8>(h, w, T, d, E, z, s);
-  if (per_sm <= 4300) return launch_logits_mx<4, 2, 2, 2, 2, 4, 64>(h, w, T, d, E, z, s);
-  if (per_sm <= 10000) return launch_logits_mx<8, 4, 8, 2, 2, 3, 64>(h, w, T, d, E, z, s);
-  if (per_sm <= 20000) return launch_logits_mx<8, 4, 4, 2, 2, 3, 64>(h, w, T, d, E, z, s);
-  return launch_logits_mx<8, 4, 8, 2, 2, 4>(h, w, T, d, E, z, s);
+  if (per_sm <= 216) return launch_logits_mx<4, 1, 1, 4, 1, 8>(h, w, T, d, E, z, zw, nz, s);
+  if (per_sm <= 1080) return launch_logits_mx<4, 1, 2, 4, 1, 8>(h, w, T, d, E, z, zw, nz, s);
+  if (per_sm <= 4300) return launch_logits_mx<4, 2, 2, 2, 2, 4, 64>(h, w, T, d, E, z, zw, nz, s);
+  if (per_sm <= 10000) return launch_logits_mx<8, 4, 8, 2, 2, 3, 64>(h, w, T, d, E, z, zw, nz, s);
+  if (per_sm <= 20000) return launch_logits_mx<8, 4, 4, 2, 2, 3, 64>(h, w, T, d, E, z, zw, nz, s);
+  return launch_logits_mx<8, 4, 8, 2, 2, 4>(h, w, T, d, E, z, zw, nz, s);
 }
 
 }  // namespace
 
 cudaError_t launch_router_logits(int dtype, const void* hidden,
                                  const void* w_router, int T, int d, int E,
-                                 float* z, int num_sms, cudaStream_t stream) {
+                                 float* z, uint32_t* zero_words, int n_zero,
+                                 int num_sms, cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
   if (dtype == 0)
     return logits_dispatch(static_cast<const float*>(hidden),
                            static_cast<const float*>(w_router), T, d, E, z,
-                           num_sms, stream);
+                           zero_words, n_zero, num_sms, stream);
   return logits_dispatch(static_cast<const __nv_bfloat16*>(hidden),
                          static_cast<const __nv_bfloat16*>(w_router), T, d, E,
-                         z, num_sms, stream);
+                         z, zero_words, n_zero, num_sms, stream);
 }
 
 cudaError_t launch_router_select(const float* z, const int32_t* k, int T,

@@ -39,7 +39,8 @@ def oracle_allocate(state: dict, p: B.reflex_alloc_params):
                            k_min=p.k_min, k_base=p.k_base, k_max=p.k_max,
                            delta_role=p.delta_role, delta_cur=p.delta_cur,
                            q=p.q, theta=p.theta, w_cf=p.w_cf, v_ref=p.v_ref,
-                           tau=p.tau)
+                           tau=p.tau, signal=p.signal, role_shuffle=p.role_shuffle,
+                           shuffle_seed=p.shuffle_seed)
 
 
 def to_f32(x: torch.Tensor) -> np.ndarray:

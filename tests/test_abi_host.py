@@ -48,7 +48,7 @@ def test_status_strings_and_version(lib):
     assert B.reflex_status_string(B.REFLEX_OK) == "ok"
     assert "workspace" in B.reflex_status_string(B.REFLEX_EWORKSPACE)
     assert B.reflex_status_string(999) == "unknown status"
-    assert B.reflex_abi_version() >= 100
+    assert B.reflex_abi_version() >= 110
 
 
 def test_default_params_are_the_paper_settings(lib):
@@ -58,6 +58,10 @@ def test_default_params_are_the_paper_settings(lib):
     assert p.q == pytest.approx(0.25) and p.theta == pytest.approx(0.9)
     assert p.v_ref == pytest.approx(0.01) and p.tau == pytest.approx(0.05)
     assert p.w_cf == pytest.approx(0.30)
+    # the ablation fields sit where the C struct has them (a layout mismatch
+    # would show up as garbage here): FPS, no shuffle
+    assert (p.signal, p.role_shuffle, p.shuffle_seed) == (B.REFLEX_SIGNAL_FPS, 0, 0)
+    assert ctypes.sizeof(B.reflex_alloc_params) == 56
 
 
 def test_workspace_size(lib):
@@ -86,6 +90,10 @@ def test_host_rejections_enqueue_nothing(lib):
     bad = B.make_params(k_min=5, k_max=4)
     assert lib.reflex_allocate(None, 1, 1, 1, 1, 1, 1, 1, 4, 1, 8,
                                ctypes.byref(bad), 1, None, None, None) == B.REFLEX_EINVAL
+    for bad in (B.make_params(signal=5), B.make_params(signal=-1),
+                B.make_params(role_shuffle=2)):
+        assert lib.reflex_allocate(None, 1, 1, 1, 1, 1, 1, 1, 4, 1, 8,
+                                   ctypes.byref(bad), 1, None, None, None) == B.REFLEX_EINVAL
     assert lib.reflex_allocate(None, 1, 1, 1, 1, 1, 1, 1, 4, 0, 8,
                                ctypes.byref(p), 1, None, None, None) == B.REFLEX_EINVAL
     # forward: bad shapes, missing workspace

@@ -53,6 +53,13 @@ ALLOC_VARIANTS = {
     "fger_only": dict(delta_role=0),
     "wide_clip": dict(k_max=14),
     "tight_tau": dict(tau=0.01),
+    # App. C ablations: rank keys of the Eq. 9 groups, Role-Shuffled RRB
+    "frontier_only": dict(signal=B.REFLEX_SIGNAL_FRONTIER),
+    "progress_only": dict(signal=B.REFLEX_SIGNAL_PROGRESS),
+    "confidence_only": dict(signal=B.REFLEX_SIGNAL_CONFIDENCE),
+    "uncertainty_only": dict(signal=B.REFLEX_SIGNAL_UNCERTAINTY),
+    "role_shuffled_rrb": dict(delta_cur=0, role_shuffle=1, shuffle_seed=12345),
+    "reflex_shuffled": dict(role_shuffle=1, shuffle_seed=2**63 + 7),
 }
 
 
@@ -69,6 +76,20 @@ def test_allocate_bit_exact(name, hist, variant):
         assert status == B.REFLEX_OK
         assert np.array_equal(k_gpu, k_ref)
         assert ksum == int(k_ref.sum())
+
+
+def test_allocate_role_shuffle_long_sequence_flags_capacity():
+    # one 8192-token sequence: longer than the shuffle's 4096-token limit, so
+    # the counts stay unshuffled and REFLEX_ECAPACITY is reported
+    cfg = CFG["llada2_mini"]
+    state = W.make_state(cfg, 3)
+    state["seq_offsets"] = np.array([0, state["block_id"].size], np.int32)
+    state["active_block"] = state["active_block"][:1].copy()
+    p = G.params_of(cfg, delta_cur=0, role_shuffle=1, shuffle_seed=9)
+    k_gpu, ksum, status = G.gpu_allocate(state, p)
+    assert status == B.REFLEX_ECAPACITY
+    k_ref = G.oracle_allocate(state, G.params_of(cfg, delta_cur=0))
+    assert np.array_equal(k_gpu, k_ref) and ksum == int(k_ref.sum())
 
 
 def test_allocate_mixed_history_and_ties():

@@ -307,6 +307,163 @@ def test_role_shuffle_preserves_pairs():
 
 
 # --------------------------------------------------------------------------
+# App. C ablations: rank keys of the Eq. 9 groups and Role-Shuffled RRB
+# --------------------------------------------------------------------------
+def _grid(x):
+    """Values on a 2^-8 grid, so c1 - c2 and c1 + vbar are exact in fp32."""
+    return np.round(np.asarray(x, np.float64) * 256) / 256
+
+
+def _expected_groups(order, nj, q=0.25, k_cur=12, dc=2):
+    """Counts of J_h members listed in rank order (first = highest key)."""
+    n = math.floor(q * nj)
+    k = np.full(nj, k_cur)
+    k[order[:n]] += dc
+    if n:
+        k[order[nj - n:]] -= dc
+    return k
+
+
+def _active_case(c1, c2, hist):
+    nj = len(c1)
+    bid = [0, 0] + [1] * nj
+    msk = [0, 0] + [1] * nj
+    c1 = np.concatenate([[0.5, 0.5], c1]).astype(np.float32)
+    c2 = np.concatenate([[0.5, 0.5], c2]).astype(np.float32)
+    hist = np.concatenate([[2, 2], hist]).astype(np.uint8)
+    return bid, msk, c1, c2, hist
+
+
+def test_signal_frontier_orders_by_distance_to_gate_midpoint():
+    # F(c) = sig((c - theta + w) / tau) * sig((theta - c) / tau) is symmetric
+    # about c = theta - w/2 and falls with the distance from it (the two
+    # arguments sum to w / tau), so "F only" ranks J_h by |chat - (theta - w/2)|.
+    w = 0.30
+    chat = _grid([0.75, 0.70, 0.82, 0.60, 0.95, 0.40, 0.78, 0.30])
+    v = _grid([0.10, -0.12, 0.0, 0.05, -0.05, 0.14, -0.02, 0.08])  # |v| < w/2
+    c1 = chat - v
+    c2 = c1 - v
+    bid, msk, C1, C2, H = _active_case(c1, c2, np.full(8, 2))
+    k, key = _alloc(bid, 1, msk, C1, C2, hist=H, signal=1, w_cf=w)
+    order = np.argsort(np.abs(chat - (0.9 - w / 2)), kind="stable")
+    assert k[2:].tolist() == _expected_groups(order, 8).tolist()
+    # the same tokens under FPS rank differently (the progress factor matters)
+    k_fps, _ = _alloc(bid, 1, msk, C1, C2, hist=H, signal=0, w_cf=w)
+    assert k_fps[2:].tolist() != k[2:].tolist()
+
+
+def test_signal_progress_orders_single_observation_then_slowest():
+    # P = sig((v_ref - vbar) / tau) falls with vbar; one observation gives 1,
+    # above any value of sig at the clipped velocities (vbar >= -w/2).
+    v = _grid([0.10, -0.12, 0.0, 0.05, -0.05, 0.14, -0.02, 0.08])
+    hist = np.array([2, 2, 1, 2, 2, 2, 1, 2])
+    c1 = _grid([0.6, 0.3, 0.9, 0.5, 0.7, 0.4, 0.2, 0.8])
+    c2 = c1 - v
+    bid, msk, C1, C2, H = _active_case(c1, c2, hist)
+    k, _ = _alloc(bid, 1, msk, C1, C2, hist=H, signal=2)
+    keyv = np.where(hist >= 2, v, -1.0)   # single observation first
+    order = np.lexsort((np.arange(8), keyv))
+    assert k[2:].tolist() == _expected_groups(order, 8).tolist()
+
+
+@pytest.mark.parametrize("signal,sign", [(3, -1), (4, 1)])
+def test_signal_confidence_and_uncertainty_are_plain_sorts(signal, sign):
+    c1 = _grid([0.6, 0.3, 0.9, 0.5, 0.7, 0.4, 0.2, 0.8, 0.55, 0.35, 0.65, 0.45])
+    c2 = _grid(np.clip(c1 - 0.1, 0, 1))
+    bid, msk, C1, C2, H = _active_case(c1, c2, np.full(12, 2))
+    k, _ = _alloc(bid, 1, msk, C1, C2, hist=H, signal=signal)
+    order = np.argsort(sign * c1, kind="stable")   # confidence: high first
+    assert k[2:].tolist() == _expected_groups(order, 12).tolist()
+
+
+def test_signal_ties_keep_lower_position_first():
+    c1 = _grid([0.7] * 8)
+    bid, msk, C1, C2, H = _active_case(c1, c1, np.full(8, 2))
+    for signal in range(5):
+        k, _ = _alloc(bid, 1, msk, C1, C2, hist=H, signal=signal)
+        assert k[2:].tolist() == [14, 14, 12, 12, 12, 12, 10, 10]
+
+
+@pytest.mark.parametrize("seed", range(5))
+def test_role_shuffle_keeps_each_sequence_multiset(seed):
+    rng = np.random.default_rng(300 + seed)
+    bid, act, msk, c1, c2, h, so = _random_case(rng, hist=None)
+    for kw in (dict(delta_cur=0), dict()):   # Role-Shuffled RRB, and REFLEX
+        k0, _ = _alloc(bid, act, msk, c1, c2, hist=h, seq_offsets=so, **kw)
+        k1, _ = _alloc(bid, act, msk, c1, c2, hist=h, seq_offsets=so,
+                       role_shuffle=1, shuffle_seed=seed, **kw)
+        for s in range(len(act)):
+            a, b = so[s], so[s + 1]
+            assert sorted(k0[a:b].tolist()) == sorted(k1[a:b].tolist())
+        assert not np.array_equal(k0, k1)
+        k2, _ = _alloc(bid, act, msk, c1, c2, hist=h, seq_offsets=so,
+                       role_shuffle=1, shuffle_seed=seed, **kw)
+        assert np.array_equal(k1, k2)              # deterministic per seed
+
+
+def test_role_shuffle_uniform_fixed_counts_untouched():
+    # a uniform allocation is a fixed point of any permutation
+    rng = np.random.default_rng(9)
+    bid, act, msk, c1, c2, h, so = _random_case(rng)
+    k, _ = _alloc(bid, act, msk, c1, c2, seq_offsets=so, delta_role=0,
+                  delta_cur=0, role_shuffle=1, shuffle_seed=77)
+    assert np.all(k == 8)
+
+
+def test_role_shuffle_is_uniform_over_seeds():
+    # 6 positions (prompt, blocks 1..5 with block 3 active: role counts 4, 8,
+    # 12, 12, 12, 8 by Eq. 5): every position receives count v with frequency
+    # (multiplicity of v) / 6 over seeds; chi-square with 6 x (values - 1)
+    # degrees of freedom.
+    bid = [0, 1, 2, 3, 4, 5]
+    act, msk = 3, [0] * 6
+    c1 = np.full(6, 0.5, np.float32)
+    base, _ = _alloc(bid, act, msk, c1, delta_cur=0)
+    vals, mult = np.unique(base, return_counts=True)
+    n_seeds = 3000
+    hits = np.zeros((6, len(vals)))
+    for seed in range(n_seeds):
+        k, _ = _alloc(bid, act, msk, c1, delta_cur=0, role_shuffle=1, shuffle_seed=seed)
+        for pos in range(6):
+            hits[pos, np.searchsorted(vals, k[pos])] += 1
+    expect = n_seeds * mult[None, :] / 6.0
+    chi2 = float(((hits - expect) ** 2 / expect).sum())
+    dof = 6 * (len(vals) - 1)
+    assert chi2 < dof + 6 * math.sqrt(2 * dof)     # far inside the upper tail
+
+
+def test_role_shuffle_follows_key_order():
+    # definition check of the assignment: token i takes the count of place
+    # rank(key_i, i) in the sequence (keys from the generator, numpy sort)
+    rng = np.random.default_rng(21)
+    bid, act, msk, c1, c2, h, so = _random_case(rng, n_seq=2)
+    k0, _ = _alloc(bid, act, msk, c1, c2, seq_offsets=so, delta_cur=0)
+    seed = 123456789
+    k1, _ = _alloc(bid, act, msk, c1, c2, seq_offsets=so, delta_cur=0,
+                   role_shuffle=1, shuffle_seed=seed)
+    for s in range(len(act)):
+        a, b = int(so[s]), int(so[s + 1])
+        keys = np.array([oracle.splitmix64(seed, i + 1) >> 32 for i in range(a, b)],
+                        np.uint64)
+        ranks = np.empty(b - a, np.int64)
+        ranks[np.lexsort((np.arange(b - a), keys))] = np.arange(b - a)
+        assert k1[a:b].tolist() == k0[a:b][ranks].tolist()
+
+
+def test_splitmix64_bits_are_uniform_and_mix():
+    out = np.array([oracle.splitmix64(42, n) for n in range(1, 1 << 15)], np.uint64)
+    top = (out >> np.uint64(56)).astype(np.int64)
+    hist = np.bincount(top, minlength=256)
+    e = out.size / 256
+    chi2 = float(((hist - e) ** 2 / e).sum())
+    assert chi2 < 255 + 6 * math.sqrt(2 * 255)
+    # neighbouring counters differ in about half of the 64 bits
+    diff = [bin(int(a) ^ int(b)).count("1") for a, b in zip(out[:-1], out[1:])]
+    assert 30 < float(np.mean(diff)) < 34
+    assert len(set(out.tolist())) == out.size
+
+
+# --------------------------------------------------------------------------
 # Router scores: exact integer cases, summation order, fma, error bound
 # --------------------------------------------------------------------------
 def test_router_logits_exact_integers():
