@@ -64,6 +64,8 @@ def parse():
     ap.add_argument("--sweep", action="store_true",
                     help="token-count x count-skew sweep on the LLaDA2.0-mini "
                          "layer (one JSON line per point)")
+    ap.add_argument("--trajectory", action="store_true",
+                    help="whole denoising trajectories: NFE and pairs per sample")
     ap.add_argument("--ablation", action="store_true",
                     help="REFLEX and its App. C allocation ablations on one layer")
     ap.add_argument("--seed", type=int, default=0)
@@ -707,6 +709,55 @@ def run_ablation(args, rank, world, local_rank):
         print(json.dumps(line), flush=True)
 
 
+def run_trajectory(args, rank, world, local_rank):
+    """Whole denoising trajectories (allocation -> MoE layer -> state update per
+    forward, from the all-mask start until every block is resolved) with the
+    synthetic confidence model; one JSON line per workload and allocation:
+    NFE, pairs per sample, AvgK and wall time."""
+    import torch
+    from paper_2608_01784_gb300 import _binding as B
+    from paper_2608_01784_gb300 import api, build
+    from paper_2608_01784_gb300 import trajectory as TR
+
+    build.build()
+    B.load()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    stream = torch.cuda.current_stream(dev)
+    for name in ("llada_moe", "llada2_mini"):
+        cfg = W.CONFIGS[name]
+        dl = api.layer_to_device(W.make_layer(cfg, args.seed), cfg.dtype, dev)
+        moe = api.MoELayer(dl, dtype=cfg.dtype, d=cfg.d, E=cfg.E, inter=cfg.inter,
+                           shared_inter=cfg.shared_inter, k_max=cfg.k_max,
+                           max_tokens=cfg.T, device=dev)
+        st0 = TR.initial_state(W.make_state(cfg, args.seed))
+        for alloc, over in (("reflex", {}), ("fixed_topk", dict(delta_role=0, delta_cur=0))):
+            p = B.make_params(**cfg.alloc_params(**over))
+            TR.simulate(api.state_to_device(st0, dev), p, cfg.E, seed=args.seed, moe=moe,
+                        hidden=dl["hidden"], check_every=4, graph=True)  # warm-up run
+            ds = api.state_to_device(st0, dev)
+            torch.cuda.synchronize(dev)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            r = TR.simulate(ds, p, cfg.E, seed=args.seed, moe=moe, hidden=dl["hidden"],
+                            check_every=4, graph=True)
+            b.record(stream)
+            torch.cuda.synchronize(dev)
+            ms = a.elapsed_time(b)
+            assert r["alloc_status"] == B.REFLEX_OK and r["update_status"] == B.REFLEX_OK
+            lens = np.diff(st0["seq_offsets"])
+            line = dict(trajectory=name, allocation=alloc, sequences=int(lens.size),
+                        nfe_mean=float(r["nfe"].mean()), nfe_max=int(r["nfe"].max()),
+                        forwards_run=r["forwards"],
+                        pairs_per_sample=float(r["pairs"].mean()),
+                        avg_k=float(r["pairs"].sum() / (r["nfe"] * lens).sum()),
+                        ms_total=ms, ms_per_forward=ms / max(1, r["forwards"]),
+                        samples_per_s=lens.size / (ms * 1e-3),
+                        note="synthetic confidences; 1 MoE layer per forward; one "
+                             "forward per CUDA-graph replay")
+            print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     cfg = W.CONFIGS.get(args.config, W.CONFIGS["llada_moe_b32"])
@@ -723,6 +774,9 @@ def main():
         elif args.ablation:
             if rank == 0:
                 run_ablation(args, rank, world, local_rank)
+        elif args.trajectory:
+            if rank == 0:
+                run_trajectory(args, rank, world, local_rank)
         elif args.config == "llada_moe_stack16":
             run_stack(args, rank, world, local_rank)
         else:

@@ -164,6 +164,42 @@ int reflex_allocate(const float* router_scores, const float* conf_prev1,
                     const reflex_alloc_params* p, int32_t* k_out,
                     int64_t* k_sum_out, int32_t* dev_status, void* stream);
 
+/*
+ * reflex_update_state — refinement-state update after one denoising forward
+ * of block-wise inference (Sec. 3.1, Eq. 1): commits, confidence history and
+ * active-block advance, in place, for the next forward's reflex_allocate.
+ *
+ * Per sequence s with a = active_block[s] (1 <= a <= num_blocks[s]) and J =
+ * the masked positions of block a:
+ *   - C = {i in J : conf_new[i] >= theta_commit} is committed (masked -> 0);
+ *     if C is empty and J is not, the most confident member of J (lower
+ *     position on ties) is committed instead;
+ *   - every position masked during the forward shifts its history:
+ *     conf_prev2 <- conf_prev1, conf_prev1 <- conf_new, hist_len <-
+ *     min(hist_len + 1, 2);
+ *   - when no position of block a is left masked, active_block[s] = a + 1.
+ * A sequence with active_block[s] > num_blocks[s] is finished and untouched.
+ *
+ *   conf_new        [T] fp32  c^t of the forward (read where masked).
+ *   conf_prev1/2    [T] fp32  in/out, as in reflex_allocate.
+ *   hist_len        [T] u8    in/out.
+ *   masked          [T] u8    in/out.
+ *   block_id        [T] int32, seq_offsets [B+1]: as in reflex_allocate.
+ *   active_block    [B] int32 in/out.
+ *   num_blocks      [B] int32 Q of each sequence (its last target block).
+ *   theta_commit    commitment threshold of Eq. 1 (Sec. 5.1: 0.9).
+ *   committed_out   [B] int32 nullable: positions committed in each sequence.
+ *   dev_status      [1] int32 nullable; error bits are OR-ed in (not cleared).
+ * Device buffers, one CTA per sequence; returns REFLEX_EINVAL for null
+ * pointers, T < 0, B < 1 or a non-finite theta_commit.
+ */
+int reflex_update_state(const float* conf_new, float* conf_prev1, float* conf_prev2,
+                        uint8_t* hist_len, uint8_t* masked, const int32_t* block_id,
+                        const int32_t* seq_offsets, int32_t* active_block,
+                        const int32_t* num_blocks, int32_t T, int32_t B,
+                        float theta_commit, int32_t* committed_out,
+                        int32_t* dev_status, void* stream);
+
 /* Device pointers into the workspace after a forward (the routing record). */
 typedef struct {
     int32_t* ids;     /* [T, k_max] selected experts in router rank order,

@@ -87,6 +87,8 @@ def _load():
                                        i32, i32, i32, i32, i32,
                                        f32, f32, f32, f32, f32,
                                        i32, i32, ctypes.c_uint64, p, p]
+    lib.oracle_update_state.restype = ctypes.c_int
+    lib.oracle_update_state.argtypes = [p, p, p, p, p, p, p, p, p, i32, i32, f32, p]
     lib.oracle_rank_key.restype = f32
     lib.oracle_rank_key.argtypes = [i32, f32, f32, i32, f32, f32, f32, f32]
     lib.oracle_splitmix64.restype = ctypes.c_uint64
@@ -169,6 +171,31 @@ def allocate(conf1, conf2, hist_len, masked, block_id, seq_offsets,
     if rc != 0:
         raise ValueError("oracle_allocate: invalid input")
     return (k, s) if return_scores else k
+
+
+def update_state(state: dict, conf_new, num_blocks, theta_commit: float):
+    """Block-wise inference after one forward (Sec. 3.1, Eq. 1) on a numpy
+    state dict: returns (new state dict, committed per sequence)."""
+    st = {k: np.array(v, copy=True) for k, v in state.items()}
+    st["conf1"] = _c(st["conf1"], np.float32)
+    st["conf2"] = _c(st["conf2"], np.float32)
+    st["hist_len"] = _c(st["hist_len"], np.uint8)
+    st["masked"] = _c(st["masked"], np.uint8)
+    st["active_block"] = _c(st["active_block"], np.int32)
+    conf_new = _c(conf_new, np.float32)
+    block_id = _c(st["block_id"], np.int32)
+    seq_off = _c(st["seq_offsets"], np.int32)
+    nb = _c(num_blocks, np.int32)
+    T = block_id.size
+    B = st["active_block"].size
+    committed = np.zeros(B, np.int32)
+    rc = _load().oracle_update_state(
+        _ptr(conf_new), _ptr(st["conf1"]), _ptr(st["conf2"]), _ptr(st["hist_len"]),
+        _ptr(st["masked"]), _ptr(block_id), _ptr(seq_off), _ptr(st["active_block"]),
+        _ptr(nb), T, B, theta_commit, _ptr(committed))
+    if rc != 0:
+        raise ValueError("oracle_update_state: invalid input")
+    return st, committed
 
 
 def rank_key(signal: int, c1: float, c2: float, hist: int, theta: float,

@@ -14,6 +14,11 @@
  *                        Frontier-Guided Expert Reallocation (Sec. 4.3,
  *                        forecast, Eq. 6-8 and Eq. 9), then the clip of every
  *                        count to [K_min, K_max] required by Eq. 3.
+ *   oracle_update_state  block-wise inference after one forward (Sec. 3.1,
+ *                        Eq. 1): threshold commits in the active block (the
+ *                        most confident one when none reaches the threshold),
+ *                        the confidence history of every masked position, and
+ *                        the active-block advance once the block is resolved.
  *   oracle_allocate_ex   the same with the ablations of App. C: the rank key
  *                        of the Eq. 9 groups (FPS, F only, P only, c^{t-1},
  *                        1 - c^{t-1}) and Role-Shuffled RRB (a seeded
@@ -304,6 +309,59 @@ int oracle_allocate(const float* conf1, const float* conf2,
 /*   acc = +0;  for k = 0..d-1: acc = fmaf(h[t,k], W_r[e,k], acc)            */
 /* Inputs are widened exactly from bf16 when dtype = 1.                      */
 /* ------------------------------------------------------------------------ */
+/* ------------------------------------------------------------------------ */
+/* Refinement-state update after forward t (Sec. 3.1, Eq. 1), per sequence: */
+/*  J = masked positions of the active block a (skip when a > Q).           */
+/*  C = {i in J : c_i >= theta}; if C is empty and J is not, C = {the i in J */
+/*  with the largest c_i, lowest position among equals}.  x_i <- candidate  */
+/*  for i in C (masked_i = 0); J \ C stays masked; other positions keep.   */
+/*  History: every position masked during the forward got the prediction   */
+/*  c_i: c^{t-2} <- c^{t-1}, c^{t-1} <- c_i, hist <- min(hist + 1, 2).      */
+/*  If block a has no masked position left, a <- a + 1.                     */
+/* committed (nullable) receives |C| per sequence.                           */
+/* ------------------------------------------------------------------------ */
+int oracle_update_state(const float* conf_new, float* conf1, float* conf2,
+                        uint8_t* hist_len, uint8_t* masked, const int32_t* block_id,
+                        const int32_t* seq_off, int32_t* active, const int32_t* num_blocks,
+                        int32_t T, int32_t B, float theta, int32_t* committed) {
+    if (T < 0 || B < 0) return OR_EINVAL;
+    if (T > 0 && seq_off[B] != T) return OR_EINVAL;
+    for (int32_t s = 0; s < B; ++s) {
+        int32_t lo = seq_off[s], hi = seq_off[s + 1];
+        int32_t a = active[s];
+        if (committed) committed[s] = 0;
+        if (a < 1) return OR_EINVAL;
+        if (a > num_blocks[s]) continue;                  /* finished */
+        /* the masked set seen by the forward, before any commit */
+        uint8_t* was_masked = (uint8_t*)malloc((size_t)(hi - lo + 1));
+        for (int32_t i = lo; i < hi; ++i) was_masked[i - lo] = masked[i];
+        int32_t nj = 0, nc = 0, best = -1;
+        for (int32_t i = lo; i < hi; ++i) {
+            if (!was_masked[i - lo] || block_id[i] != a) continue;
+            ++nj;
+            if (best < 0 || conf_new[i] > conf_new[best]) best = i;  /* first max */
+            if (conf_new[i] >= theta) {
+                masked[i] = 0;
+                ++nc;
+            }
+        }
+        if (nj > 0 && nc == 0) {
+            masked[best] = 0;
+            nc = 1;
+        }
+        for (int32_t i = lo; i < hi; ++i) {
+            if (!was_masked[i - lo]) continue;
+            conf2[i] = conf1[i];
+            conf1[i] = conf_new[i];
+            hist_len[i] = (uint8_t)(hist_len[i] >= 2 ? 2 : hist_len[i] + 1);
+        }
+        if (nj - nc == 0) active[s] = a + 1;
+        if (committed) committed[s] = nc;
+        free(was_masked);
+    }
+    return OR_OK;
+}
+
 void oracle_router_logits(int32_t dtype, const void* hidden,
                           const void* w_router, int32_t T, int32_t d,
                           int32_t E, float* z) {

@@ -42,7 +42,7 @@ EXPORTED = (
     "reflex_default_params", "reflex_allocate", "reflex_moe_workspace_size",
     "reflex_moe_forward", "reflex_moe_status", "reflex_read_status",
     "reflex_selftest_wait_timeout", "reflex_status_string",
-    "reflex_abi_version", "reflex_route_noalloc",
+    "reflex_abi_version", "reflex_route_noalloc", "reflex_update_state",
 )
 
 
@@ -110,6 +110,9 @@ def load():
     lib.reflex_status_string.argtypes = [ctypes.c_int]
     lib.reflex_abi_version.restype = ctypes.c_int
     lib.reflex_abi_version.argtypes = []
+    lib.reflex_update_state.restype = ctypes.c_int
+    lib.reflex_update_state.argtypes = [P, P, P, P, P, P, P, P, P, i32, i32,
+                                        ctypes.c_float, P, P, P]
     lib.reflex_route_noalloc.restype = ctypes.c_int
     lib.reflex_route_noalloc.argtypes = [i32, P, P, P, i32, i32, i32, i32,
                                          ctypes.c_uint32, P, P, P, P]
@@ -153,6 +156,20 @@ def make_params(**kw) -> reflex_alloc_params:
     for k, v in kw.items():
         setattr(p, k, v)
     return p
+
+
+def reflex_update_state(conf_new, conf_prev1, conf_prev2, hist_len, masked,
+                        block_id, seq_offsets, active_block, num_blocks, T: int,
+                        B: int, theta_commit: float, committed_out=None,
+                        dev_status=None, stream=None, check: bool = True) -> int:
+    rc = load().reflex_update_state(
+        _ptr(conf_new), _ptr(conf_prev1), _ptr(conf_prev2), _ptr(hist_len),
+        _ptr(masked), _ptr(block_id), _ptr(seq_offsets), _ptr(active_block),
+        _ptr(num_blocks), T, B, float(theta_commit), _ptr(committed_out),
+        _ptr(dev_status), _stream(stream))
+    if check and rc != REFLEX_OK:
+        raise ReflexError(rc, "reflex_update_state")
+    return rc
 
 
 def reflex_allocate(router_scores, conf_prev1, conf_prev2, hist_len, masked,

@@ -52,6 +52,24 @@ def allocate(state: dict, params: B.reflex_alloc_params, E: int = 0,
     return k_out, k_sum, status
 
 
+def update_state(state: dict, conf_new: torch.Tensor, num_blocks: torch.Tensor,
+                 theta_commit: float, stream=None,
+                 committed: torch.Tensor | None = None,
+                 status: torch.Tensor | None = None):
+    """reflex_update_state in place on device state tensors (Eq. 1 commits,
+    confidence history, active-block advance); returns committed [B]."""
+    T = int(state["block_id"].numel())
+    nseq = int(state["active_block"].numel())
+    dev = state["block_id"].device
+    committed = (torch.empty(nseq, dtype=torch.int32, device=dev)
+                 if committed is None else committed)
+    B.reflex_update_state(conf_new, state["conf1"], state["conf2"], state["hist_len"],
+                          state["masked"], state["block_id"], state["seq_offsets"],
+                          state["active_block"], num_blocks, T, nseq, theta_commit,
+                          committed, status, stream)
+    return committed
+
+
 class MoELayer:
     """One variable-count MoE layer on the device with its workspace sized for
     `max_tokens` tokens at `k_max`."""

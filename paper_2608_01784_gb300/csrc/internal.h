@@ -28,6 +28,13 @@ cudaError_t launch_budget(const float* conf1, const float* conf2,
 cudaError_t launch_wait_selftest(uint32_t* err, uint64_t limit_ns,
                                  cudaStream_t stream);
 
+// ---- refinement-state update (state.cu) ------------------------------------
+cudaError_t launch_update_state(const float* conf_new, float* conf1, float* conf2,
+                                uint8_t* hist_len, uint8_t* masked, const int32_t* block_id,
+                                const int32_t* seq_off, int32_t* active,
+                                const int32_t* num_blocks, int T, int B, float theta,
+                                int32_t* committed, uint32_t* err, cudaStream_t stream);
+
 // ---- routing (router.cu) --------------------------------------------------
 // z[T, E] = router scores (sequential fp32 fma chain over the hidden index).
 // The first CTA also clears zero_words[0, n_zero) (nullable): the call's

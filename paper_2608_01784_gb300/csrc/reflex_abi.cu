@@ -4,6 +4,7 @@
 // (except the explicit status readers).
 #include <cudaTypedefs.h>
 
+#include <cmath>
 #include <cstring>
 #include <mutex>
 
@@ -201,6 +202,26 @@ int reflex_allocate(const float* router_scores, const float* conf_prev1,
                             seq_offsets, active_block, T, B, a, k_out,
                             reinterpret_cast<unsigned long long*>(k_sum_out),
                             err, s));
+  return REFLEX_OK;
+}
+
+int reflex_update_state(const float* conf_new, float* conf_prev1, float* conf_prev2,
+                        uint8_t* hist_len, uint8_t* masked, const int32_t* block_id,
+                        const int32_t* seq_offsets, int32_t* active_block,
+                        const int32_t* num_blocks, int32_t T, int32_t B,
+                        float theta_commit, int32_t* committed_out,
+                        int32_t* dev_status, void* stream) {
+  if (T < 0 || B < 1 || !std::isfinite(theta_commit)) return REFLEX_EINVAL;
+  if (seq_offsets == nullptr || active_block == nullptr || num_blocks == nullptr)
+    return REFLEX_EINVAL;
+  if (T > 0 && (conf_new == nullptr || conf_prev1 == nullptr || conf_prev2 == nullptr ||
+                hist_len == nullptr || masked == nullptr || block_id == nullptr))
+    return REFLEX_EINVAL;
+  RX_CUDA(rx::launch_update_state(conf_new, conf_prev1, conf_prev2, hist_len, masked,
+                                  block_id, seq_offsets, active_block, num_blocks, T, B,
+                                  theta_commit, committed_out,
+                                  reinterpret_cast<uint32_t*>(dev_status),
+                                  static_cast<cudaStream_t>(stream)));
   return REFLEX_OK;
 }
 

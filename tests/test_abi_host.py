@@ -118,3 +118,14 @@ def test_host_rejections_enqueue_nothing(lib):
     assert rec.ids == 256 + 256          # first region after the header
     assert lib.reflex_selftest_wait_timeout(None, 10, None) == B.REFLEX_EINVAL
     assert lib.reflex_read_status(None, None) == B.REFLEX_EINVAL
+
+
+def test_update_state_host_rejections(lib):
+    from paper_2608_01784_gb300 import _binding as B
+    # every check returns before a pointer is used
+    assert lib.reflex_update_state(None, None, None, None, None, None, None, None, None,
+                                   4, 0, 0.9, None, None, None) == B.REFLEX_EINVAL
+    assert lib.reflex_update_state(None, None, None, None, None, None, 1, 1, 1,
+                                   4, 1, 0.9, None, None, None) == B.REFLEX_EINVAL
+    assert lib.reflex_update_state(1, 1, 1, 1, 1, 1, 1, 1, 1, 4, 1, float("nan"),
+                                   None, None, None) == B.REFLEX_EINVAL
