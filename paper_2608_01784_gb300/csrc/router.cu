@@ -191,7 +191,8 @@ cudaError_t launch_logits_tile(const Tin* h, const Tin* w, int T, int d, int E,
     if (e != cudaSuccess) return e;
   }
   const dim3 g((T + C::BT - 1) / C::BT, (E + C::BE - 1) / C::BE);
-  return launch_pdl(kern, g, dim3(C::kThreads), C::kSmem, s, h, w, T, d, E, z, zw, nz);
+  kern<<<g, C::kThreads, C::kSmem, s>>>(h, w, T, d, E, z, zw, nz);
+  return cudaGetLastError();
 }
 
 __device__ __forceinline__ uint32_t order_bits(float v) {
@@ -398,7 +399,8 @@ cudaError_t launch_logits_short(const Tin* h, const Tin* w, int T, int d, int E,
     if (e != cudaSuccess) return e;
   }
   const dim3 g((T + 8 * TM - 1) / (8 * TM), (E + 63) / 64);
-  return launch_pdl(kern, g, dim3(kThreadsS), smem, s, h, w, T, d, E, z, zw, nz);
+  kern<<<g, kThreadsS, smem, s>>>(h, w, T, d, E, z, zw, nz);
+  return cudaGetLastError();
 }
 
 // ---- bf16 scores with mixed-precision fma ----------------------------------
@@ -556,7 +558,8 @@ cudaError_t launch_logits_mx(const __nv_bfloat16* h, const __nv_bfloat16* w, int
     if (e != cudaSuccess) return e;
   }
   const dim3 g((T + C::BT - 1) / C::BT, (E + C::BE - 1) / C::BE);
-  return launch_pdl(kern, g, dim3(C::NT), C::kSmem, s, h, w, T, d, E, z, zw, nz);
+  kern<<<g, C::NT, C::kSmem, s>>>(h, w, T, d, E, z, zw, nz);
+  return cudaGetLastError();
 }
 
 // fp32 inputs: the widened-buffer tiles when they fill most SMs without
@@ -575,6 +578,12 @@ cudaError_t logits_dispatch(const float* h, const float* w, int T, int d, int E,
   return launch_logits_short<float, 1>(h, w, T, d, E, z, zw, nz, s);
 }
 
+// The score kernels are launched without programmatic serialization: with a
+// tile count of one or two CTAs per SM, CTAs placed early on the SMs that a
+// wide predecessor (the previous layer's combine) frees first pile up there,
+// and the unbalanced placement cost up to 100 us at 4096 x 256 scores on
+// GB300.  They still clear the header and let the next kernel launch early.
+//
 // bf16 inputs: mixed-precision fma tiles, chosen by the number of chains
 // T x E per SM (measured on GB300 over T = 256 .. 65536, E = 64 and 256).
 // Few chains: small thread tiles so every SM gets warps; many chains: 4 x 8
