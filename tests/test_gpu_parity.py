@@ -173,6 +173,8 @@ def _bf16_case(T, d, E, inter, shared, kmax, seed):
     (777, 512, 16, 256, 128, 6, "random"),  # shared expert, N > one tile
     (1, 256, 8, 128, 0, 4, "random"),      # single token
     (300, 256, 64, 128, 0, 2, "one"),      # many empty experts
+    (500, 256, 16, 128, 0, 8, "max"),      # every token at k_max: two ragged m-tiles per group
+    (1500, 256, 8, 256, 0, 4, "random"),   # 1-SM tiles, a few hundred rows per group
     (4096, 256, 4, 128, 0, 4, "random"),   # CTA-pair (2-SM) GEMMs, ragged groups
     (2048, 512, 8, 256, 0, 4, "max"),      # CTA-pair GEMMs, several n-tiles
 ])
