@@ -50,7 +50,7 @@ METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
 # ncu capture of the current kernel on the same workload
 # (profiles/grouped_gemm_llada_moe_T1024.md); workloads without a capture of
 # the current kernel report null.
-NCU_TRAFFIC_BYTES = {"llada_moe": 568977664}
+NCU_TRAFFIC_BYTES = {"llada_moe": 561247744}
 
 
 def parse():
