@@ -174,7 +174,8 @@ def _bf16_case(T, d, E, inter, shared, kmax, seed):
     (1, 256, 8, 128, 0, 4, "random"),      # single token
     (300, 256, 64, 128, 0, 2, "one"),      # many empty experts
     (500, 256, 16, 128, 0, 8, "max"),      # every token at k_max: two ragged m-tiles per group
-    (1500, 256, 8, 256, 0, 4, "random"),   # 1-SM tiles, a few hundred rows per group
+    (1500, 256, 8, 256, 0, 4, "random"),   # CTA-pair tiles, a few hundred rows per group
+    (4096, 256, 256, 512, 0, 6, "random"),  # 1-SM 256-wide tiles, ~48 rows per group
     (4096, 256, 4, 128, 0, 4, "random"),   # CTA-pair (2-SM) GEMMs, ragged groups
     (2048, 512, 8, 256, 0, 4, "max"),      # CTA-pair GEMMs, several n-tiles
 ])
