@@ -349,14 +349,20 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
         return REFLEX_ECUDA;
       rx::TcGemmArgs g1{&ma1, &mb1, d, inter, 2 * inter, inter, grouped, amid, inter, err, sms};
       rx::TcGemmArgs g2{&ma2, &mb2, inter, d, d, 0, grouped, xperm, d, err, sms};
+      // the dense shared expert on CTA pairs once it has enough rows: a 256 x
+      // 256 pair tile moves a quarter of the operand bytes per output that a
+      // 128 x 128 tile of the 1-SM kernel moves from L2 (LLaDA2.0-mini layer
+      // 0.750 -> 0.736 ms; at 1024 tokens the 1-SM tiles stay 6 us faster)
+      const bool pair_shared =
+          shared_inter > 0 && T >= 2048 && shared_inter % 128 == 0 && d % 256 == 0;
       CUtensorMap sa1, sb1, sa2, sb2;
       if (shared_inter &&
           (!make_map(&sa1, hidden, T, d, rx::kTileM) ||
            !make_map(&sb1, shared_gate_up, 2 * static_cast<int64_t>(shared_inter), d,
-                     rx::tc_b_box_rows(true, bn_sup)) ||
+                     pair_shared ? 128 : rx::tc_b_box_rows(true, bn_sup)) ||
            !make_map(&sa2, ash, T, shared_inter, rx::kTileM) ||
            !make_map(&sb2, shared_down, d, shared_inter,
-                     rx::tc_b_box_rows(false, bn_sdn))))
+                     pair_shared ? 128 : rx::tc_b_box_rows(false, bn_sdn))))
         return REFLEX_ECUDA;
       rx::TcGemmArgs h1{&sa1, &sb1, d, shared_inter, 2 * shared_inter, shared_inter,
                         dense, ash, shared_inter, err, sms};
@@ -366,14 +372,24 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
           RX_CUDA(rx::launch_swiglu_tc_pair(g1, s));
         else
           RX_CUDA(rx::launch_swiglu_tc(g1, bn_up, s));
-        if (shared_inter) RX_CUDA(rx::launch_swiglu_tc(h1, bn_sup, s));
+        if (shared_inter) {
+          if (pair_shared)
+            RX_CUDA(rx::launch_swiglu_tc_pair(h1, s));
+          else
+            RX_CUDA(rx::launch_swiglu_tc(h1, bn_sup, s));
+        }
       }
       if (down) {
         if (pair_routed)
           RX_CUDA(rx::launch_down_tc_pair(g2, s));
         else
           RX_CUDA(rx::launch_down_tc(g2, bn_dn, s));
-        if (shared_inter) RX_CUDA(rx::launch_down_tc(h2, bn_sdn, s));
+        if (shared_inter) {
+          if (pair_shared)
+            RX_CUDA(rx::launch_down_tc_pair(h2, s));
+          else
+            RX_CUDA(rx::launch_down_tc(h2, bn_sdn, s));
+        }
       }
     }
   }
