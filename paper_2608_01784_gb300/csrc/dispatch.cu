@@ -20,16 +20,19 @@
 namespace rx {
 namespace {
 
-constexpr int kBlk = kDispatchBlock;  // tokens per block (8 mask words)
-constexpr int kWords = kBlk / 32;
 
 __device__ __forceinline__ int clamp_k(int kt, int kcap) {
   return kt < 1 ? 1 : (kt > kcap ? kcap : kt);
 }
 
+// BLK tokens per block (one CTA of BLK threads), BLK / 32 mask words per
+// expert: 32-token blocks up to 4096 tokens (more CTAs for short batches),
+// 256-token blocks beyond (fewer blocks for the scan).
+template <int BLK>
 __device__ void build_masks(uint32_t* mask, const int32_t* ids,
                             const int32_t* k, int T, int E, int k_max,
                             uint32_t* err) {
+  constexpr int kBlk = BLK, kWords = BLK / 32;
   for (int i = threadIdx.x; i < E * kWords; i += kBlk) mask[i] = 0u;
   __syncthreads();
   const int t = blockIdx.x * kBlk + threadIdx.x;
@@ -46,14 +49,16 @@ __device__ void build_masks(uint32_t* mask, const int32_t* ids,
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(kBlk)
+template <int BLK>
+__global__ void __launch_bounds__(BLK)
     count_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ k,
                  int T, int E, int k_max, int32_t* __restrict__ blk_count,
                  uint32_t* __restrict__ err) {
+  constexpr int kBlk = BLK, kWords = BLK / 32;
   extern __shared__ uint32_t mask[];
   grid_dep_wait();
   grid_dep_launch();
-  build_masks(mask, ids, k, T, E, k_max, err);
+  build_masks<BLK>(mask, ids, k, T, E, k_max, err);
   for (int e = threadIdx.x; e < E; e += kBlk) {
     int c = 0;
 #pragma unroll
@@ -129,17 +134,19 @@ __global__ void __launch_bounds__(1024)
   }
 }
 
-__global__ void __launch_bounds__(kBlk)
+template <int BLK>
+__global__ void __launch_bounds__(BLK)
     scatter_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ k,
                    int T, int E, int k_max,
                    const int32_t* __restrict__ blk_off,
                    const int32_t* __restrict__ offsets,
                    int32_t* __restrict__ perm, int32_t* __restrict__ row_of,
                    uint32_t* __restrict__ err) {
+  constexpr int kBlk = BLK, kWords = BLK / 32;
   extern __shared__ uint32_t mask[];
   grid_dep_wait();
   grid_dep_launch();
-  build_masks(mask, ids, k, T, E, k_max, nullptr);
+  build_masks<BLK>(mask, ids, k, T, E, k_max, nullptr);
   const int t = blockIdx.x * kBlk + threadIdx.x;
   if (t >= T) return;
   const int kt = clamp_k(k[t], k_max < E ? k_max : E);
@@ -212,26 +219,34 @@ __global__ void __launch_bounds__(256)
 
 }  // namespace
 
-cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T, int E,
-                            int k_max, const DispatchBufs& b,
-                            cudaStream_t stream) {
-  if (T == 0) return cudaSuccess;
-  const int nblk = (T + kBlk - 1) / kBlk;
-  const size_t smem = static_cast<size_t>(E) * kWords * sizeof(uint32_t);
+template <int BLK>
+cudaError_t launch_dispatch_blk(const int32_t* ids, const int32_t* k, int T, int E, int k_max,
+                                const DispatchBufs& b, cudaStream_t stream) {
+  const int nblk = (T + BLK - 1) / BLK;
+  const size_t smem = static_cast<size_t>(E) * (BLK / 32) * sizeof(uint32_t);
   if (smem > 48 * 1024) {
-    cudaError_t e1 = cudaFuncSetAttribute(count_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    cudaError_t e2 = cudaFuncSetAttribute(scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e1 = cudaFuncSetAttribute(count_kernel<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e2 = cudaFuncSetAttribute(scatter_kernel<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e1 != cudaSuccess) return e1;
     if (e2 != cudaSuccess) return e2;
   }
-  cudaError_t e = launch_pdl(count_kernel, dim3(nblk), dim3(kBlk), smem, stream, ids, k, T,
+  cudaError_t e = launch_pdl(count_kernel<BLK>, dim3(nblk), dim3(BLK), smem, stream, ids, k, T,
                              E, k_max, b.blk_count, b.err);
   if (e != cudaSuccess) return e;
   e = launch_pdl(scan_kernel, dim3(1), dim3(1024), 0, stream, b.blk_count, nblk, E, b.blk_off,
                  b.counts, b.offsets, b.mt_prefix, b.mt2_prefix, b.totals);
   if (e != cudaSuccess) return e;
-  return launch_pdl(scatter_kernel, dim3(nblk), dim3(kBlk), smem, stream, ids, k, T, E, k_max,
-                    b.blk_off, b.offsets, b.perm, b.row_of, b.err);
+  return launch_pdl(scatter_kernel<BLK>, dim3(nblk), dim3(BLK), smem, stream, ids, k, T, E,
+                    k_max, b.blk_off, b.offsets, b.perm, b.row_of, b.err);
+}
+
+cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T, int E,
+                            int k_max, const DispatchBufs& b,
+                            cudaStream_t stream) {
+  if (T == 0) return cudaSuccess;
+  if (dispatch_block(T) == kDispatchBlockSmall)
+    return launch_dispatch_blk<kDispatchBlockSmall>(ids, k, T, E, k_max, b, stream);
+  return launch_dispatch_blk<kDispatchBlock>(ids, k, T, E, k_max, b, stream);
 }
 
 cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* row_of,

@@ -62,7 +62,17 @@ struct DispatchBufs {
   int32_t* totals;     // header: total_pairs, total_mtiles, total_mtiles2
   uint32_t* err;
 };
-constexpr int kDispatchBlock = 256;  // tokens per dispatch block
+constexpr int kDispatchBlock = 256;       // tokens per dispatch block, large batches
+constexpr int kDispatchBlockSmall = 32;   // tokens per dispatch block up to 4096 tokens
+constexpr int kDispatchSmallT = 4096;
+inline int dispatch_block(int T) { return T <= kDispatchSmallT ? kDispatchBlockSmall : kDispatchBlock; }
+// per-block count buffers sized for either block size (monotonic in T, so a
+// workspace sized for a batch also fits every smaller one)
+inline int64_t dispatch_blocks_alloc(int T) {
+  const int ts = T < kDispatchSmallT ? T : kDispatchSmallT;
+  return (ts + kDispatchBlockSmall - 1) / kDispatchBlockSmall +
+         (T + kDispatchBlock - 1) / kDispatchBlock;
+}
 cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T,
                             int E, int k_max, const DispatchBufs& b,
                             cudaStream_t stream);

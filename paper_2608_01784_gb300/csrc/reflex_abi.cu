@@ -43,7 +43,7 @@ Layout make_layout(int32_t dtype, int32_t T, int32_t d, int32_t E,
   Layout L{};
   const size_t es = dtype == REFLEX_DTYPE_F32 ? 4 : 2;
   const int64_t cap = static_cast<int64_t>(T) * k_max;
-  const int nblk = (T + rx::kDispatchBlock - 1) / rx::kDispatchBlock;
+  const int64_t nblk = rx::dispatch_blocks_alloc(T);
   size_t o = 0;
   auto take = [&](size_t bytes) {
     const size_t at = o;
