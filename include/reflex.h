@@ -211,6 +211,8 @@ typedef struct {
                          (expert, token)                                    */
     int32_t* row_of;  /* [T, k_max] pair row of (token, slot), -1 unused    */
     int32_t* totals;  /* [2] device: sum k (pairs), number of 128-row tiles */
+    float* scores;    /* [T, E] router scores r_i (fp32, the fma chain of
+                         reflex_moe_forward); valid after the ROUTE stage   */
 } reflex_route_record;
 
 /* Bytes of workspace reflex_moe_forward needs for these shapes (0 if the

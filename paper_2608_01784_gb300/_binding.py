@@ -60,7 +60,7 @@ class reflex_route_record(ctypes.Structure):
     _fields_ = [("ids", ctypes.c_void_p), ("alpha", ctypes.c_void_p),
                 ("counts", ctypes.c_void_p), ("offsets", ctypes.c_void_p),
                 ("perm", ctypes.c_void_p), ("row_of", ctypes.c_void_p),
-                ("totals", ctypes.c_void_p)]
+                ("totals", ctypes.c_void_p), ("scores", ctypes.c_void_p)]
 
 
 class ReflexError(RuntimeError):

@@ -132,4 +132,5 @@ class MoELayer:
             perm=self._view(self.rec.perm, n_pairs),
             row_of=self._view(self.rec.row_of, T * km).view(T, km),
             totals=totals,
+            scores=self._view(self.rec.scores, T * E, torch.float32).view(T, E),
         )

@@ -38,11 +38,12 @@ cudaError_t launch_update_state(const float* conf_new, float* conf1, float* conf
 // ---- routing (router.cu) --------------------------------------------------
 // z[T, E] = router scores (sequential fp32 fma chain over the hidden index).
 // The first CTA also clears zero_words[0, n_zero) (nullable): the call's
-// header or error word, so no memset precedes the first kernel.
+// header or error word, so no memset precedes the first kernel.  err
+// (nullable) receives kErrTimeout if a bounded wait of a kernel expires.
 cudaError_t launch_router_logits(int dtype, const void* hidden,
                                  const void* w_router, int T, int d, int E,
                                  float* z, uint32_t* zero_words, int n_zero,
-                                 int num_sms, cudaStream_t stream);
+                                 uint32_t* err, int num_sms, cudaStream_t stream);
 // ids/alpha [T, k_max] from z and the counts k.
 cudaError_t launch_router_select(const float* z, const int32_t* k, int T,
                                  int E, int k_max, bool renorm, int32_t* ids,

@@ -133,7 +133,7 @@ int map_err_bits(uint32_t bits) {
 
 extern "C" {
 
-int reflex_abi_version(void) { return 110; }
+int reflex_abi_version(void) { return 111; }
 
 const char* reflex_status_string(int s) {
   switch (s) {
@@ -259,6 +259,7 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
     rec->perm = I32(L.perm);
     rec->row_of = I32(L.row_of);
     rec->totals = totals;
+    rec->scores = reinterpret_cast<float*>(ws + L.z);
   }
   if (T == 0) return REFLEX_OK;
   if (hidden == nullptr || w_router == nullptr || w_gate_up == nullptr ||
@@ -307,7 +308,7 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
     // kernel before the router reads it
     RX_CUDA(rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z,
                                      reinterpret_cast<uint32_t*>(hdr),
-                                     static_cast<int>(sizeof(WsHeader) / 4), sms, s));
+                                     static_cast<int>(sizeof(WsHeader) / 4), err, sms, s));
     RX_CUDA(rx::launch_router_select(z, k, T, E, k_max,
                                      (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
                                      I32(L.ids), alpha, err, s));

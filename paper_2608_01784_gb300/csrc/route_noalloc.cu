@@ -77,8 +77,8 @@ extern "C" int reflex_route_noalloc(int32_t dtype, const void* hidden,
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint32_t* err = reinterpret_cast<uint32_t*>(dev_status);
   // the router clears the error word before select may set bits in it
-  if (rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z, err, err ? 1 : 0, sms,
-                               s) != cudaSuccess)
+  if (rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z, err, err ? 1 : 0, err,
+                               sms, s) != cudaSuccess)
     return REFLEX_ECUDA;
   if (rx::launch_router_select(z, k, T, E, k_max, (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
                                ids_out, alpha_out, err, s) != cudaSuccess)

@@ -167,6 +167,32 @@ def _bf16_case(T, d, E, inter, shared, kmax, seed):
     return cfg, layer
 
 
+# every score-kernel band of the bf16 router (chains T x E per SM on 152 SMs)
+@pytest.mark.parametrize("T,E,d", [
+    (100, 64, 2048),     # ring kernel, 1 x 1 thread tiles
+    (1000, 64, 2048),    # whole rows resident, ragged token tile
+    (1200, 48, 512),     # whole rows resident, ragged expert tile
+    (250, 256, 1024),    # whole rows resident, 4 chunks
+    (2000, 64, 256),     # ring kernel, 1 x 2
+    (4096, 64, 256),     # ring kernel, 2 x 2, 64-k chunks
+    (8192, 128, 256),    # ring kernel, 4 x 8
+    (8192, 256, 256),    # ring kernel, 4 x 4
+    (16384, 256, 256),   # ring kernel, 4 x 8, 4 stages
+])
+def test_router_scores_bit_exact_every_band(T, E, d):
+    cfg, layer = _bf16_case(T, d, E, 128, 0, 8, seed=T + E + d)
+    k = np.random.default_rng(T).integers(1, 9, T).astype(np.int32)
+    gl = G.GpuLayer(cfg, layer)
+    _, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE)
+    assert status == B.REFLEX_OK
+    z = oracle.router_logits(layer["hidden"], layer["w_router"])
+    assert np.array_equal(rec["scores"].view(np.uint32), z.view(np.uint32))
+    ids, alpha = oracle.select(z, k, cfg.k_max)
+    assert np.array_equal(rec["ids"], ids)
+    valid = ids >= 0
+    np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
+
+
 @pytest.mark.parametrize("T,d,E,inter,shared,kmax,kmode", [
     (96, 256, 8, 128, 0, 4, "random"),     # one partial m-tile per expert
     (1000, 256, 4, 128, 0, 4, "max"),      # 8 m-tiles per expert, ragged tail
