@@ -1,9 +1,10 @@
 """Benchmark of the REFLEX per-forward MoE hot path on GB300.
 
-One step = one denoising forward's hot path on one batch:
-  reflex_allocate (per-token counts, Eq. 5 / Eq. 9 + clip)
-  + reflex_moe_forward (router scores, variable-count TopK, pair dispatch,
-    grouped SwiGLU expert GEMMs on tcgen05, weighted combine; Eq. 2).
+One step = one denoising forward's hot path on one batch, one reflex_step
+call: the per-token counts of reflex_allocate (Eq. 5 / Eq. 9 + clip) and
+reflex_moe_forward with them (router scores, variable-count TopK, pair
+dispatch, grouped SwiGLU expert GEMMs on tcgen05, weighted combine; Eq. 2),
+the count kernel running beside the router scores.
 Default workload: the LLaDA-MoE-shaped layer (T = 1024 tokens: 512 prompt +
 512 generated in blocks of 32; d = 2048, E = 64 SwiGLU experts with inter =
 1024; K in [2, 12]; bf16 storage, fp32 accumulation), synthetic inputs.
@@ -253,14 +254,14 @@ def run_gpu(args, cfg, rank, world, local_rank):
     # every call takes the current stream, so the steps can be captured into
     # CUDA graphs (the library never synchronises with the host)
     def step(params, hidden=None):
-        api.allocate(ds, params, E, None, k_buf, k_sum, st)
-        moe.forward(dl["hidden"] if hidden is None else hidden, k_buf, out, F)
+        moe.step(ds, params, dl["hidden"] if hidden is None else hidden, out=out,
+                 k_out=k_buf, k_sum=k_sum, status=st, flags=F)
 
     def staged_step(params, up_events):
         # the same work as step(), split so that events bracket the gate/up GEMM
-        api.allocate(ds, params, E, None, k_buf, k_sum, st)
         h = dl["hidden"]
-        moe.forward(h, k_buf, out, F | B.REFLEX_STAGE_ROUTE | B.REFLEX_STAGE_DISPATCH)
+        moe.step(ds, params, h, out=out, k_out=k_buf, k_sum=k_sum, status=st,
+                 flags=F | B.REFLEX_STAGE_ROUTE | B.REFLEX_STAGE_DISPATCH)
         up_events[0].record()
         moe.forward(h, k_buf, out, F | B.REFLEX_STAGE_EXPERT_UP)
         up_events[1].record()
@@ -365,8 +366,8 @@ def run_gpu(args, cfg, rank, world, local_rank):
                     ev_up[b].record(copy_s)
                 stream.wait_event(ev_up[b])
                 stream.wait_event(ev_read[b])      # read-back of step i-2 done
-                api.allocate(dev_state[b], p_reflex, E, None, k_buf, k_sum, st)
-                moe.forward(dev_h[b], k_buf, dev_out[b], F)
+                moe.step(dev_state[b], p_reflex, dev_h[b], out=dev_out[b], k_out=k_buf,
+                         k_sum=k_sum, status=st, flags=F)
                 ev_done[b].record(stream)
             if i > 0:
                 pb = (i - 1) & 1
@@ -434,7 +435,8 @@ def run_gpu(args, cfg, rank, world, local_rank):
         config=dict(workload=cfg.name, description=cfg.description,
                     tokens_per_step=T, parallelism=f"replicas{world}",
                     l2="no flush: expert weights > 129 MB L2 stream from HBM every step",
-                    timing="CUDA-graph replay of one step (allocation + forward) per "
+                    timing="CUDA-graph replay of one step (one reflex_step call: "
+                           "allocation + forward) per "
                            "timed iteration; e2e: eager API calls, each step's upload "
                            "and read-back from pinned host memory on a copy stream, "
                            "double-buffered so they overlap the neighbouring steps"),
@@ -692,8 +694,8 @@ def run_ablation(args, rank, world, local_rank):
             api.allocate(ds, params[i % steps], E, stream, k_buf, k_sum, st)
 
         def step(i):
-            alloc(i)
-            moe.forward(dl["hidden"], k_buf, out, F)
+            moe.step(ds, params[i % steps], dl["hidden"], out=out, k_out=k_buf,
+                     k_sum=k_sum, status=st, flags=F)
 
         alloc(0)
         moe.forward(dl["hidden"], k_buf, out, F)

@@ -259,6 +259,39 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
                        void* out, reflex_route_record* rec, void* stream);
 
 /*
+ * reflex_step — one denoising forward's hot path in one call: the per-token
+ * counts of reflex_allocate (Eq. 5, Eq. 6-9, clip to [K_min, K_max]) for the
+ * state arrays, then reflex_moe_forward with those counts (Eq. 2).  Every
+ * output equals, bit for bit, that of reflex_allocate followed by
+ * reflex_moe_forward on the same stream with the same arguments.  The
+ * router scores do not depend on the counts, so the count kernel is launched
+ * right behind the score kernel and runs beside it; the TopK selection waits
+ * for both.
+ *
+ *   conf_prev1 .. active_block, B, p, k_out, k_sum_out: as for
+ *                   reflex_allocate (T is the forward's T); alloc_status is
+ *                   its device error word (nullable; stored or cleared by the
+ *                   call, then OR-ed), separate from the forward's error word
+ *                   in the workspace.
+ *   dtype .. rec:   as for reflex_moe_forward; the counts read by the forward
+ *                   are k_out (written by this call).
+ * Ownership and errors: every pointer except rec and p is device memory owned
+ * by the caller; nothing is allocated.  Any argument error of either half
+ * returns its status before anything is launched.  The REFLEX_STAGE_* bits of
+ * flags select the forward's stages as for reflex_moe_forward; the counts are
+ * computed in every case.
+ */
+int reflex_step(const float* conf_prev1, const float* conf_prev2, const uint8_t* hist_len,
+                const uint8_t* masked, const int32_t* block_id, const int32_t* seq_offsets,
+                const int32_t* active_block, int32_t B, const reflex_alloc_params* p,
+                int32_t* k_out, int64_t* k_sum_out, int32_t* alloc_status,
+                int32_t dtype, const void* hidden, const void* w_router,
+                const void* w_gate_up, const void* w_down, const void* shared_gate_up,
+                const void* shared_down, int32_t shared_inter, int32_t T, int32_t d,
+                int32_t E, int32_t inter, int32_t k_max, uint32_t flags, void* workspace,
+                size_t ws_bytes, void* out, reflex_route_record* rec, void* stream);
+
+/*
  * reflex_route_noalloc — the routing step of reflex_moe_forward (router
  * scores, TopK(r_i, k_i), router weights) for callers that cannot allocate
  * device memory: code inside a framework that owns the device allocator and

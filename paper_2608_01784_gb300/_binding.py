@@ -43,6 +43,7 @@ EXPORTED = (
     "reflex_moe_forward", "reflex_moe_status", "reflex_read_status",
     "reflex_selftest_wait_timeout", "reflex_status_string",
     "reflex_abi_version", "reflex_route_noalloc", "reflex_update_state",
+    "reflex_step",
 )
 
 
@@ -113,6 +114,11 @@ def load():
     lib.reflex_update_state.restype = ctypes.c_int
     lib.reflex_update_state.argtypes = [P, P, P, P, P, P, P, P, P, i32, i32,
                                         ctypes.c_float, P, P, P]
+    lib.reflex_step.restype = ctypes.c_int
+    lib.reflex_step.argtypes = [P, P, P, P, P, P, P, i32, ctypes.POINTER(reflex_alloc_params),
+                                P, P, P, i32, P, P, P, P, P, P, i32, i32, i32, i32, i32,
+                                i32, ctypes.c_uint32, P, ctypes.c_size_t, P,
+                                ctypes.POINTER(reflex_route_record), P]
     lib.reflex_route_noalloc.restype = ctypes.c_int
     lib.reflex_route_noalloc.argtypes = [i32, P, P, P, i32, i32, i32, i32,
                                          ctypes.c_uint32, P, P, P, P]
@@ -205,6 +211,25 @@ def reflex_moe_forward(dtype: int, hidden, w_router, w_gate_up, w_down,
         ctypes.byref(rec) if rec is not None else None, _stream(stream))
     if check and rc != REFLEX_OK:
         raise ReflexError(rc, "reflex_moe_forward")
+    return rc
+
+
+def reflex_step(conf_prev1, conf_prev2, hist_len, masked, block_id, seq_offsets,
+                active_block, B: int, params: reflex_alloc_params, k_out, k_sum_out,
+                alloc_status, dtype: int, hidden, w_router, w_gate_up, w_down,
+                shared_gate_up, shared_down, shared_inter: int, T: int, d: int, E: int,
+                inter: int, k_max: int, flags: int, workspace, ws_bytes: int, out,
+                rec: reflex_route_record | None = None, stream=None,
+                check: bool = True) -> int:
+    rc = load().reflex_step(
+        _ptr(conf_prev1), _ptr(conf_prev2), _ptr(hist_len), _ptr(masked), _ptr(block_id),
+        _ptr(seq_offsets), _ptr(active_block), B, ctypes.byref(params), _ptr(k_out),
+        _ptr(k_sum_out), _ptr(alloc_status), dtype, _ptr(hidden), _ptr(w_router),
+        _ptr(w_gate_up), _ptr(w_down), _ptr(shared_gate_up), _ptr(shared_down),
+        shared_inter, T, d, E, inter, k_max, flags, _ptr(workspace), ws_bytes, _ptr(out),
+        ctypes.byref(rec) if rec is not None else None, _stream(stream))
+    if check and rc != REFLEX_OK:
+        raise ReflexError(rc, "reflex_step")
     return rc
 
 

@@ -111,6 +111,36 @@ class MoELayer:
         self._T = T
         return out
 
+    def step(self, state: dict, params: B.reflex_alloc_params, hidden: torch.Tensor,
+             out=None, k_out: torch.Tensor | None = None,
+             k_sum: torch.Tensor | None = None, status: torch.Tensor | None = None,
+             flags: int = B.REFLEX_FLAG_RENORM_TOPK, stream=None, check: bool = True):
+        """reflex_step: the counts of `state` (as allocate) and the forward with
+        them in one call -> (out, k int32 [T], k_sum int64 [1], status int32 [1])."""
+        T = int(hidden.shape[0])
+        if T > self.max_tokens:
+            raise ValueError("more tokens than the workspace was sized for")
+        if int(state["block_id"].numel()) != T:
+            raise ValueError("state and hidden disagree on the token count")
+        dev = hidden.device
+        nseq = int(state["active_block"].numel())
+        out = torch.empty((T, self.d), dtype=self.tdtype, device=dev) if out is None else out
+        k_out = torch.empty(T, dtype=torch.int32, device=dev) if k_out is None else k_out
+        k_sum = torch.zeros(1, dtype=torch.int64, device=dev) if k_sum is None else k_sum
+        status = torch.zeros(1, dtype=torch.int32, device=dev) if status is None else status
+        ws_bytes = B.reflex_moe_workspace_size(self.dtype, T, self.d, self.E,
+                                               self.inter, self.shared_inter,
+                                               self.k_max)
+        B.reflex_step(state["conf1"], state["conf2"], state["hist_len"], state["masked"],
+                      state["block_id"], state["seq_offsets"], state["active_block"],
+                      nseq, params, k_out, k_sum, status, self.dtype, hidden,
+                      self.w["w_router"], self.w["w_gate_up"], self.w["w_down"],
+                      self.w.get("shared_gate_up"), self.w.get("shared_down"),
+                      self.shared_inter, T, self.d, self.E, self.inter, self.k_max,
+                      flags, self.ws, ws_bytes, out, self.rec, stream, check)
+        self._T = T
+        return out, k_out, k_sum, status
+
     def status(self, stream=None) -> int:
         return B.reflex_moe_status(self.ws, stream)
 

@@ -103,17 +103,17 @@ __device__ __forceinline__ int clip(int k, int lo, int hi) {
   return k < lo ? lo : (k > hi ? hi : k);
 }
 
-__global__ void __launch_bounds__(kThreads)
-    budget_kernel(const float* __restrict__ conf1,
-                  const float* __restrict__ conf2,
-                  const uint8_t* __restrict__ hist_len,
-                  const uint8_t* __restrict__ masked,
-                  const int32_t* __restrict__ block_id,
-                  const int32_t* __restrict__ seq_off,
-                  const int32_t* __restrict__ active_block, int T, AllocArgs a,
-                  int32_t* __restrict__ k_out,
-                  unsigned long long* __restrict__ k_sum,
-                  uint32_t* __restrict__ err) {
+__device__ __forceinline__ void budget_body(const float* __restrict__ conf1,
+                                            const float* __restrict__ conf2,
+                                            const uint8_t* __restrict__ hist_len,
+                                            const uint8_t* __restrict__ masked,
+                                            const int32_t* __restrict__ block_id,
+                                            const int32_t* __restrict__ seq_off,
+                                            const int32_t* __restrict__ active_block,
+                                            int T, const AllocArgs& a,
+                                            int32_t* __restrict__ k_out,
+                                            unsigned long long* __restrict__ k_sum,
+                                            uint32_t* __restrict__ err) {
   // J_h scores and positions; the role shuffle reuses the same 32 KB as
   // kMaxJ 64-bit sort words
   __shared__ __align__(16) uint64_t s_raw[kMaxJ];
@@ -122,8 +122,6 @@ __global__ void __launch_bounds__(kThreads)
   __shared__ int s_nj;
   __shared__ unsigned long long s_sum;
   __shared__ uint32_t s_err;
-  grid_dep_wait();
-  grid_dep_launch();
   // With one sequence (one CTA) the sum and the error word are stored
   // outright at the end, so the caller needs no clearing; with several,
   // the host clears them and each CTA adds its share.
@@ -266,6 +264,25 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
+// defer = 0: waits for the previous kernel before reading anything.
+// defer = 1: launched right behind a kernel that writes none of its inputs
+// (the router scores of the same forward); it runs alongside that kernel and
+// waits for it only before exiting, so that its own completion still implies
+// the completion of everything before it in the stream.
+__global__ void __launch_bounds__(kThreads)
+    budget_kernel(const float* __restrict__ conf1, const float* __restrict__ conf2,
+                  const uint8_t* __restrict__ hist_len, const uint8_t* __restrict__ masked,
+                  const int32_t* __restrict__ block_id, const int32_t* __restrict__ seq_off,
+                  const int32_t* __restrict__ active_block, int T, AllocArgs a,
+                  int32_t* __restrict__ k_out, unsigned long long* __restrict__ k_sum,
+                  uint32_t* __restrict__ err, int defer) {
+  if (!defer) grid_dep_wait();
+  grid_dep_launch();
+  budget_body(conf1, conf2, hist_len, masked, block_id, seq_off, active_block, T, a, k_out,
+              k_sum, err);
+  if (defer) grid_dep_wait();
+}
+
 __global__ void wait_selftest_kernel(uint32_t* err, uint64_t limit_ns) {
   __shared__ __align__(8) uint64_t bar;
   if (threadIdx.x == 0) {
@@ -288,15 +305,17 @@ cudaError_t launch_budget(const float* conf1, const float* conf2,
                           const int32_t* active_block, int T, int B,
                           const AllocArgs& a, int32_t* k_out,
                           unsigned long long* k_sum, uint32_t* err,
-                          cudaStream_t stream) {
+                          cudaStream_t stream, bool alongside) {
   if (B <= 0) return cudaSuccess;
-  if (B == 1)  // nothing to clear first: programmatic launch after the previous kernel
-    return launch_pdl(budget_kernel, dim3(1), dim3(kThreads), 0, stream, conf1, conf2,
+  // programmatic launch when nothing is cleared right before it: a single
+  // sequence, or alongside the router scores (the caller cleared first)
+  if (B == 1 || alongside)
+    return launch_pdl(budget_kernel, dim3(B), dim3(kThreads), 0, stream, conf1, conf2,
                       hist_len, masked, block_id, seq_off, active_block, T, a, k_out,
-                      k_sum, err);
+                      k_sum, err, alongside ? 1 : 0);
   budget_kernel<<<B, kThreads, 0, stream>>>(conf1, conf2, hist_len, masked,
                                             block_id, seq_off, active_block, T, a,
-                                            k_out, k_sum, err);
+                                            k_out, k_sum, err, 0);
   return cudaGetLastError();
 }
 

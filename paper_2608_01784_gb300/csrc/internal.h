@@ -18,13 +18,17 @@ struct AllocArgs {
 };
 
 // ---- allocation (budget.cu) -----------------------------------------------
+// alongside: launched right after a kernel that writes none of the inputs
+// (the router scores of the same forward), with err / k_sum already cleared
+// when B > 1; the counts then run next to that kernel, and the budget grid
+// still completes only after it.
 cudaError_t launch_budget(const float* conf1, const float* conf2,
                           const uint8_t* hist_len, const uint8_t* masked,
                           const int32_t* block_id, const int32_t* seq_off,
                           const int32_t* active_block, int T, int B,
                           const AllocArgs& a, int32_t* k_out,
                           unsigned long long* k_sum, uint32_t* err,
-                          cudaStream_t stream);
+                          cudaStream_t stream, bool alongside = false);
 cudaError_t launch_wait_selftest(uint32_t* err, uint64_t limit_ns,
                                  cudaStream_t stream);
 

@@ -129,6 +129,65 @@ int map_err_bits(uint32_t bits) {
     if ((x) != cudaSuccess) return REFLEX_ECUDA;    \
   } while (0)
 
+// Argument checks of the allocation (reflex_allocate, reflex_step).
+int check_alloc(const float* c1, const float* c2, const uint8_t* hl, const uint8_t* m,
+                const int32_t* bid, const int32_t* so, const int32_t* act, int32_t T,
+                int32_t B, const reflex_alloc_params* p, const int32_t* k_out) {
+  if (p == nullptr || T < 0 || B < 1) return REFLEX_EINVAL;
+  if (T > 0 && (c1 == nullptr || c2 == nullptr || hl == nullptr || m == nullptr ||
+                bid == nullptr || k_out == nullptr))
+    return REFLEX_EINVAL;
+  if (so == nullptr || act == nullptr) return REFLEX_EINVAL;
+  if (p->k_min < 1 || p->k_min > p->k_max || p->k_base < 1 ||
+      p->delta_role < 0 || p->delta_cur < 0)
+    return REFLEX_EINVAL;
+  if (!(p->q > 0.0f && p->q <= 0.5f) || !(p->w_cf > 0.0f) || !(p->tau > 0.0f))
+    return REFLEX_EINVAL;
+  if (p->signal < REFLEX_SIGNAL_FPS || p->signal > REFLEX_SIGNAL_UNCERTAINTY ||
+      (p->role_shuffle != 0 && p->role_shuffle != 1))
+    return REFLEX_EINVAL;
+  return REFLEX_OK;
+}
+
+// One allocation to run inside reflex_step.
+struct AllocCall {
+  const float* c1;
+  const float* c2;
+  const uint8_t* hl;
+  const uint8_t* m;
+  const int32_t* bid;
+  const int32_t* so;
+  const int32_t* act;
+  int32_t B;
+  rx::AllocArgs a;
+  int32_t* k_out;
+  unsigned long long* k_sum;
+  uint32_t* err;
+};
+
+rx::AllocArgs alloc_args(const reflex_alloc_params* p) {
+  return rx::AllocArgs{p->k_min, p->k_base,  p->k_max, p->delta_role, p->delta_cur,
+                       p->q,     p->theta,   p->w_cf,  p->v_ref,      p->tau,
+                       p->signal, p->role_shuffle, p->shuffle_seed};
+}
+
+// The error word and the pair sum are stored outright by a single-sequence
+// count kernel; with several sequences each CTA adds its share to cleared words.
+cudaError_t clear_alloc_outputs(const AllocCall& c, cudaStream_t s) {
+  if (c.B <= 1) return cudaSuccess;
+  if (c.err) {
+    const cudaError_t e = cudaMemsetAsync(c.err, 0, sizeof(int32_t), s);
+    if (e != cudaSuccess) return e;
+  }
+  if (c.k_sum) return cudaMemsetAsync(c.k_sum, 0, sizeof(int64_t), s);
+  return cudaSuccess;
+}
+
+cudaError_t launch_alloc(const AllocCall& c, int32_t T, cudaStream_t s, bool alongside) {
+  return rx::launch_budget(c.c1, c.c2, c.hl, c.m, c.bid, c.so, c.act, T, c.B, c.a, c.k_out,
+                           c.k_sum, c.err, s, alongside);
+}
+
 }  // namespace
 
 extern "C" {
@@ -175,33 +234,16 @@ int reflex_allocate(const float* router_scores, const float* conf_prev1,
                     int64_t* k_sum_out, int32_t* dev_status, void* stream) {
   (void)router_scores;  // the REFLEX count rule does not read router scores
   (void)E;
-  if (p == nullptr || T < 0 || B < 1) return REFLEX_EINVAL;
-  if (T > 0 && (conf_prev1 == nullptr || conf_prev2 == nullptr ||
-                hist_len == nullptr || masked == nullptr ||
-                block_id == nullptr || k_out == nullptr))
-    return REFLEX_EINVAL;
-  if (seq_offsets == nullptr || active_block == nullptr) return REFLEX_EINVAL;
-  if (p->k_min < 1 || p->k_min > p->k_max || p->k_base < 1 ||
-      p->delta_role < 0 || p->delta_cur < 0)
-    return REFLEX_EINVAL;
-  if (!(p->q > 0.0f && p->q <= 0.5f) || !(p->w_cf > 0.0f) || !(p->tau > 0.0f))
-    return REFLEX_EINVAL;
-  if (p->signal < REFLEX_SIGNAL_FPS || p->signal > REFLEX_SIGNAL_UNCERTAINTY ||
-      (p->role_shuffle != 0 && p->role_shuffle != 1))
-    return REFLEX_EINVAL;
+  const int chk = check_alloc(conf_prev1, conf_prev2, hist_len, masked, block_id,
+                              seq_offsets, active_block, T, B, p, k_out);
+  if (chk != REFLEX_OK) return chk;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  uint32_t* err = reinterpret_cast<uint32_t*>(dev_status);
-  if (B > 1) {  // a single-sequence call stores both from its one CTA
-    if (err) RX_CUDA(cudaMemsetAsync(err, 0, sizeof(int32_t), s));
-    if (k_sum_out) RX_CUDA(cudaMemsetAsync(k_sum_out, 0, sizeof(int64_t), s));
-  }
-  rx::AllocArgs a{p->k_min, p->k_base,  p->k_max, p->delta_role, p->delta_cur,
-                  p->q,     p->theta,   p->w_cf,  p->v_ref,      p->tau,
-                  p->signal, p->role_shuffle, p->shuffle_seed};
-  RX_CUDA(rx::launch_budget(conf_prev1, conf_prev2, hist_len, masked, block_id,
-                            seq_offsets, active_block, T, B, a, k_out,
-                            reinterpret_cast<unsigned long long*>(k_sum_out),
-                            err, s));
+  const AllocCall c{conf_prev1, conf_prev2, hist_len, masked, block_id, seq_offsets,
+                    active_block, B, alloc_args(p), k_out,
+                    reinterpret_cast<unsigned long long*>(k_sum_out),
+                    reinterpret_cast<uint32_t*>(dev_status)};
+  RX_CUDA(clear_alloc_outputs(c, s));
+  RX_CUDA(launch_alloc(c, T, s, false));
   return REFLEX_OK;
 }
 
@@ -232,13 +274,17 @@ size_t reflex_moe_workspace_size(int32_t dtype, int32_t T, int32_t d,
   return make_layout(dtype, T, d, E, inter, shared_inter, k_max).total;
 }
 
-int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
-                       const void* w_gate_up, const void* w_down,
-                       const void* shared_gate_up, const void* shared_down,
-                       int32_t shared_inter, const int32_t* k, int32_t T,
-                       int32_t d, int32_t E, int32_t inter, int32_t k_max,
-                       uint32_t flags, void* workspace, size_t ws_bytes,
-                       void* out, reflex_route_record* rec, void* stream) {
+// The forward; with `ac`, the allocation of its counts too (k = ac->k_out):
+// cleared outputs first, then the count kernel right behind the router
+// scores, which it does not read, so the two run side by side.
+static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
+                        const void* w_gate_up, const void* w_down,
+                        const void* shared_gate_up, const void* shared_down,
+                        int32_t shared_inter, const int32_t* k, int32_t T,
+                        int32_t d, int32_t E, int32_t inter, int32_t k_max,
+                        uint32_t flags, void* workspace, size_t ws_bytes,
+                        void* out, reflex_route_record* rec, void* stream,
+                        const AllocCall* ac) {
   if (!shapes_ok(dtype, T, d, E, inter, shared_inter, k_max)) return REFLEX_EINVAL;
   if (shared_inter > 0 && (shared_gate_up == nullptr || shared_down == nullptr))
     return REFLEX_EINVAL;
@@ -261,7 +307,14 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
     rec->totals = totals;
     rec->scores = reinterpret_cast<float*>(ws + L.z);
   }
-  if (T == 0) return REFLEX_OK;
+  if (T == 0) {
+    if (ac != nullptr) {
+      cudaStream_t s0 = static_cast<cudaStream_t>(stream);
+      RX_CUDA(clear_alloc_outputs(*ac, s0));
+      RX_CUDA(launch_alloc(*ac, 0, s0, false));
+    }
+    return REFLEX_OK;
+  }
   if (hidden == nullptr || w_router == nullptr || w_gate_up == nullptr ||
       w_down == nullptr || k == nullptr || out == nullptr)
     return REFLEX_EINVAL;
@@ -303,15 +356,19 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
   void* ash = shared_inter ? ws + L.ash : nullptr;
   void* ysh = shared_inter ? ws + L.ysh : nullptr;
 
+  if (ac != nullptr) RX_CUDA(clear_alloc_outputs(*ac, s));
   if (stages & REFLEX_STAGE_ROUTE) {
     // the router's first CTA clears the header (error word, totals): no
     // kernel before the router reads it
     RX_CUDA(rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z,
                                      reinterpret_cast<uint32_t*>(hdr),
                                      static_cast<int>(sizeof(WsHeader) / 4), err, sms, s));
+    if (ac != nullptr) RX_CUDA(launch_alloc(*ac, T, s, true));
     RX_CUDA(rx::launch_router_select(z, k, T, E, k_max,
                                      (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
                                      I32(L.ids), alpha, err, s));
+  } else if (ac != nullptr) {
+    RX_CUDA(launch_alloc(*ac, T, s, false));
   }
   if (stages & REFLEX_STAGE_DISPATCH) {
     rx::DispatchBufs b{I32(L.blk_count), I32(L.blk_off),   I32(L.counts),
@@ -400,6 +457,40 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
                                k_max, cap, out, err, sms, s));
   }
   return REFLEX_OK;
+}
+
+int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
+                       const void* w_gate_up, const void* w_down,
+                       const void* shared_gate_up, const void* shared_down,
+                       int32_t shared_inter, const int32_t* k, int32_t T,
+                       int32_t d, int32_t E, int32_t inter, int32_t k_max,
+                       uint32_t flags, void* workspace, size_t ws_bytes,
+                       void* out, reflex_route_record* rec, void* stream) {
+  return forward_impl(dtype, hidden, w_router, w_gate_up, w_down, shared_gate_up,
+                      shared_down, shared_inter, k, T, d, E, inter, k_max, flags,
+                      workspace, ws_bytes, out, rec, stream, nullptr);
+}
+
+int reflex_step(const float* conf_prev1, const float* conf_prev2, const uint8_t* hist_len,
+                const uint8_t* masked, const int32_t* block_id, const int32_t* seq_offsets,
+                const int32_t* active_block, int32_t B, const reflex_alloc_params* p,
+                int32_t* k_out, int64_t* k_sum_out, int32_t* alloc_status,
+                int32_t dtype, const void* hidden, const void* w_router,
+                const void* w_gate_up, const void* w_down, const void* shared_gate_up,
+                const void* shared_down, int32_t shared_inter, int32_t T, int32_t d,
+                int32_t E, int32_t inter, int32_t k_max, uint32_t flags, void* workspace,
+                size_t ws_bytes, void* out, reflex_route_record* rec, void* stream) {
+  const int chk = check_alloc(conf_prev1, conf_prev2, hist_len, masked, block_id,
+                              seq_offsets, active_block, T, B, p, k_out);
+  if (chk != REFLEX_OK) return chk;
+  if (T > 0 && k_out == nullptr) return REFLEX_EINVAL;
+  const AllocCall c{conf_prev1, conf_prev2, hist_len, masked, block_id, seq_offsets,
+                    active_block, B, alloc_args(p), k_out,
+                    reinterpret_cast<unsigned long long*>(k_sum_out),
+                    reinterpret_cast<uint32_t*>(alloc_status)};
+  return forward_impl(dtype, hidden, w_router, w_gate_up, w_down, shared_gate_up,
+                      shared_down, shared_inter, k_out, T, d, E, inter, k_max, flags,
+                      workspace, ws_bytes, out, rec, stream, &c);
 }
 
 int reflex_read_status(const int32_t* dev_status, void* stream) {

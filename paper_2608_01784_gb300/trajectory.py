@@ -114,13 +114,15 @@ def simulate(state: dict, params: B.reflex_alloc_params, E: int, *, theta_commit
         out = torch.empty((T, moe.d), dtype=moe.tdtype, device=dev)
     def forward(t):
         running = (state["active_block"] <= nb).to(torch.int64)
-        api.allocate(state, params, E, None, k, ksum, status)
+        if moe is not None:   # counts and the first layer in one call
+            moe.step(state, params, hidden, out=out, k_out=k, k_sum=ksum, status=status)
+            for _ in range(layers - 1):
+                moe.forward(hidden, k, out)
+        else:
+            api.allocate(state, params, E, None, k, ksum, status)
         nfe.add_(running)
         pairs.add_(torch.zeros(Bn, dtype=torch.int64, device=dev).index_add_(
             0, sidx, k.to(torch.int64)) * running)
-        if moe is not None:
-            for _ in range(layers):
-                moe.forward(hidden, k, out)
         conf = synthetic_confidence(state, t, seed, sidx)
         api.update_state(state, conf, nb, theta_commit, committed=committed, status=upd_status)
 

@@ -129,3 +129,25 @@ def test_update_state_host_rejections(lib):
                                    4, 1, 0.9, None, None, None) == B.REFLEX_EINVAL
     assert lib.reflex_update_state(1, 1, 1, 1, 1, 1, 1, 1, 1, 4, 1, float("nan"),
                                    None, None, None) == B.REFLEX_EINVAL
+
+
+def test_step_host_rejections(lib):
+    # reflex_step checks both halves before it launches anything
+    import ctypes
+    from paper_2608_01784_gb300 import _binding as B
+    p = B.reflex_alloc_params()
+    lib.reflex_default_params(ctypes.byref(p))
+    state = (1, 1, 1, 1, 1, 1, 1)          # dummy device pointers, never read
+
+    def step(B_=1, params=ctypes.byref(p), T=4, d=256, ws=1 << 30, k_out=1, q=None):
+        return lib.reflex_step(*state, B_, params, k_out, None, None, 1, 1, 1, 1, 1,
+                               None, None, 0, T, d, 8, 128, 4, 1, 256, ws, 1, None, None)
+    assert step(params=None) == B.REFLEX_EINVAL          # no allocation parameters
+    assert step(B_=0) == B.REFLEX_EINVAL                 # no sequence
+    assert step(k_out=None) == B.REFLEX_EINVAL           # nowhere to put the counts
+    assert step(d=100) == B.REFLEX_EINVAL                # forward shape rule
+    assert step(ws=16) == B.REFLEX_EWORKSPACE            # workspace too small
+    bad = B.reflex_alloc_params()
+    lib.reflex_default_params(ctypes.byref(bad))
+    bad.q = 0.75                                         # q outside (0, 1/2]
+    assert step(params=ctypes.byref(bad)) == B.REFLEX_EINVAL
