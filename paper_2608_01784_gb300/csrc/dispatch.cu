@@ -105,10 +105,18 @@ __global__ void __launch_bounds__(1024)
   const int e = threadIdx.x;  // E <= 1024
   int run = 0;
   if (e < E) {
-    for (int b = 0; b < nblk; ++b) {
-      const int64_t o = static_cast<int64_t>(b) * E + e;
-      blk_off[o] = run;
-      run += blk_count[o];
+    // eight loads in flight per thread, then their prefix
+    constexpr int kBatch = 8;
+    for (int b0 = 0; b0 < nblk; b0 += kBatch) {
+      int c[kBatch];
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u)
+        c[u] = b0 + u < nblk ? blk_count[static_cast<int64_t>(b0 + u) * E + e] : 0;
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u) {
+        if (b0 + u < nblk) blk_off[static_cast<int64_t>(b0 + u) * E + e] = run;
+        run += c[u];
+      }
     }
     counts[e] = run;
   }
