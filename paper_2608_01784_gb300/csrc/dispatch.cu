@@ -3,7 +3,8 @@
 // out grouped by expert and, within an expert, in token order, so that each
 // expert's rows form one contiguous range of a grouped GEMM.
 //
-// Three launches, no atomics whose order matters:
+// Three launches (two for short batches, whose count and scan share one
+// CTA), no atomics whose order matters:
 //   count   per block of 256 tokens, a bitmask per expert in shared memory
 //           (bit = token of the block selected the expert; a token selects
 //           an expert at most once) and its popcount per expert;
@@ -142,6 +143,66 @@ __global__ void __launch_bounds__(1024)
   }
 }
 
+// Short batches: the count and scan steps in one CTA.  Every pair adds one
+// to its (32-token block, expert) counter in shared memory (integer sums, so
+// the order of the additions does not matter); then, per expert, the block
+// prefixes and the total, and the expert and tile prefixes as in scan_kernel.
+// The block counts never leave shared memory.
+__global__ void __launch_bounds__(1024)
+    count_scan_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ k,
+                      int T, int E, int k_max, int nblk, int32_t* __restrict__ blk_off,
+                      int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
+                      int32_t* __restrict__ mt_prefix, int32_t* __restrict__ mt2_prefix,
+                      int32_t* __restrict__ totals, uint32_t* __restrict__ err) {
+  extern __shared__ int s_cnt[];  // [nblk][E]
+  __shared__ int s_warp[32];
+  grid_dep_wait();
+  grid_dep_launch();
+  for (int i = threadIdx.x; i < nblk * E; i += 1024) s_cnt[i] = 0;
+  __syncthreads();
+  const int kcap = k_max < E ? k_max : E;
+  for (int t = threadIdx.x; t < T; t += 1024) {
+    const int kt = clamp_k(k[t], kcap);
+    int* row = s_cnt + (t / kDispatchBlockSmall) * E;
+    for (int j = 0; j < kt; ++j) {
+      const int e = ids[static_cast<int64_t>(t) * k_max + j];
+      if (e >= 0 && e < E)
+        atomicAdd(&row[e], 1);
+      else
+        set_err(err, kErrIndex);
+    }
+  }
+  __syncthreads();
+  const int e = threadIdx.x;  // E <= 1024
+  int run = 0;
+  if (e < E) {
+    for (int b = 0; b < nblk; ++b) {
+      blk_off[static_cast<int64_t>(b) * E + e] = run;
+      run += s_cnt[b * E + e];
+    }
+    counts[e] = run;
+  }
+  int total_pairs, total_tiles, total_tiles2;
+  const int off = block_exclusive_scan(e < E ? run : 0, s_warp, &total_pairs);
+  const int tiles = e < E ? (run + kTileM - 1) / kTileM : 0;
+  const int toff = block_exclusive_scan(tiles, s_warp, &total_tiles);
+  const int tiles2 = e < E ? (run + 2 * kTileM - 1) / (2 * kTileM) : 0;
+  const int toff2 = block_exclusive_scan(tiles2, s_warp, &total_tiles2);
+  if (e < E) {
+    offsets[e] = off;
+    mt_prefix[e] = toff;
+    mt2_prefix[e] = toff2;
+  }
+  if (e == 0) {
+    offsets[E] = total_pairs;
+    mt_prefix[E] = total_tiles;
+    mt2_prefix[E] = total_tiles2;
+    totals[0] = total_pairs;
+    totals[1] = total_tiles;
+    totals[2] = total_tiles2;
+  }
+}
+
 template <int BLK>
 __global__ void __launch_bounds__(BLK)
     scatter_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ k,
@@ -248,10 +309,42 @@ cudaError_t launch_dispatch_blk(const int32_t* ids, const int32_t* k, int T, int
                     k_max, b.blk_off, b.offsets, b.perm, b.row_of, b.err);
 }
 
+// Short batches whose block counts fit in shared memory: count + scan in one
+// CTA, then the scatter.
+constexpr size_t kCountScanSmem = 160 * 1024;
+
+static cudaError_t launch_dispatch_small(const int32_t* ids, const int32_t* k, int T, int E,
+                                  int k_max, const DispatchBufs& b, cudaStream_t stream) {
+  constexpr int BLK = kDispatchBlockSmall;
+  const int nblk = (T + BLK - 1) / BLK;
+  const size_t cs_smem = static_cast<size_t>(nblk) * E * sizeof(int);
+  if (cs_smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(
+        count_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cs_smem);
+    if (e != cudaSuccess) return e;
+  }
+  cudaError_t e = launch_pdl(count_scan_kernel, dim3(1), dim3(1024), cs_smem, stream, ids, k,
+                             T, E, k_max, nblk, b.blk_off, b.counts, b.offsets, b.mt_prefix,
+                             b.mt2_prefix, b.totals, b.err);
+  if (e != cudaSuccess) return e;
+  const size_t smem = static_cast<size_t>(E) * (BLK / 32) * sizeof(uint32_t);
+  if (smem > 48 * 1024) {
+    e = cudaFuncSetAttribute(scatter_kernel<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  return launch_pdl(scatter_kernel<BLK>, dim3(nblk), dim3(BLK), smem, stream, ids, k, T, E,
+                    k_max, b.blk_off, b.offsets, b.perm, b.row_of, b.err);
+}
+
 cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T, int E,
                             int k_max, const DispatchBufs& b,
                             cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
+  if (dispatch_block(T) == kDispatchBlockSmall &&
+      static_cast<size_t>((T + kDispatchBlockSmall - 1) / kDispatchBlockSmall) * E *
+              sizeof(int) <= kCountScanSmem)
+    return launch_dispatch_small(ids, k, T, E, k_max, b, stream);
   if (dispatch_block(T) == kDispatchBlockSmall)
     return launch_dispatch_blk<kDispatchBlockSmall>(ids, k, T, E, k_max, b, stream);
   return launch_dispatch_blk<kDispatchBlock>(ids, k, T, E, k_max, b, stream);
