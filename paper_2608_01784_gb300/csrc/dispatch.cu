@@ -237,15 +237,16 @@ __global__ void __launch_bounds__(BLK)
   }
 }
 
-// Token-order gather: one warp per token reads the token's hidden row once
-// (up to 8 16-byte vectors per lane in flight) and writes it to each of the
-// token's k_t pair rows, so every hidden row crosses HBM once however many
-// experts selected it.
+// Token-order gather: W warps per token (W = 1 for long batches), each
+// reading one 1/W segment of the token's hidden row once (up to 8 16-byte
+// vectors per lane in flight) and writing it to each of the token's k_t pair
+// rows, so every hidden row crosses HBM once however many experts selected
+// it.  Short batches split rows across warps so that every SM gets work.
 template <typename Te>
 __global__ void __launch_bounds__(256)
     gather_kernel(const Te* __restrict__ x, const int32_t* __restrict__ row_of,
                   const int32_t* __restrict__ k, int k_max, int cap_rows, int T,
-                  int d, Te* __restrict__ xp, uint32_t* __restrict__ err) {
+                  int d, int wpt, Te* __restrict__ xp, uint32_t* __restrict__ err) {
   constexpr int kVecElems = 16 / sizeof(Te);  // elements per 16-byte vector
   constexpr int kMaxVec = 8;                  // vectors per lane per pass
   grid_dep_wait();
@@ -253,7 +254,11 @@ __global__ void __launch_bounds__(256)
   const int lane = threadIdx.x & 31;
   const int warps = gridDim.x * 8;
   const int row_vecs = d / kVecElems;
-  for (int t = blockIdx.x * 8 + (threadIdx.x >> 5); t < T; t += warps) {
+  const int seg_vecs = row_vecs / wpt;        // vectors of one warp's segment
+  const int units = T * wpt;
+  for (int u = blockIdx.x * 8 + (threadIdx.x >> 5); u < units; u += warps) {
+    const int t = u / wpt;
+    const int v0 = (u % wpt) * seg_vecs;
     int kt = k[t];
     kt = kt < 1 ? 1 : (kt > k_max ? k_max : kt);
     int my_row = -1;
@@ -264,22 +269,22 @@ __global__ void __launch_bounds__(256)
         my_row = -1;
       }
     }
-    const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(t) * d);
-    for (int base = 0; base < row_vecs; base += 32 * kMaxVec) {
+    const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(t) * d) + v0;
+    for (int base = 0; base < seg_vecs; base += 32 * kMaxVec) {
       uint4 v[kMaxVec];
 #pragma unroll
       for (int i = 0; i < kMaxVec; ++i) {
         const int q = base + lane + 32 * i;
-        if (q < row_vecs) v[i] = __ldg(src + q);
+        if (q < seg_vecs) v[i] = __ldg(src + q);
       }
       for (int j = 0; j < kt; ++j) {
         const int r = __shfl_sync(0xffffffffu, my_row, j);
         if (r < 0) continue;
-        uint4* dst = reinterpret_cast<uint4*>(xp + static_cast<int64_t>(r) * d);
+        uint4* dst = reinterpret_cast<uint4*>(xp + static_cast<int64_t>(r) * d) + v0;
 #pragma unroll
         for (int i = 0; i < kMaxVec; ++i) {
           const int q = base + lane + 32 * i;
-          if (q < row_vecs) dst[q] = v[i];
+          if (q < seg_vecs) dst[q] = v[i];
         }
       }
     }
@@ -355,15 +360,22 @@ cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* row
                                int d, void* x_perm, uint32_t* err, int num_sms,
                                cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
-  int grid = (T + 7) / 8;
+  // warps per token: enough warps for 16 per SM, each segment whole vectors
+  const int row_vecs = d * (dtype == 0 ? 4 : 2) / 16;
+  int wpt = 1;
+  while (wpt < 8 && static_cast<int64_t>(T) * wpt < 16LL * num_sms &&
+         row_vecs % (2 * wpt) == 0)
+    wpt *= 2;
+  const int64_t warps = static_cast<int64_t>(T) * wpt;
+  int grid = static_cast<int>((warps + 7) / 8);
   if (grid > 16 * num_sms) grid = 16 * num_sms;
   if (dtype == 0)
     return launch_pdl(gather_kernel<float>, dim3(grid), dim3(256), 0, stream,
                       static_cast<const float*>(hidden), row_of, k, k_max, cap_rows, T, d,
-                      static_cast<float*>(x_perm), err);
+                      wpt, static_cast<float*>(x_perm), err);
   return launch_pdl(gather_kernel<__nv_bfloat16>, dim3(grid), dim3(256), 0, stream,
                     static_cast<const __nv_bfloat16*>(hidden), row_of, k, k_max, cap_rows, T,
-                    d, static_cast<__nv_bfloat16*>(x_perm), err);
+                    d, wpt, static_cast<__nv_bfloat16*>(x_perm), err);
 }
 
 }  // namespace rx
