@@ -64,6 +64,13 @@ extern "C" {
 /* Residual connection for stacked layers: out = hidden + MoE(hidden), summed
  * in fp32 with the expert outputs and rounded once. */
 #define REFLEX_FLAG_RESIDUAL 0x4u
+/* bf16: compute every router score with the canonical fma chain.  Without
+ * it (and with REFLEX_FLAG_RENORM_TOPK) the scores come from a tensor-core
+ * GEMM and only the experts that could be selected are recomputed with the
+ * chain: the selected experts, their weights and their scores are the same
+ * bits either way (the screen's bound is stated with reflex_moe_forward);
+ * only the record's other scores differ (tensor-core estimates). */
+#define REFLEX_FLAG_EXACT_SCORES 0x8u
 /* Stage selection.  No stage bit = all five stages in order.  Stages read
  * what the previous stages left in the same workspace; running a stage whose
  * predecessors did not run on that workspace gives unspecified values (every
@@ -211,8 +218,11 @@ typedef struct {
                          (expert, token)                                    */
     int32_t* row_of;  /* [T, k_max] pair row of (token, slot), -1 unused    */
     int32_t* totals;  /* [2] device: sum k (pairs), number of 128-row tiles */
-    float* scores;    /* [T, E] router scores r_i (fp32, the fma chain of
-                         reflex_moe_forward); valid after the ROUTE stage   */
+    float* scores;    /* [T, E] router scores r_i (fp32), valid after the
+                         ROUTE stage: the fma chain of reflex_moe_forward for
+                         every expert that could be selected (all experts
+                         with REFLEX_FLAG_EXACT_SCORES or fp32), tensor-core
+                         estimates for the others                           */
 } reflex_route_record;
 
 /* Bytes of workspace reflex_moe_forward needs for these shapes (0 if the
@@ -229,6 +239,15 @@ size_t reflex_moe_workspace_size(int32_t dtype, int32_t T, int32_t d,
  * multiply-add chain over the hidden index from +0), TopK ties broken to the
  * lower expert index, and SwiGLU experts
  *   E_e(h) = (silu(h W_g,e^T) * (h W_u,e^T)) W_d,e^T.
+ * The TopK is decided on the canonical chain's scores.  bf16 layers with
+ * renormalised weights screen first: tensor-core scores z~ with an interval
+ * z~ -/+ (gamma_d + 2^-12 + (s+1) 2^-24) ||h_i|| ||w_e|| (gamma_d = d u /
+ * (1 - d u), u = 2^-24, s split-K slices) that holds both the chain's score
+ * and the exact product; experts whose interval lies below the k_i-th
+ * largest lower end cannot be selected, all others are recomputed with the
+ * chain.  This assumes the tensor cores' fp32 accumulation errs by at most
+ * 2^-12 sum_k |h_k w_k|; REFLEX_FLAG_EXACT_SCORES computes every score with
+ * the chain instead.
  *
  *   dtype           REFLEX_DTYPE_F32 or REFLEX_DTYPE_BF16 (all float arrays).
  *   hidden          [T, d]

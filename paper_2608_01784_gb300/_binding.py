@@ -27,6 +27,7 @@ REFLEX_DTYPE_BF16 = 1
 REFLEX_FLAG_RENORM_TOPK = 0x1
 REFLEX_FLAG_SIMT_EXPERTS = 0x2
 REFLEX_FLAG_RESIDUAL = 0x4
+REFLEX_FLAG_EXACT_SCORES = 0x8
 REFLEX_SIGNAL_FPS = 0
 REFLEX_SIGNAL_FRONTIER = 1
 REFLEX_SIGNAL_PROGRESS = 2

@@ -46,7 +46,7 @@ constexpr int kRingBytes = 192 * 1024;  // TMA ring budget per CTA
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr uint64_t kDrainNs = 1000000000ull;
 
-enum { kModeSwiGLU = 0, kModeDown = 1 };
+enum { kModeSwiGLU = 0, kModeDown = 1, kModeScores = 2 };
 
 template <int BN>
 struct Cfg {
@@ -72,6 +72,15 @@ struct KParams {
   __nv_bfloat16* out;
   int ldo;
   uint32_t* err;
+  // scores mode (dense, fp32 out): K is cut into k_splits slices; slice ks of
+  // tile (m, n) writes out_f32 + ks * split_stride; columns >= n_valid dropped
+  int k_splits;
+  float* out_f32;
+  int64_t split_stride;
+  int n_valid;
+  // 1: launched right behind a kernel that writes none of this kernel's
+  // inputs or outputs; start at once and wait for it only before exiting
+  int defer_wait;
 };
 
 // ---- PTX wrappers ---------------------------------------------------------
@@ -188,12 +197,13 @@ __device__ __forceinline__ void tmem_ld_wait() {
 struct Tile {
   int e, n, row0, rows;
   int mtiles;  // m-tiles of the tile's group (readers of each weight tile)
+  int ks;      // K slice (scores mode; 0 otherwise)
 };
 
 __device__ __forceinline__ int total_tiles(const KParams& p) {
   int mt;
   if (p.g.offsets == nullptr) {
-    mt = (p.g.dense_rows + p.tile_rows - 1) / p.tile_rows;
+    mt = (p.g.dense_rows + p.tile_rows - 1) / p.tile_rows * p.k_splits;
   } else {
     mt = p.mt_prefix[p.g.E];
     if (mt < 0) mt = 0;
@@ -206,13 +216,17 @@ __device__ __forceinline__ int total_tiles(const KParams& p) {
 __device__ __forceinline__ bool decode_tile(const KParams& p, int t, Tile& o) {
   if (p.g.offsets == nullptr) {
     const int mt = (p.g.dense_rows + p.tile_rows - 1) / p.tile_rows;
+    const int per = mt * p.n_tiles;
+    o.ks = t / per;
+    t -= o.ks * per;
     o.e = 0;
     o.n = t / mt;
     o.row0 = (t % mt) * p.tile_rows;
     o.rows = min(p.tile_rows, p.g.dense_rows - o.row0);
     o.mtiles = mt;
-    return true;
+    return o.ks < p.k_splits;
   }
+  o.ks = 0;
   int lo = 0, hi = p.g.E;  // n_tiles*prefix[lo] <= t < n_tiles*prefix[hi]
   while (hi - lo > 1) {
     const int mid = (lo + hi) >> 1;
@@ -274,10 +288,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  grid_dep_wait();  // the tile count and every operand come from earlier kernels
+  // the tile count and every operand come from earlier kernels
+  if (!p.defer_wait) grid_dep_wait();
   grid_dep_launch();
   const int ntiles = total_tiles(p);
-  const int nk = p.K / BK;
+  const int nk = p.K / BK / p.k_splits;  // k-blocks per tile
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer ----------------
@@ -302,7 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const uint32_t fb = smem_addr(&full[stage]);
         mbar_expect_tx(fb, C::kStageBytes);
-        const int k0 = kb * BK;
+        const int k0 = (tl.ks * nk + kb) * BK;
         tma_load_2d(smem_addr(sa + stage * C::kABytes), &map_a, k0, tl.row0, fb);
         const uint32_t b_dst = smem_addr(sb + stage * C::kBBytes);
         const int wr = tl.e * p.b_rows_per_group + tl.n * (MODE == kModeSwiGLU ? BN / 2 : BN);
@@ -405,7 +420,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool store = tile_ok && row < tl.rows;
       __nv_bfloat16* orow =
           p.out + static_cast<int64_t>(tl.row0 + (store ? row : 0)) * p.ldo;
-      if (MODE == kModeSwiGLU) {
+      if (MODE == kModeScores) {
+        float* srow = p.out_f32 + tl.ks * p.split_stride +
+                      static_cast<int64_t>(tl.row0 + (store ? row : 0)) * p.ldo;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t v32[32];
+          tmem_ld32(tbase + c, v32);
+          tmem_ld_wait();
+          const int col0 = tl.n * BN + c;
+          if (store) {
+            if (col0 + 32 <= p.n_valid && (p.ldo & 3) == 0) {
+              float4* dst = reinterpret_cast<float4*>(srow + col0);
+#pragma unroll
+              for (int v = 0; v < 8; ++v)
+                dst[v] = make_float4(__uint_as_float(v32[4 * v]), __uint_as_float(v32[4 * v + 1]),
+                                     __uint_as_float(v32[4 * v + 2]),
+                                     __uint_as_float(v32[4 * v + 3]));
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (col0 + i < p.n_valid) srow[col0 + i] = __uint_as_float(v32[i]);
+            }
+          }
+        }
+      } else if (MODE == kModeSwiGLU) {
 #pragma unroll 1
         for (int c = 0; c < BN / 2; c += 32) {
           uint32_t g[32], u[32];
@@ -465,6 +504,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
     tmem_dealloc(tmem_base, C::kTmemCols);
   }
+  if (p.defer_wait) grid_dep_wait();
 }
 
 template <int BN, int MODE>
@@ -487,6 +527,11 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.err = a.err;
   p.mt_prefix = a.g.mt_prefix;
   p.tile_rows = BM;
+  p.k_splits = 1;
+  p.out_f32 = nullptr;
+  p.split_stride = 0;
+  p.n_valid = 0;
+  p.defer_wait = 0;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);
@@ -849,6 +894,11 @@ cudaError_t launch_pair_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.out = static_cast<__nv_bfloat16*>(a.out);
   p.ldo = a.ldo;
   p.err = a.err;
+  p.k_splits = 1;
+  p.out_f32 = nullptr;
+  p.split_stride = 0;
+  p.n_valid = 0;
+  p.defer_wait = 0;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   int pairs = a.num_sms / 2;
@@ -881,9 +931,55 @@ cudaError_t launch_down_tc(const TcGemmArgs& a, int bn, cudaStream_t stream) {
   if (bn == 128) return launch_impl<128, kModeDown>(a, stream);
   return launch_impl<256, kModeDown>(a, stream);
 }
+template <int BN>
+cudaError_t launch_scores_impl(const TcGemmArgs& a, int k_splits, float* out,
+                               int64_t split_stride, int n_valid, bool defer_wait,
+                               cudaStream_t stream) {
+  using C = Cfg<BN>;
+  auto kernel = grouped_gemm_kernel<BN, kModeScores>;
+  if (a.g.offsets != nullptr || k_splits < 1 || (a.K / BK) % k_splits != 0 ||
+      a.K % BK != 0 || n_valid < 1)
+    return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(
+      kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  KParams p{};
+  p.K = a.K;
+  p.n_tiles = (n_valid + BN - 1) / BN;
+  p.b_rows_per_group = 0;
+  p.b_up_offset = 0;
+  p.g = a.g;
+  p.max_mtiles = (a.g.dense_rows + BM - 1) / BM;
+  p.out = nullptr;
+  p.ldo = a.ldo;
+  p.err = a.err;
+  p.mt_prefix = nullptr;
+  p.tile_rows = BM;
+  p.k_splits = k_splits;
+  p.out_f32 = out;
+  p.split_stride = split_stride;
+  p.n_valid = n_valid;
+  p.defer_wait = defer_wait ? 1 : 0;
+  const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles * k_splits;
+  if (max_tiles == 0) return cudaSuccess;
+  const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);
+  return launch_pdl(kernel, dim3(grid), dim3(kThreads), C::kSmemBytes, stream, *a.map_a,
+                    *a.map_b, p);
+}
+
 // SwiGLU loads gate and up halves as two boxes of bn/2 rows; down loads one
 // box of bn rows.
 int tc_b_box_rows(bool swiglu, int bn) { return swiglu ? bn / 2 : bn; }
+
+cudaError_t launch_scores_tc(const TcGemmArgs& a, int bn, int k_splits, float* out,
+                             int64_t split_stride, int n_valid, bool defer_wait,
+                             cudaStream_t stream) {
+  if (bn == 64)
+    return launch_scores_impl<64>(a, k_splits, out, split_stride, n_valid, defer_wait, stream);
+  if (bn == 128)
+    return launch_scores_impl<128>(a, k_splits, out, split_stride, n_valid, defer_wait, stream);
+  return cudaErrorInvalidValue;
+}
 
 cudaError_t launch_swiglu_tc_pair(const TcGemmArgs& a, cudaStream_t stream) {
   return launch_pair_impl<kModeSwiGLU>(a, stream);

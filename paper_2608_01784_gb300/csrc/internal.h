@@ -48,6 +48,28 @@ cudaError_t launch_router_logits(int dtype, const void* hidden,
                                  const void* w_router, int T, int d, int E,
                                  float* z, uint32_t* zero_words, int n_zero,
                                  uint32_t* err, int num_sms, cudaStream_t stream);
+// Screened routing (bf16, renormalised weights): nw[e] = ||w_e||_2 rounded up
+// (first kernel of the forward; clears zero_words like the score kernels);
+// then, from the tensor-core score slices z[s][t][e] (s < k_splits), the
+// exact TopK, alpha and ids, with the canonical chain recomputed for every
+// expert that could be selected (written back into z's first slice).
+cudaError_t launch_router_wnorm(const __nv_bfloat16* w, int E, int d, float* nw,
+                                uint32_t* zero_words, int n_zero, cudaStream_t stream);
+cudaError_t launch_router_screen_select(const __nv_bfloat16* h, const __nv_bfloat16* w,
+                                        float* z, int k_splits, int64_t split_stride,
+                                        const float* nw, const int32_t* k, int T, int E,
+                                        int d, int k_max, int32_t* ids, float* alpha,
+                                        uint32_t* err, cudaStream_t stream);
+// Tile width and K slices of the screen GEMM for T x E scores over d: slices
+// double while the tile count stays within 152 (this GPU's SM count).
+inline int screen_bn(int E) { return E <= 64 ? 64 : 128; }
+inline int screen_splits(int T, int E, int d) {
+  const int64_t mt = (T + 127) / 128, nt = (E + screen_bn(E) - 1) / screen_bn(E);
+  const int nkb = d / 64;
+  int s = 1;
+  while (s < 16 && mt * nt * s * 2 <= 152 && nkb % (2 * s) == 0) s *= 2;
+  return s;
+}
 // ids/alpha [T, k_max] from z and the counts k.
 cudaError_t launch_router_select(const float* z, const int32_t* k, int T,
                                  int E, int k_max, bool renorm, int32_t* ids,
@@ -126,6 +148,15 @@ struct TcGemmArgs {
 cudaError_t launch_swiglu_tc(const TcGemmArgs& a, int bn, cudaStream_t stream);
 cudaError_t launch_down_tc(const TcGemmArgs& a, int bn, cudaStream_t stream);
 int tc_b_box_rows(bool swiglu, int bn);
+// Router-score screen: out[ks][t][e] = sum over the ks-th of k_splits equal
+// slices of k of A[t, k] B[e, k] (fp32 accumulators, dense rows t < T =
+// a.g.dense_rows, columns e < n_valid, row stride a.ldo), bn in {64, 128}
+// (B tensor map box of bn rows); a.K / 64 must be a multiple of k_splits.
+// defer_wait: launched right behind a kernel that writes none of its inputs
+// or outputs (it then overlaps that kernel and waits for it before exiting).
+cudaError_t launch_scores_tc(const TcGemmArgs& a, int bn, int k_splits, float* out,
+                             int64_t split_stride, int n_valid, bool defer_wait,
+                             cudaStream_t stream);
 // CTA-pair (2-SM, cta_group::2) variants: 256 x 256 tiles, cluster of two
 // CTAs; A and B tensor maps both with boxes of 128 rows; needs
 // GroupRows::mt2_prefix in grouped mode.  n_total must be a multiple of 128

@@ -21,7 +21,7 @@ size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 // Byte offsets of every workspace region (all 256-byte aligned).
 struct Layout {
-  size_t hdr, z, ids, alpha, blk_count, blk_off, counts, offsets, mt_prefix,
+  size_t hdr, z, wnorm, ids, alpha, blk_count, blk_off, counts, offsets, mt_prefix,
       mt2_prefix, perm, row_of, xperm, amid, ash, ysh, total;
   int64_t cap_rows;
   int nblk;
@@ -51,7 +51,10 @@ Layout make_layout(int32_t dtype, int32_t T, int32_t d, int32_t E,
     return at;
   };
   L.hdr = take(sizeof(WsHeader));
-  L.z = take(static_cast<size_t>(T) * E * 4);
+  // bf16: room for the screen GEMM's split-K slices of the scores
+  const int zslices = dtype == REFLEX_DTYPE_F32 ? 1 : rx::screen_splits(T, E, d);
+  L.z = take(static_cast<size_t>(zslices) * T * E * 4);
+  L.wnorm = take(static_cast<size_t>(E) * 4);
   L.ids = take(cap * 4);
   L.alpha = take(cap * 4);
   L.blk_count = take(static_cast<size_t>(nblk) * E * 4);
@@ -357,7 +360,35 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
   void* ysh = shared_inter ? ws + L.ysh : nullptr;
 
   if (ac != nullptr) RX_CUDA(clear_alloc_outputs(*ac, s));
-  if (stages & REFLEX_STAGE_ROUTE) {
+  // bf16 with renormalised weights and many experts: tensor-core scores
+  // screen the experts and only those that could be selected get the
+  // canonical chain (router.cu).  The recheck costs about as much per chain
+  // as 40 chains of the dense score kernels, so it pays from 128 experts on
+  // (LLaDA2.0-mini layer, 256 experts: routing 213 -> 113 us; with 64
+  // experts the dense kernels stay faster at every batch size measured).
+  const bool screen = dtype == REFLEX_DTYPE_BF16 && (flags & REFLEX_FLAG_RENORM_TOPK) &&
+                      !(flags & REFLEX_FLAG_EXACT_SCORES) && d % 128 == 0 && E >= 128;
+  if ((stages & REFLEX_STAGE_ROUTE) && screen) {
+    const int bn = rx::screen_bn(E), ks = rx::screen_splits(T, E, d);
+    CUtensorMap mh, mw;
+    if (!make_map(&mh, hidden, T, d, rx::kTileM) || !make_map(&mw, w_router, E, d, bn))
+      return REFLEX_ECUDA;
+    float* nw = reinterpret_cast<float*>(ws + L.wnorm);
+    const int64_t zs = static_cast<int64_t>(T) * E;
+    // the first kernel clears the header (error word, totals); the score GEMM
+    // reads and writes nothing it touches, so it runs beside it, and so does
+    // the count kernel of reflex_step
+    RX_CUDA(rx::launch_router_wnorm(static_cast<const __nv_bfloat16*>(w_router), E, d, nw,
+                                    reinterpret_cast<uint32_t*>(hdr),
+                                    static_cast<int>(sizeof(WsHeader) / 4), s));
+    rx::GroupRows rows{nullptr, nullptr, nullptr, nullptr, 1, T, T};
+    rx::TcGemmArgs sa{&mh, &mw, d, E, 0, 0, rows, nullptr, E, err, sms};
+    RX_CUDA(rx::launch_scores_tc(sa, bn, ks, z, zs, E, true, s));
+    if (ac != nullptr) RX_CUDA(launch_alloc(*ac, T, s, true));
+    RX_CUDA(rx::launch_router_screen_select(
+        static_cast<const __nv_bfloat16*>(hidden), static_cast<const __nv_bfloat16*>(w_router),
+        z, ks, zs, nw, k, T, E, d, k_max, I32(L.ids), alpha, err, s));
+  } else if (stages & REFLEX_STAGE_ROUTE) {
     // the router's first CTA clears the header (error word, totals): no
     // kernel before the router reads it
     RX_CUDA(rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z,

@@ -726,6 +726,243 @@ cudaError_t launch_logits_res(const __nv_bfloat16* h, const __nv_bfloat16* w, in
   return cudaGetLastError();
 }
 
+// ---- screened selection (bf16 inputs, weights renormalised over the set) --
+// The tensor cores give every score z~[t, e] (fp32 accumulators, split-K
+// partial sums added in slice order).  Both z~ and the canonical chain z lie
+// within their error bounds of the exact dot product: for the chain (one
+// rounding per fma, d steps) |z - z*| <= gamma_d sum_k |h_k w_k| with
+// gamma_d = d u / (1 - d u), u = 2^-24; the tensor-core estimate is taken to
+// err by at most 2^-12 sum |h_k w_k| (about 4x a crude worst case of a few
+// units in the last place per 16-product step, and far above what is
+// observed), plus one rounding per split-K slice.  With sum |h_k w_k| <=
+// ||h_t|| ||w_e|| (Cauchy-Schwarz) every z lies in [lo_e, hi_e] = z~_e -/+
+// delta_e.  Let L be the k_t-th largest lo: at least k_t experts have z >= L,
+// so an expert with hi_e < L cannot be among the k_t largest; the candidates
+// C = {e : hi_e >= L} contain the canonical TopK set.  Their scores are
+// recomputed with the canonical chain (the same fma.rn.f32.bf16 sequence as
+// the score kernels), and the TopK over C (same keys, same tie rule) is the
+// TopK over all experts.  Scores of the other experts stay tensor-core
+// estimates in z.  One warp per token; a token with more than 32 candidates
+// recomputes every expert.
+constexpr int kScreenWarps = 8;
+
+// ||w_e||_2, rounded up (every step of the fp32 sum of squares is covered by
+// the factors below).
+// The first kernel of a screened forward: it also clears zero_words[0, nz).
+__global__ void __launch_bounds__(256)
+    wnorm_kernel(const __nv_bfloat16* __restrict__ w, int E, int d, float* __restrict__ nw,
+                 uint32_t* __restrict__ zw, int nz) {
+  grid_dep_wait();
+  grid_dep_launch();
+  if (zw != nullptr && blockIdx.x == 0)
+    for (int i = threadIdx.x; i < nz; i += blockDim.x) zw[i] = 0u;
+  const int lane = threadIdx.x & 31;
+  const int e = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (e >= E) return;
+  const uint4* row = reinterpret_cast<const uint4*>(w + static_cast<int64_t>(e) * d);
+  float ss = 0.f;
+  for (int v = lane; v < d / 8; v += 32) {
+    const uint4 q = row[v];
+    const uint32_t wd[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float a = __uint_as_float(wd[i] << 16), b = __uint_as_float(wd[i] & 0xffff0000u);
+      ss = fmaf(a, a, ss);
+      ss = fmaf(b, b, ss);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if (lane == 0) nw[e] = sqrtf(ss * (1.0f + 0x1p-10f)) * (1.0f + 0x1p-20f);
+}
+
+// canonical chain of one (token, expert) pair: fma over k = 0 .. d-1 in
+// order.  The token row comes from shared memory (the same address in every
+// lane), the expert row from L2.  (A ring keeping 8-16 expert-row loads in
+// flight per lane made short batches faster but cost occupancy at 8192 and
+// more tokens, where the screen is used.)
+constexpr int kRing = 16;  // d must be a multiple of 8 kRing
+__device__ __forceinline__ float chain_bf16(const uint4* __restrict__ hs,
+                                            const __nv_bfloat16* __restrict__ we, int d) {
+  const uint4* wv = reinterpret_cast<const uint4*>(we);
+  const int nv = d / 8;
+  float acc = 0.f;
+#pragma unroll 4
+  for (int v = 0; v < nv; ++v) {
+    const uint4 a = hs[v], b = __ldg(wv + v);
+    fma_lo(acc, a.x, b.x);
+    fma_hi(acc, a.x, b.x);
+    fma_lo(acc, a.y, b.y);
+    fma_hi(acc, a.y, b.y);
+    fma_lo(acc, a.z, b.z);
+    fma_hi(acc, a.z, b.z);
+    fma_lo(acc, a.w, b.w);
+    fma_hi(acc, a.w, b.w);
+  }
+  return acc;
+}
+
+__device__ __forceinline__ unsigned long long score_key(float v, int e) {
+  v = (v == 0.0f) ? 0.0f : v;  // -0 and +0 are equal scores
+  return (static_cast<unsigned long long>(order_bits(v)) << 32) |
+         static_cast<unsigned long long>(0xffffffffu - static_cast<uint32_t>(e));
+}
+
+template <int NPL>
+__global__ void __launch_bounds__(kScreenWarps * 32)
+    screen_select_kernel(const __nv_bfloat16* __restrict__ h,
+                         const __nv_bfloat16* __restrict__ w, float* __restrict__ z,
+                         int k_splits, int64_t split_stride, const float* __restrict__ nw,
+                         float g, const int32_t* __restrict__ kin, int T, int E, int d,
+                         int k_max, int32_t* __restrict__ ids, float* __restrict__ alpha,
+                         uint32_t* __restrict__ err) {
+  extern __shared__ uint4 s_h[];  // [kScreenWarps][d / 8]: the warps' token rows
+  __shared__ float s_z[kScreenWarps][32];
+  __shared__ int32_t s_e[kScreenWarps][32];
+  __shared__ int32_t s_c[kScreenWarps][32];
+  grid_dep_wait();
+  grid_dep_launch();
+  const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = blockIdx.x * kScreenWarps + wid;
+  if (t >= T) return;
+  const int kcap = k_max < E ? k_max : E;
+  int kt = kin[t];
+  if (kt < 1 || kt > kcap) {
+    if (lane == 0) set_err(err, kErrKRange);
+    kt = kt < 1 ? 1 : kcap;
+  }
+  const __nv_bfloat16* ht = h + static_cast<int64_t>(t) * d;
+  uint4* hs = s_h + static_cast<int64_t>(wid) * (d / 8);
+  // the token row into shared memory and ||h_t||_2, rounded up
+  float ss = 0.f;
+  for (int v = lane; v < d / 8; v += 32) {
+    const uint4 q = reinterpret_cast<const uint4*>(ht)[v];
+    hs[v] = q;
+    const uint32_t wd[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float a = __uint_as_float(wd[i] << 16), b = __uint_as_float(wd[i] & 0xffff0000u);
+      ss = fmaf(a, a, ss);
+      ss = fmaf(b, b, ss);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  __syncwarp();  // the row in shared memory is visible to every lane
+  const float nh = sqrtf(ss * (1.0f + 0x1p-10f)) * (1.0f + 0x1p-20f);
+  // screen estimates and their intervals; L = k_t-th largest lower end
+  float* zt = z + static_cast<int64_t>(t) * E;
+  float zs[NPL], hi[NPL];
+  unsigned long long key[NPL];
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    const int e = lane + 32 * i;
+    zs[i] = 0.f;
+    hi[i] = -INFINITY;
+    key[i] = 0ull;
+    if (e < E) {
+      float v = zt[e];
+      for (int s = 1; s < k_splits; ++s) v += zt[s * split_stride + e];
+      const float del = g * nh * nw[e] * (1.0f + 0x1p-16f) + fabsf(v) * 0x1p-22f;
+      zs[i] = v;
+      hi[i] = v + del;
+      key[i] = score_key(v - del, e);
+    }
+  }
+  unsigned long long best = 0ull;
+  for (int j = 0; j < kt; ++j) {
+    best = key[0];
+#pragma unroll
+    for (int i = 1; i < NPL; ++i) best = key[i] > best ? key[i] : best;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+      best = other > best ? other : best;
+    }
+    const int e = static_cast<int>(0xffffffffu - static_cast<uint32_t>(best & 0xffffffffull));
+    if ((e & 31) == lane) {
+#pragma unroll
+      for (int i = 0; i < NPL; ++i)
+        if (i == (e >> 5)) key[i] = 0ull;
+    }
+  }
+  const float L = from_order_bits(static_cast<uint32_t>(best >> 32));
+  // candidates: hi_e >= L, compacted into s_c (at most 32, else all experts)
+  int m = 0;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    const bool c = hi[i] >= L;
+    const uint32_t mask = __ballot_sync(0xffffffffu, c);
+    const int pos = m + __popc(mask & ((1u << lane) - 1u));
+    if (c && pos < 32) s_c[wid][pos] = lane + 32 * i;
+    m += __popc(mask);
+  }
+  __syncwarp();
+  // every screen estimate stays in z, then the recomputed scores replace the
+  // candidates' entries
+#pragma unroll
+  for (int i = 0; i < NPL; ++i)
+    if (lane + 32 * i < E) zt[lane + 32 * i] = zs[i];
+  __syncwarp();  // the estimates land before any lane overwrites a candidate's
+  unsigned long long ck[NPL];
+  if (m <= 32) {
+    unsigned long long mine = 0ull;
+    if (lane < m) {
+      const int e = s_c[wid][lane];
+      const float v = chain_bf16(hs, w + static_cast<int64_t>(e) * d, d);
+      zt[e] = v;
+      mine = score_key(v, e);
+    }
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) ck[i] = i == 0 ? mine : 0ull;
+  } else {
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) {
+      const int e = lane + 32 * i;
+      ck[i] = 0ull;
+      if (e < E) {
+        const float v = chain_bf16(hs, w + static_cast<int64_t>(e) * d, d);
+        zt[e] = v;
+        ck[i] = score_key(v, e);
+      }
+    }
+  }
+  // TopK over the recomputed scores (same keys and tie rule as select_token)
+  for (int j = 0; j < kt; ++j) {
+    unsigned long long b = ck[0];
+#pragma unroll
+    for (int i = 1; i < NPL; ++i) b = ck[i] > b ? ck[i] : b;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long other = __shfl_xor_sync(0xffffffffu, b, o);
+      b = other > b ? other : b;
+    }
+#pragma unroll
+    for (int i = 0; i < NPL; ++i)
+      if (ck[i] == b) ck[i] = 0ull;
+    if (lane == 0) {
+      s_e[wid][j] = static_cast<int>(0xffffffffu - static_cast<uint32_t>(b & 0xffffffffull));
+      s_z[wid][j] = from_order_bits(static_cast<uint32_t>(b >> 32));
+    }
+  }
+  __syncwarp();
+  const float zmax = s_z[wid][0];
+  const float mine = lane < kt ? expf(s_z[wid][lane] - zmax) : 0.f;
+  float sel = mine;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sel += __shfl_xor_sync(0xffffffffu, sel, o);
+  for (int j = lane; j < k_max; j += 32) {
+    const int64_t o = static_cast<int64_t>(t) * k_max + j;
+    if (j < kt) {
+      ids[o] = s_e[wid][j];
+      alpha[o] = mine / sel;
+    } else {
+      ids[o] = -1;
+      alpha[o] = 0.f;
+    }
+  }
+}
+
 template <int LY, int TM, int TN, int WT, int WE, int S, int KC = 32>
 cudaError_t launch_logits_mx(const __nv_bfloat16* h, const __nv_bfloat16* w, int T,
                              int d, int E, float* z, uint32_t* zw, int nz, cudaStream_t s) {
@@ -800,6 +1037,42 @@ cudaError_t launch_router_logits(int dtype, const void* hidden,
   return logits_dispatch(static_cast<const __nv_bfloat16*>(hidden),
                          static_cast<const __nv_bfloat16*>(w_router), T, d, E,
                          z, zero_words, n_zero, err, num_sms, stream);
+}
+
+cudaError_t launch_router_wnorm(const __nv_bfloat16* w, int E, int d, float* nw,
+                                uint32_t* zero_words, int n_zero, cudaStream_t stream) {
+  // plain launch: the first kernel of the forward
+  wnorm_kernel<<<(E + 7) / 8, 256, 0, stream>>>(w, E, d, nw, zero_words, n_zero);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_router_screen_select(const __nv_bfloat16* h, const __nv_bfloat16* w,
+                                        float* z, int k_splits, int64_t split_stride,
+                                        const float* nw, const int32_t* k, int T, int E,
+                                        int d, int k_max, int32_t* ids, float* alpha,
+                                        uint32_t* err, cudaStream_t stream) {
+  if (T == 0) return cudaSuccess;
+  if (d % (8 * kRing) != 0 || E > 1024 || k_splits < 1) return cudaErrorInvalidValue;
+  const size_t smem = static_cast<size_t>(kScreenWarps) * d * 2;  // bf16 token rows
+  const double u = 1.0 / 16777216.0;
+  const double gamma = d * u / (1.0 - d * u);
+  // chain bound + tensor-core allowance + one rounding per split-K slice
+  const float g = static_cast<float>((gamma + 1.0 / 4096.0 + (k_splits + 1) * u) * (1.0 + 1e-3));
+  const dim3 grid((T + kScreenWarps - 1) / kScreenWarps), block(kScreenWarps * 32);
+#define RX_SCREEN(N)                                                                     \
+  (smem > 48 * 1024 && cudaFuncSetAttribute(screen_select_kernel<N>,                     \
+                                            cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                                            static_cast<int>(smem)) != cudaSuccess)      \
+      ? cudaErrorInvalidValue                                                            \
+      : launch_pdl(screen_select_kernel<N>, grid, block, smem, stream, h, w, z, k_splits, \
+                   split_stride, nw, g, k, T, E, d, k_max, ids, alpha, err)
+  if (E <= 32) return RX_SCREEN(1);
+  if (E <= 64) return RX_SCREEN(2);
+  if (E <= 128) return RX_SCREEN(4);
+  if (E <= 256) return RX_SCREEN(8);
+  if (E <= 512) return RX_SCREEN(16);
+  return RX_SCREEN(32);
+#undef RX_SCREEN
 }
 
 cudaError_t launch_router_select(const float* z, const int32_t* k, int T,

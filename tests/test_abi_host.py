@@ -115,7 +115,7 @@ def test_host_rejections_enqueue_nothing(lib):
     rec = B.reflex_route_record()
     assert fw(1, None, None, None, None, None, None, 0, None, 0, 256, 8, 128, 4,
               1, 256, 1 << 20, None, ctypes.byref(rec), None) == B.REFLEX_OK
-    assert rec.ids == 256 + 256          # first region after the header
+    assert rec.ids == 3 * 256            # after the header, scores and expert norms
     assert lib.reflex_selftest_wait_timeout(None, 10, None) == B.REFLEX_EINVAL
     assert lib.reflex_read_status(None, None) == B.REFLEX_EINVAL
 

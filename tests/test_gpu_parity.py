@@ -183,7 +183,8 @@ def test_router_scores_bit_exact_every_band(T, E, d):
     cfg, layer = _bf16_case(T, d, E, 128, 0, 8, seed=T + E + d)
     k = np.random.default_rng(T).integers(1, 9, T).astype(np.int32)
     gl = G.GpuLayer(cfg, layer)
-    _, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE)
+    _, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE |
+                                B.REFLEX_FLAG_EXACT_SCORES)
     assert status == B.REFLEX_OK
     z = oracle.router_logits(layer["hidden"], layer["w_router"])
     assert np.array_equal(rec["scores"].view(np.uint32), z.view(np.uint32))
@@ -191,6 +192,86 @@ def test_router_scores_bit_exact_every_band(T, E, d):
     assert np.array_equal(rec["ids"], ids)
     valid = ids >= 0
     np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
+
+
+def _bf16_floats(bits: np.ndarray) -> np.ndarray:
+    return (bits.astype(np.uint32) << 16).view(np.float32)
+
+
+def _screen_bound(layer, d, k_splits_max=16):
+    # the screen's interval half-width for every (token, expert), as the
+    # kernel states it: (gamma_d + 2^-12 + (s + 1) u) ||h_t|| ||w_e||
+    u = 2.0 ** -24
+    g = d * u / (1 - d * u) + 2.0 ** -12 + (k_splits_max + 1) * u
+    hn = np.linalg.norm(_bf16_floats(layer["hidden"]).astype(np.float64), axis=1)
+    wn = np.linalg.norm(_bf16_floats(layer["w_router"]).astype(np.float64), axis=1)
+    return g * np.outer(hn, wn) * 1.01
+
+
+# screened routing (tensor-core scores, exact recomputation of the experts
+# that could be selected): ids, alpha and the selected scores bit for bit
+@pytest.mark.parametrize("T,E,d,kmax", [
+    (1024, 128, 2048, 12),   # 8 split-K slices
+    (777, 256, 1024, 12),    # ragged token tiles, two 128-wide score tiles
+    (4096, 256, 2048, 8),    # LLaDA2.0-mini expert count, one slice
+    (100, 160, 512, 6),      # ragged expert tile
+    (33, 128, 256, 4),       # fewer tokens than one tile
+])
+def test_screened_routing_bit_exact(T, E, d, kmax):
+    cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=3 * T + E)
+    k = np.random.default_rng(T + 1).integers(1, kmax + 1, T).astype(np.int32)
+    gl = G.GpuLayer(cfg, layer)
+    _, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE)
+    assert status == B.REFLEX_OK
+    z = oracle.router_logits(layer["hidden"], layer["w_router"])
+    ids, alpha = oracle.select(z, k, kmax)
+    assert np.array_equal(rec["ids"], ids)
+    valid = ids >= 0
+    np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
+    rows = np.repeat(np.arange(T), kmax).reshape(T, kmax)[valid]
+    got = rec["scores"][rows, ids[valid]]
+    assert np.array_equal(got.view(np.uint32), z[rows, ids[valid]].view(np.uint32))
+    # every other score is a tensor-core estimate inside the stated bound
+    assert np.all(np.abs(rec["scores"].astype(np.float64) - z) <= _screen_bound(layer, d))
+
+
+def test_screened_routing_ties_and_many_candidates():
+    # exact ties (duplicated router rows: the lower index wins), near ties
+    # (rows one bf16 step apart) and 40 identical rows, more candidates than
+    # one warp recomputes (every expert of such a token is recomputed)
+    T, E, d, kmax = 512, 128, 1024, 8
+    cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=99)
+    w = layer["w_router"].copy()
+    w[5] = w[3]
+    w[9] = w[3]
+    w[12] = w[11]
+    w[12, 7] ^= np.uint16(1)                       # one bf16 ulp away
+    w[20:60] = w[19]                               # 41 identical experts
+    layer["w_router"] = w
+    k = np.random.default_rng(5).integers(1, kmax + 1, T).astype(np.int32)
+    gl = G.GpuLayer(cfg, layer)
+    _, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE)
+    assert status == B.REFLEX_OK
+    z = oracle.router_logits(layer["hidden"], layer["w_router"])
+    ids, alpha = oracle.select(z, k, kmax)
+    assert np.array_equal(rec["ids"], ids)
+    valid = ids >= 0
+    np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
+    assert np.any(ids == 19) and not np.any(ids == 59)  # a tie group is resolved low
+
+
+def test_screened_and_exact_routing_agree_on_the_whole_layer():
+    cfg = CFG["llada2_mini"]
+    layer = W.make_layer(cfg, 4)
+    k = _k_for(cfg)
+    gl = G.GpuLayer(cfg, layer)
+    out_s, rec_s, st_s = gl.forward(k)
+    out_e, rec_e, st_e = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK |
+                                    B.REFLEX_FLAG_EXACT_SCORES)
+    assert st_s == st_e == B.REFLEX_OK
+    for key in ("ids", "alpha", "offsets", "perm", "row_of"):
+        assert np.array_equal(rec_s[key], rec_e[key]), key
+    assert np.array_equal(out_s.view(np.uint32), out_e.view(np.uint32))
 
 
 @pytest.mark.parametrize("T,d,E,inter,shared,kmax,kmode", [
