@@ -157,11 +157,11 @@ def test_forward_tiny_fp32_full():
     assert rel <= G.F32_REL_L2 and mx <= G.F32_MAX_ABS, (rel, mx)
 
 
-def _bf16_case(T, d, E, inter, shared, kmax, seed):
+def _bf16_case(T, d, E, inter, shared, kmax, seed, weight_std=0.05):
     cfg = W.LayerConfig(name="case", dtype="bf16", d=d, E=E, inter=inter,
                         shared_inter=shared, k_min=1, k_base=min(2, kmax),
                         k_max=kmax, delta_role=1, delta_cur=1, w_cf=0.3, n_seq=1,
-                        prompt_len=T, gen_len=0, block=32, weight_std=0.05,
+                        prompt_len=T, gen_len=0, block=32, weight_std=weight_std,
                         conf="uniform", mask_rule="half")
     layer = W.make_layer(cfg, seed, T=T)
     return cfg, layer
@@ -299,6 +299,26 @@ def test_forward_bf16_small(T, d, E, inter, shared, kmax, kmode, simt):
     gl = G.GpuLayer(cfg, layer)
     flags = B.REFLEX_FLAG_RENORM_TOPK | (B.REFLEX_FLAG_SIMT_EXPERTS if simt else 0)
     out, rec, status = gl.forward(k, flags=flags)
+    assert status == B.REFLEX_OK
+    ref = G.oracle_layer(cfg, layer, k)
+    G.check_routing(rec, ref, k, cfg.E)
+    rel, mx = G.out_errors(out, ref["out"])
+    assert rel <= G.BF16_REL_L2 and mx <= G.BF16_MAX_ABS, (rel, mx)
+
+
+@pytest.mark.parametrize("T,d,E,inter,kmax", [
+    (300, 4096, 16, 128, 8),    # d > 2048: warp-per-token combine, ring score kernel
+    (256, 256, 1024, 128, 32),  # 1024 experts, k up to 32: 32 scores per lane, and
+                                # screened tokens with more than 32 candidates
+])
+def test_forward_bf16_edges(T, d, E, inter, kmax):
+    # the benchmark layers' weight scale (std 0.02), so the outputs have their
+    # magnitude and the absolute bound means the same thing
+    cfg, layer = _bf16_case(T, d, E, inter, 0, kmax, seed=T + d + E, weight_std=0.02)
+    k = np.random.default_rng(E).integers(1, kmax + 1, T).astype(np.int32)
+    k[:8] = kmax
+    gl = G.GpuLayer(cfg, layer)
+    out, rec, status = gl.forward(k)
     assert status == B.REFLEX_OK
     ref = G.oracle_layer(cfg, layer, k)
     G.check_routing(rec, ref, k, cfg.E)
