@@ -426,7 +426,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
         layer_bytes += 3 * S * d * es
     layer_flops = flops_step + (6.0 * d * S * T if S else 0.0)
     t_roof = max(layer_bytes / (peaks["hbm"] * 1e9), layer_flops / (peaks["bf16"] * 1e12))
-    launches_per_step = 10 + (2 if S else 0)
+    launches_per_step = api.step_launches(cfg.dtype, T, d, E, S, F)
     line = dict(
         metric=METRIC, value=tokens_per_s, unit="tokens/s",
         n_gpus=world, steps=args.steps, warmup=args.warmup, ms_per_step=ms_step,
@@ -567,7 +567,8 @@ def run_stack(args, rank, world, local_rank):
         fixed_topk=dict(k=cfg.k_base, pairs_per_layer=pairs_fixed, ms_per_step=ms_fixed,
                         value=R.whole_job_rate(T, world, ms_fixed),
                         expert_tflops=flops_fixed * world / (ms_fixed * 1e-3) / 1e12),
-        gpu_launches=args.steps * (1 + 10 * L),
+        # the counts once, then every layer's forward
+        gpu_launches=args.steps * (1 + L * (api.step_launches(cfg.dtype, T, d, E, 0, F) - 1)),
         clocks=dict(sm_mhz=clocks["sm_mhz"], sm_max_mhz=clocks["sm_max_mhz"],
                     reasons=clocks["reasons"], samples=clocks["samples"]),
         peak_source=peaks["source"] + " (sustained bf16, long step)")

@@ -360,14 +360,17 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
   void* ysh = shared_inter ? ws + L.ysh : nullptr;
 
   if (ac != nullptr) RX_CUDA(clear_alloc_outputs(*ac, s));
-  // bf16 with renormalised weights and many experts: tensor-core scores
-  // screen the experts and only those that could be selected get the
-  // canonical chain (router.cu).  The recheck costs about as much per chain
-  // as 40 chains of the dense score kernels, so it pays from 128 experts on
-  // (LLaDA2.0-mini layer, 256 experts: routing 213 -> 113 us; with 64
-  // experts the dense kernels stay faster at every batch size measured).
+  // bf16 with renormalised weights, many experts and many scores: tensor-
+  // core scores screen the experts and only those that could be selected get
+  // the canonical chain (router.cu).  The recheck costs about as much per
+  // chain as 40 chains of the dense score kernels and has a latency floor, so
+  // it pays from 128 experts and 2048 x 256 scores on (LLaDA2.0-mini layer:
+  // routing 213 -> 113 us at 8192 tokens, layer 4.90 -> 4.35 ms at 65536;
+  // below 2048 tokens, and with 64 experts at every size, the dense kernels
+  // are faster).
   const bool screen = dtype == REFLEX_DTYPE_BF16 && (flags & REFLEX_FLAG_RENORM_TOPK) &&
-                      !(flags & REFLEX_FLAG_EXACT_SCORES) && d % 128 == 0 && E >= 128;
+                      !(flags & REFLEX_FLAG_EXACT_SCORES) && d % 128 == 0 && E >= 128 &&
+                      static_cast<int64_t>(T) * E >= 2048 * 256;
   if ((stages & REFLEX_STAGE_ROUTE) && screen) {
     const int bn = rx::screen_bn(E), ks = rx::screen_splits(T, E, d);
     CUtensorMap mh, mw;

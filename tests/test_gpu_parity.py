@@ -210,12 +210,13 @@ def _screen_bound(layer, d, k_splits_max=16):
 
 # screened routing (tensor-core scores, exact recomputation of the experts
 # that could be selected): ids, alpha and the selected scores bit for bit
+# (the screen runs from 128 experts and 2048 x 256 scores on)
 @pytest.mark.parametrize("T,E,d,kmax", [
-    (1024, 128, 2048, 12),   # 8 split-K slices
-    (777, 256, 1024, 12),    # ragged token tiles, two 128-wide score tiles
-    (4096, 256, 2048, 8),    # LLaDA2.0-mini expert count, one slice
-    (100, 160, 512, 6),      # ragged expert tile
-    (33, 128, 256, 4),       # fewer tokens than one tile
+    (4096, 128, 2048, 12),   # 128-wide score tiles, one slice
+    (2100, 256, 1024, 12),   # ragged token tiles, two score tiles per row
+    (4096, 256, 2048, 8),    # LLaDA2.0-mini expert count
+    (3300, 160, 512, 6),     # ragged expert tile
+    (2048, 256, 256, 4),     # short rows
 ])
 def test_screened_routing_bit_exact(T, E, d, kmax):
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=3 * T + E)
@@ -239,7 +240,7 @@ def test_screened_routing_ties_and_many_candidates():
     # exact ties (duplicated router rows: the lower index wins), near ties
     # (rows one bf16 step apart) and 40 identical rows, more candidates than
     # one warp recomputes (every expert of such a token is recomputed)
-    T, E, d, kmax = 512, 128, 1024, 8
+    T, E, d, kmax = 4096, 128, 1024, 8
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=99)
     w = layer["w_router"].copy()
     w[5] = w[3]
@@ -308,7 +309,7 @@ def test_forward_bf16_small(T, d, E, inter, shared, kmax, kmode, simt):
 
 @pytest.mark.parametrize("T,d,E,inter,kmax", [
     (300, 4096, 16, 128, 8),    # d > 2048: warp-per-token combine, ring score kernel
-    (256, 256, 1024, 128, 32),  # 1024 experts, k up to 32: 32 scores per lane, and
+    (512, 256, 1024, 128, 32),  # 1024 experts, k up to 32: 32 scores per lane, and
                                 # screened tokens with more than 32 candidates
 ])
 def test_forward_bf16_edges(T, d, E, inter, kmax):

@@ -160,3 +160,26 @@ def test_step_llada_moe_against_oracle():
     G.check_routing({kk: v.cpu().numpy() for kk, v in moe.record().items()}, ref, k_ref, cfg.E)
     rel, mx = G.out_errors(G.to_f32(out), ref["out"])
     assert rel <= G.BF16_REL_L2 and mx <= G.BF16_MAX_ABS, (rel, mx)
+
+
+@pytest.mark.parametrize("name", ["llada_moe", "llada2_mini", "llada_moe_b32"])
+def test_step_launch_count_matches_a_profile(name):
+    # the bench's launch claim (api.step_launches) against the kernels a
+    # profiler sees in one step; memsets are not kernels
+    profiler = pytest.importorskip("torch.profiler")
+    cfg, layer, dl, moe = _setup(name, 1)
+    p = G.params_of(cfg)
+    ds = api.state_to_device(W.make_state(cfg, 0, hist_len=None))
+    moe.step(ds, p, dl["hidden"])          # warm: first-call attribute setup
+    torch.cuda.synchronize()
+    with profiler.profile(activities=[profiler.ProfilerActivity.CUDA]):
+        moe.step(ds, p, dl["hidden"])      # warm the profiler itself
+        torch.cuda.synchronize()
+    with profiler.profile(activities=[profiler.ProfilerActivity.CUDA]) as prof:
+        moe.step(ds, p, dl["hidden"])
+        torch.cuda.synchronize()
+    names = [e.name for e in prof.events()
+             if e.device_type == torch.autograd.DeviceType.CUDA and "rx::" in e.name]
+    if not names:
+        pytest.skip("no kernel activity recorded by the profiler")
+    assert len(names) == api.step_launches(cfg.dtype, cfg.T, cfg.d, cfg.E, cfg.shared_inter)
