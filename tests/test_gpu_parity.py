@@ -173,6 +173,9 @@ def _bf16_case(T, d, E, inter, shared, kmax, seed, weight_std=0.05):
     (1000, 64, 2048),    # whole rows resident, ragged token tile
     (1200, 48, 512),     # whole rows resident, ragged expert tile
     (250, 256, 1024),    # whole rows resident, 4 chunks
+    (700, 128, 2048),    # whole rows resident, ragged token tile, 4 expert tiles
+    (2000, 32, 512),     # whole rows resident, one expert tile
+    (500, 160, 1024),    # whole rows resident, 5 expert tiles, ragged expert tile
     (2000, 64, 256),     # ring kernel, 1 x 2
     (4096, 64, 256),     # ring kernel, 2 x 2, 64-k chunks
     (8192, 128, 256),    # ring kernel, 4 x 8
@@ -189,6 +192,22 @@ def test_router_scores_bit_exact_every_band(T, E, d):
     z = oracle.router_logits(layer["hidden"], layer["w_router"])
     assert np.array_equal(rec["scores"].view(np.uint32), z.view(np.uint32))
     ids, alpha = oracle.select(z, k, cfg.k_max)
+    assert np.array_equal(rec["ids"], ids)
+    valid = ids >= 0
+    np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
+
+
+@pytest.mark.parametrize("T,E,d", [(1000, 64, 2048), (250, 256, 1024)])
+def test_router_without_renorm_bit_exact(T, E, d):
+    # weights over all experts' scores (softmax over every expert)
+    cfg, layer = _bf16_case(T, d, E, 128, 0, 8, seed=T + 7)
+    k = np.random.default_rng(T + 2).integers(1, 9, T).astype(np.int32)
+    gl = G.GpuLayer(cfg, layer)
+    _, rec, status = gl.forward(k, flags=B.REFLEX_STAGE_ROUTE)
+    assert status == B.REFLEX_OK
+    z = oracle.router_logits(layer["hidden"], layer["w_router"])
+    assert np.array_equal(rec["scores"].view(np.uint32), z.view(np.uint32))
+    ids, alpha = oracle.select(z, k, cfg.k_max, renorm=False)
     assert np.array_equal(rec["ids"], ids)
     valid = ids >= 0
     np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
@@ -236,11 +255,13 @@ def test_screened_routing_bit_exact(T, E, d, kmax):
     assert np.all(np.abs(rec["scores"].astype(np.float64) - z) <= _screen_bound(layer, d))
 
 
-def test_screened_routing_ties_and_many_candidates():
+@pytest.mark.parametrize("T,E", [(4096, 128), (1000, 64)])
+def test_screened_routing_ties_and_many_candidates(T, E):
     # exact ties (duplicated router rows: the lower index wins), near ties
     # (rows one bf16 step apart) and 40 identical rows, more candidates than
-    # one warp recomputes (every expert of such a token is recomputed)
-    T, E, d, kmax = 4096, 128, 1024, 8
+    # one warp recomputes (every expert of such a token is recomputed); at
+    # 1000 x 64 the dense score kernels and the plain selection
+    d, kmax = 1024, 8
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=99)
     w = layer["w_router"].copy()
     w[5] = w[3]
