@@ -81,6 +81,8 @@ struct KParams {
   // 1: launched right behind a kernel that writes none of this kernel's
   // inputs or outputs; start at once and wait for it only before exiting
   int defer_wait;
+  // SwiGLU: map_b is the 3D {K, inter, 2 groups} map of tc_gate_up_3d
+  int b3d;
 };
 
 // ---- PTX wrappers ---------------------------------------------------------
@@ -119,6 +121,24 @@ __device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
       ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar), "l"(pol)
+      : "memory");
+}
+// 3D boxes: the gate and up blocks of one weight tile in one copy (the map's
+// dims are {K, rows per half, halves}: halves 2e and 2e + 1 of expert e)
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int c0,
+                                            int c1, int c2, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap* map, int c0,
+                                                 int c1, int c2, uint32_t bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(bar), "l"(pol)
       : "memory");
 }
 __device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
@@ -325,8 +345,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (once) tma_load_2d_hint(dst, &map_b, k0, row, fb, pol_once);
           else tma_load_2d(dst, &map_b, k0, row, fb);
         };
-        load_b(b_dst, wr);
-        if (MODE == kModeSwiGLU) load_b(b_dst + (BN / 2) * BK * 2, wr + p.b_up_offset);
+        if (MODE == kModeSwiGLU && p.b3d) {
+          // gate rows then up rows of the tile, one copy
+          if (once) tma_load_3d_hint(b_dst, &map_b, k0, tl.n * (BN / 2), 2 * tl.e, fb, pol_once);
+          else tma_load_3d(b_dst, &map_b, k0, tl.n * (BN / 2), 2 * tl.e, fb);
+        } else {
+          load_b(b_dst, wr);
+          if (MODE == kModeSwiGLU) load_b(b_dst + (BN / 2) * BK * 2, wr + p.b_up_offset);
+        }
         issued_mask |= 1u << stage;
         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
         if (++stage == kStages) {
@@ -532,6 +558,7 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.split_stride = 0;
   p.n_valid = 0;
   p.defer_wait = 0;
+  p.b3d = MODE == kModeSwiGLU && a.b_gate_up_3d ? 1 : 0;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);
@@ -899,6 +926,7 @@ cudaError_t launch_pair_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.split_stride = 0;
   p.n_valid = 0;
   p.defer_wait = 0;
+  p.b3d = 0;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   int pairs = a.num_sms / 2;
@@ -960,6 +988,7 @@ cudaError_t launch_scores_impl(const TcGemmArgs& a, int k_splits, float* out,
   p.split_stride = split_stride;
   p.n_valid = n_valid;
   p.defer_wait = defer_wait ? 1 : 0;
+  p.b3d = 0;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles * k_splits;
   if (max_tiles == 0) return cudaSuccess;
   const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);

@@ -44,10 +44,17 @@ cudaError_t launch_update_state(const float* conf_new, float* conf1, float* conf
 // The first CTA also clears zero_words[0, n_zero) (nullable): the call's
 // header or error word, so no memset precedes the first kernel.  err
 // (nullable) receives kErrTimeout if a bounded wait of a kernel expires.
+// pf (optional): bytes the score kernel hands to the L2 as bulk prefetches
+// while it computes (the next kernels' weights; HBM is otherwise idle then).
+struct L2Prefetch {
+  const void* base = nullptr;
+  uint64_t bytes = 0;  // a multiple of 16
+};
 cudaError_t launch_router_logits(int dtype, const void* hidden,
                                  const void* w_router, int T, int d, int E,
                                  float* z, uint32_t* zero_words, int n_zero,
-                                 uint32_t* err, int num_sms, cudaStream_t stream);
+                                 uint32_t* err, int num_sms, cudaStream_t stream,
+                                 const L2Prefetch& pf = L2Prefetch{});
 // Screened routing (bf16, renormalised weights): nw[e] = ||w_e||_2 rounded up
 // (first kernel of the forward; clears zero_words like the score kernels);
 // then, from the tensor-core score slices z[s][t][e] (s < k_splits), the
@@ -141,6 +148,9 @@ struct TcGemmArgs {
   int ldo;
   uint32_t* err;
   int num_sms;
+  // SwiGLU, 1-SM kernel: map_b is the 3D map of tc_gate_up_3d (box {64,
+  // bn / 2, 2}: a tile's gate and up rows in one copy) instead of a 2D map
+  bool b_gate_up_3d = false;
 };
 // SwiGLU: out = silu(A Wg^T) * (A Wu^T).  Down: out = A Wd^T.  bn = tile
 // width (128 or 256, from tc_pick_bn); the B tensor map's box must have

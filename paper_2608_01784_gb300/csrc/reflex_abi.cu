@@ -17,6 +17,8 @@ namespace {
 using rx::WsHeader;
 
 constexpr size_t kAlign = 256;
+// gate/up weight bytes handed to the L2 while the router scores run
+constexpr uint64_t kRouterL2Prefetch = 64ull << 20;
 size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 // Byte offsets of every workspace region (all 256-byte aligned).
@@ -113,6 +115,26 @@ bool make_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols,
   cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base),
+                  dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// Gate/up weights [groups][2][inter][K] as a 3D map {K, inter, 2 groups}:
+// one box {64, box_rows, 2} holds a tile's gate rows and the matching up rows.
+bool make_map_gate_up(CUtensorMap* m, const void* base, int64_t groups, int64_t inter,
+                      int64_t cols, int box_rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) != 0) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(inter),
+                        static_cast<cuuint64_t>(2 * groups)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(cols) * 2,
+                           static_cast<cuuint64_t>(inter) * static_cast<cuuint64_t>(cols) * 2};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(box_rows), 2};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base),
                   dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                   CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -394,9 +416,19 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
   } else if (stages & REFLEX_STAGE_ROUTE) {
     // the router's first CTA clears the header (error word, totals): no
     // kernel before the router reads it
+    // the first experts' gate/up weights are handed to the L2 while the
+    // scores run (the grouped GEMM walks the experts in order; LLaDA-MoE
+    // layer step -2 us with 64 MB)
+    rx::L2Prefetch pf;
+    if (stages & REFLEX_STAGE_EXPERT_UP) {
+      const uint64_t wbytes =
+          static_cast<uint64_t>(E) * 2 * inter * d * (dtype == REFLEX_DTYPE_F32 ? 4 : 2);
+      pf.base = w_gate_up;
+      pf.bytes = (wbytes < kRouterL2Prefetch ? wbytes : kRouterL2Prefetch) & ~uint64_t{4095};
+    }
     RX_CUDA(rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z,
                                      reinterpret_cast<uint32_t*>(hdr),
-                                     static_cast<int>(sizeof(WsHeader) / 4), err, sms, s));
+                                     static_cast<int>(sizeof(WsHeader) / 4), err, sms, s, pf));
     if (ac != nullptr) RX_CUDA(launch_alloc(*ac, T, s, true));
     RX_CUDA(rx::launch_router_select(z, k, T, E, k_max,
                                      (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
@@ -433,13 +465,15 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
     } else {
       CUtensorMap ma1, mb1, ma2, mb2;
       if (!make_map(&ma1, xperm, cap, d, rx::kTileM) ||
-          !make_map(&mb1, w_gate_up, static_cast<int64_t>(E) * 2 * inter, d,
-                    pair_routed ? 128 : rx::tc_b_box_rows(true, bn_up)) ||
+          !(pair_routed ? make_map(&mb1, w_gate_up, static_cast<int64_t>(E) * 2 * inter, d, 128)
+                        : make_map_gate_up(&mb1, w_gate_up, E, inter, d,
+                                           rx::tc_b_box_rows(true, bn_up))) ||
           !make_map(&ma2, amid, cap, inter, rx::kTileM) ||
           !make_map(&mb2, w_down, static_cast<int64_t>(E) * d, inter,
                     pair_routed ? 128 : rx::tc_b_box_rows(false, bn_dn)))
         return REFLEX_ECUDA;
-      rx::TcGemmArgs g1{&ma1, &mb1, d, inter, 2 * inter, inter, grouped, amid, inter, err, sms};
+      rx::TcGemmArgs g1{&ma1, &mb1, d, inter, 2 * inter, inter, grouped, amid, inter, err, sms,
+                        !pair_routed};
       rx::TcGemmArgs g2{&ma2, &mb2, inter, d, d, 0, grouped, xperm, d, err, sms};
       // the dense shared expert on CTA pairs once it has enough rows: a 256 x
       // 256 pair tile moves a quarter of the operand bytes per output that a
@@ -450,14 +484,16 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
       CUtensorMap sa1, sb1, sa2, sb2;
       if (shared_inter &&
           (!make_map(&sa1, hidden, T, d, rx::kTileM) ||
-           !make_map(&sb1, shared_gate_up, 2 * static_cast<int64_t>(shared_inter), d,
-                     pair_shared ? 128 : rx::tc_b_box_rows(true, bn_sup)) ||
+           !(pair_shared
+                 ? make_map(&sb1, shared_gate_up, 2 * static_cast<int64_t>(shared_inter), d, 128)
+                 : make_map_gate_up(&sb1, shared_gate_up, 1, shared_inter, d,
+                                    rx::tc_b_box_rows(true, bn_sup))) ||
            !make_map(&sa2, ash, T, shared_inter, rx::kTileM) ||
            !make_map(&sb2, shared_down, d, shared_inter,
                      pair_shared ? 128 : rx::tc_b_box_rows(false, bn_sdn))))
         return REFLEX_ECUDA;
       rx::TcGemmArgs h1{&sa1, &sb1, d, shared_inter, 2 * shared_inter, shared_inter,
-                        dense, ash, shared_inter, err, sms};
+                        dense, ash, shared_inter, err, sms, !pair_shared};
       rx::TcGemmArgs h2{&sa2, &sb2, shared_inter, d, d, 0, dense, ysh, d, err, sms};
       if (up) {
         if (pair_routed)

@@ -567,6 +567,7 @@ constexpr int kResChunkK = 256;   // k per chunk; d must be a multiple
 constexpr int kResSteps = kResChunkK / 8;  // 16-byte steps per row per chunk
 constexpr int kResMaxChunks = 16;
 constexpr int kResBarBytes = 128;
+constexpr uint64_t kL2PrefetchPiece = 64u * 1024u;
 constexpr uint64_t kResWaitNs = 2000000000ull;
 constexpr uint64_t kResDrainNs = 1000000000ull;
 
@@ -624,12 +625,30 @@ __device__ __forceinline__ void mx_fma8(float (&acc)[TM][TN], const MxOps<TM, TN
   }
 }
 
+// Each CTA hands its share of [pf.base, pf.base + pf.bytes) to the L2 as
+// bulk prefetches (the TMA unit moves them; no thread waits for them).
+__device__ __forceinline__ void l2_prefetch_share(const L2Prefetch& pf) {
+  if (pf.bytes == 0) return;
+  const uint64_t nct = static_cast<uint64_t>(gridDim.x) * gridDim.y;
+  const uint64_t cid = static_cast<uint64_t>(blockIdx.y) * gridDim.x + blockIdx.x;
+  uint64_t chunk = (pf.bytes + nct - 1) / nct;
+  chunk = (chunk + 4095u) & ~static_cast<uint64_t>(4095u);
+  const uint64_t b0 = cid * chunk;
+  const uint64_t b1 = b0 + chunk < pf.bytes ? b0 + chunk : pf.bytes;
+  const uint8_t* base = static_cast<const uint8_t*>(pf.base);
+  for (uint64_t b = b0; b < b1; b += kL2PrefetchPiece) {
+    const uint32_t n = static_cast<uint32_t>(b1 - b < kL2PrefetchPiece ? b1 - b : kL2PrefetchPiece);
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + b), "r"(n)
+                 : "memory");
+  }
+}
+
 template <int LY, int TM, int TN, int WT, int WE>
 __global__ void __launch_bounds__(ResCfg<LY, TM, TN, WT, WE>::NT, 1)
     logits_res_kernel(const __nv_bfloat16* __restrict__ h,
                       const __nv_bfloat16* __restrict__ w, int T, int d, int E,
                       float* __restrict__ z, uint32_t* __restrict__ zw, int nz,
-                      uint32_t* __restrict__ err) {
+                      uint32_t* __restrict__ err, L2Prefetch pf) {
   using C = ResCfg<LY, TM, TN, WT, WE>;
   constexpr int LX = C::LX, BT = C::BT, BE = C::BE, NT = C::NT;
   constexpr int kVecs = C::kRows * kResSteps;  // 16-byte copies per chunk
@@ -664,6 +683,7 @@ __global__ void __launch_bounds__(ResCfg<LY, TM, TN, WT, WE>::NT, 1)
     }
     cp_async_arrive_noinc(smem_addr(&bars[c]));
   }
+  if (threadIdx.x == 0) l2_prefetch_share(pf);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ty = lane / LX, tx = lane % LX;
   const int wt = warp / WE, we = warp % WE;
@@ -713,7 +733,7 @@ __global__ void __launch_bounds__(ResCfg<LY, TM, TN, WT, WE>::NT, 1)
 template <int LY, int TM, int TN, int WT, int WE>
 cudaError_t launch_logits_res(const __nv_bfloat16* h, const __nv_bfloat16* w, int T, int d,
                               int E, float* z, uint32_t* zw, int nz, uint32_t* err,
-                              cudaStream_t s) {
+                              const L2Prefetch& pf, cudaStream_t s) {
   using C = ResCfg<LY, TM, TN, WT, WE>;
   if (d % kResChunkK != 0 || d / kResChunkK > kResMaxChunks) return cudaErrorInvalidValue;
   auto kern = logits_res_kernel<LY, TM, TN, WT, WE>;
@@ -722,7 +742,7 @@ cudaError_t launch_logits_res(const __nv_bfloat16* h, const __nv_bfloat16* w, in
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const dim3 g((T + C::BT - 1) / C::BT, (E + C::BE - 1) / C::BE);
-  kern<<<g, C::NT, smem, s>>>(h, w, T, d, E, z, zw, nz, err);
+  kern<<<g, C::NT, smem, s>>>(h, w, T, d, E, z, zw, nz, err, pf);
   return cudaGetLastError();
 }
 
@@ -1006,7 +1026,7 @@ cudaError_t logits_dispatch(const float* h, const float* w, int T, int d, int E,
 // or 4 x 4 thread tiles, which need fewer operand reads per fma.
 cudaError_t logits_dispatch(const __nv_bfloat16* h, const __nv_bfloat16* w, int T,
                             int d, int E, float* z, uint32_t* zw, int nz, uint32_t* err,
-                            int num_sms, cudaStream_t s) {
+                            int num_sms, cudaStream_t s, const L2Prefetch& pf) {
   const int64_t per_sm = static_cast<int64_t>(T) * E / (num_sms > 0 ? num_sms : 1);
   // whole rows resident: 16 x 32 tiles, one CTA per SM, for about 300-640
   // chains per SM (1024 x 64 scores: 20.8 -> 18.1 us; fewer chains favour
@@ -1014,7 +1034,7 @@ cudaError_t logits_dispatch(const __nv_bfloat16* h, const __nv_bfloat16* w, int 
   using Res = ResCfg<4, 2, 2, 2, 2>;
   if (per_sm > 300 && per_sm <= 640 && d % kResChunkK == 0 &&
       d / kResChunkK <= kResMaxChunks && Res::smem(d) <= 227 * 1024)
-    return launch_logits_res<4, 2, 2, 2, 2>(h, w, T, d, E, z, zw, nz, err, s);
+    return launch_logits_res<4, 2, 2, 2, 2>(h, w, T, d, E, z, zw, nz, err, pf, s);
   if (per_sm <= 216) return launch_logits_mx<4, 1, 1, 4, 1, 8>(h, w, T, d, E, z, zw, nz, s);
   if (per_sm <= 1080) return launch_logits_mx<4, 1, 2, 4, 1, 8>(h, w, T, d, E, z, zw, nz, s);
   if (per_sm <= 4300) return launch_logits_mx<4, 2, 2, 2, 2, 4, 64>(h, w, T, d, E, z, zw, nz, s);
@@ -1028,7 +1048,8 @@ cudaError_t logits_dispatch(const __nv_bfloat16* h, const __nv_bfloat16* w, int 
 cudaError_t launch_router_logits(int dtype, const void* hidden,
                                  const void* w_router, int T, int d, int E,
                                  float* z, uint32_t* zero_words, int n_zero,
-                                 uint32_t* err, int num_sms, cudaStream_t stream) {
+                                 uint32_t* err, int num_sms, cudaStream_t stream,
+                                 const L2Prefetch& pf) {
   if (T == 0) return cudaSuccess;
   if (dtype == 0)
     return logits_dispatch(static_cast<const float*>(hidden),
@@ -1036,7 +1057,7 @@ cudaError_t launch_router_logits(int dtype, const void* hidden,
                            zero_words, n_zero, num_sms, stream);
   return logits_dispatch(static_cast<const __nv_bfloat16*>(hidden),
                          static_cast<const __nv_bfloat16*>(w_router), T, d, E,
-                         z, zero_words, n_zero, err, num_sms, stream);
+                         z, zero_words, n_zero, err, num_sms, stream, pf);
 }
 
 cudaError_t launch_router_wnorm(const __nv_bfloat16* w, int E, int d, float* nw,
