@@ -3,8 +3,7 @@
 // out grouped by expert and, within an expert, in token order, so that each
 // expert's rows form one contiguous range of a grouped GEMM.
 //
-// Three launches (two for short batches, whose count and scan share one
-// CTA), no atomics whose order matters:
+// Three launches, no atomics whose order matters:
 //   count   per block of 256 tokens, a bitmask per expert in shared memory
 //           (bit = token of the block selected the expert; a token selects
 //           an expert at most once) and its popcount per expert;
@@ -14,7 +13,11 @@
 //   scatter rebuilds the block's masks; the row of pair (t, j) is
 //           offsets[e] + block prefix + popcount of lower tokens' bits.
 // A fourth launch gathers X rows into pair order (one warp per token: the
-// hidden row is read once and written to each of its pair rows).
+// hidden row is read once and written to each of its pair rows).  Short
+// batches take two launches: count and scan in one CTA (32-token blocks,
+// one mask word per block and expert, kept in global memory), then the
+// gather, whose warps place their token's pairs from those masks as scatter
+// does.
 #include "common.cuh"
 #include "internal.h"
 
@@ -143,31 +146,34 @@ __global__ void __launch_bounds__(1024)
   }
 }
 
-// Short batches: the count and scan steps in one CTA.  Every pair adds one
-// to its (32-token block, expert) counter in shared memory (integer sums, so
-// the order of the additions does not matter); then, per expert, the block
-// prefixes and the total, and the expert and tile prefixes as in scan_kernel.
-// The block counts never leave shared memory.
+// Short batches: the count and scan steps in one CTA.  Every pair sets its
+// token's bit in the (32-token block, expert) mask word in shared memory
+// (a token selects an expert at most once; OR is order-free); then, per
+// expert, the block prefixes of the popcounts and the total, and the expert
+// and tile prefixes as in scan_kernel.  The masks and block prefixes go to
+// global memory for gather_scatter_kernel.
 __global__ void __launch_bounds__(1024)
     count_scan_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ k,
                       int T, int E, int k_max, int nblk, int32_t* __restrict__ blk_off,
                       int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
                       int32_t* __restrict__ mt_prefix, int32_t* __restrict__ mt2_prefix,
-                      int32_t* __restrict__ totals, uint32_t* __restrict__ err) {
-  extern __shared__ int s_cnt[];  // [nblk][E]
+                      int32_t* __restrict__ totals, uint32_t* __restrict__ blk_mask,
+                      uint32_t* __restrict__ err) {
+  extern __shared__ uint32_t s_mask[];  // [nblk][E]: bit = token of the block
   __shared__ int s_warp[32];
   grid_dep_wait();
   grid_dep_launch();
-  for (int i = threadIdx.x; i < nblk * E; i += 1024) s_cnt[i] = 0;
+  for (int i = threadIdx.x; i < nblk * E; i += 1024) s_mask[i] = 0u;
   __syncthreads();
   const int kcap = k_max < E ? k_max : E;
   for (int t = threadIdx.x; t < T; t += 1024) {
     const int kt = clamp_k(k[t], kcap);
-    int* row = s_cnt + (t / kDispatchBlockSmall) * E;
+    uint32_t* row = s_mask + (t / kDispatchBlockSmall) * E;
+    const uint32_t bit = 1u << (t % kDispatchBlockSmall);
     for (int j = 0; j < kt; ++j) {
       const int e = ids[static_cast<int64_t>(t) * k_max + j];
       if (e >= 0 && e < E)
-        atomicAdd(&row[e], 1);
+        atomicOr(&row[e], bit);
       else
         set_err(err, kErrIndex);
     }
@@ -177,8 +183,11 @@ __global__ void __launch_bounds__(1024)
   int run = 0;
   if (e < E) {
     for (int b = 0; b < nblk; ++b) {
-      blk_off[static_cast<int64_t>(b) * E + e] = run;
-      run += s_cnt[b * E + e];
+      const int64_t i = static_cast<int64_t>(b) * E + e;
+      const uint32_t m = s_mask[b * E + e];
+      blk_off[i] = run;
+      blk_mask[i] = m;
+      run += __popc(m);
     }
     counts[e] = run;
   }
@@ -291,6 +300,93 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// Short batches: the scatter step inside the gather.  Lane j of a warp of
+// token t places pair (t, j) at offsets[e] + block prefix + the popcount of
+// the lower tokens' bits in its block's mask word of expert e (the same row
+// as scatter_kernel), the warp of the row's first segment writes perm and
+// row_of, and every warp copies its segment of the hidden row to the pair
+// rows as gather_kernel does.
+template <typename Te>
+__global__ void __launch_bounds__(256)
+    gather_scatter_kernel(const Te* __restrict__ x, const int32_t* __restrict__ ids,
+                          const int32_t* __restrict__ k, const uint32_t* __restrict__ blk_mask,
+                          const int32_t* __restrict__ blk_off,
+                          const int32_t* __restrict__ offsets, int E, int k_max, int cap_rows,
+                          int T, int d, int wpt, int32_t* __restrict__ perm,
+                          int32_t* __restrict__ row_of, Te* __restrict__ xp,
+                          uint32_t* __restrict__ err) {
+  constexpr int kVecElems = 16 / sizeof(Te);
+  constexpr int kMaxVec = 8;
+  grid_dep_wait();
+  grid_dep_launch();
+  const int lane = threadIdx.x & 31;
+  const int warps = gridDim.x * 8;
+  const int row_vecs = d / kVecElems;
+  const int seg_vecs = row_vecs / wpt;
+  const int units = T * wpt;
+  const int kcap = k_max < E ? k_max : E;
+  for (int u = blockIdx.x * 8 + (threadIdx.x >> 5); u < units; u += warps) {
+    const int t = u / wpt;
+    const int seg = u % wpt;
+    const int v0 = seg * seg_vecs;
+    const int kt = clamp_k(k[t], kcap);
+    int my_row = -1;
+    if (lane < k_max) {
+      const int64_t o = static_cast<int64_t>(t) * k_max + lane;
+      if (lane < kt) {
+        const int e = ids[o];
+        if (e >= 0 && e < E) {
+          const int64_t bi = static_cast<int64_t>(t / kDispatchBlockSmall) * E + e;
+          const uint32_t below = (1u << (t % kDispatchBlockSmall)) - 1u;
+          my_row = offsets[e] + blk_off[bi] + __popc(blk_mask[bi] & below);
+          if (my_row < 0 || my_row >= cap_rows) {
+            set_err(err, kErrIndex);
+            my_row = -1;
+          }
+        }
+      }
+      if (seg == 0) {
+        row_of[o] = my_row;
+        if (my_row >= 0) perm[my_row] = static_cast<int32_t>(o);
+      }
+    }
+    const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(t) * d) + v0;
+    for (int base = 0; base < seg_vecs; base += 32 * kMaxVec) {
+      uint4 v[kMaxVec];
+#pragma unroll
+      for (int i = 0; i < kMaxVec; ++i) {
+        const int q = base + lane + 32 * i;
+        if (q < seg_vecs) v[i] = __ldg(src + q);
+      }
+      for (int j = 0; j < kt; ++j) {
+        const int r = __shfl_sync(0xffffffffu, my_row, j);
+        if (r < 0) continue;
+        uint4* dst = reinterpret_cast<uint4*>(xp + static_cast<int64_t>(r) * d) + v0;
+#pragma unroll
+        for (int i = 0; i < kMaxVec; ++i) {
+          const int q = base + lane + 32 * i;
+          if (q < seg_vecs) dst[q] = v[i];
+        }
+      }
+    }
+  }
+}
+
+// warps per token for the gather (enough warps for 16 per SM, each segment
+// whole 16-byte vectors) and the grid
+void gather_shape(int dtype, int T, int d, int num_sms, int* wpt_out, int* grid_out) {
+  const int row_vecs = d * (dtype == 0 ? 4 : 2) / 16;
+  int wpt = 1;
+  while (wpt < 8 && static_cast<int64_t>(T) * wpt < 16LL * num_sms &&
+         row_vecs % (2 * wpt) == 0)
+    wpt *= 2;
+  const int64_t warps = static_cast<int64_t>(T) * wpt;
+  int grid = static_cast<int>((warps + 7) / 8);
+  if (grid > 16 * num_sms) grid = 16 * num_sms;
+  *wpt_out = wpt;
+  *grid_out = grid;
+}
+
 }  // namespace
 
 template <int BLK>
@@ -314,68 +410,77 @@ cudaError_t launch_dispatch_blk(const int32_t* ids, const int32_t* k, int T, int
                     k_max, b.blk_off, b.offsets, b.perm, b.row_of, b.err);
 }
 
-// Short batches whose block counts fit in shared memory: count + scan in one
-// CTA, then the scatter.
+// Short batches whose block masks fit in shared memory: count + scan in one
+// CTA, then the gather, which also places the pairs.
 constexpr size_t kCountScanSmem = 160 * 1024;
 
-static cudaError_t launch_dispatch_small(const int32_t* ids, const int32_t* k, int T, int E,
-                                  int k_max, const DispatchBufs& b, cudaStream_t stream) {
+template <typename Te>
+static cudaError_t launch_dispatch_small(const Te* hidden, const int32_t* ids, const int32_t* k,
+                                         int T, int E, int k_max, int cap_rows, int d,
+                                         const DispatchBufs& b, Te* x_perm, int num_sms,
+                                         cudaStream_t stream) {
   constexpr int BLK = kDispatchBlockSmall;
   const int nblk = (T + BLK - 1) / BLK;
-  const size_t cs_smem = static_cast<size_t>(nblk) * E * sizeof(int);
+  const size_t cs_smem = static_cast<size_t>(nblk) * E * sizeof(uint32_t);
   if (cs_smem > 48 * 1024) {
     const cudaError_t e = cudaFuncSetAttribute(
         count_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cs_smem);
     if (e != cudaSuccess) return e;
   }
+  // the block masks reuse the block-count buffer (one word per block and
+  // expert, which the short path does not otherwise use)
+  uint32_t* masks = reinterpret_cast<uint32_t*>(b.blk_count);
   cudaError_t e = launch_pdl(count_scan_kernel, dim3(1), dim3(1024), cs_smem, stream, ids, k,
                              T, E, k_max, nblk, b.blk_off, b.counts, b.offsets, b.mt_prefix,
-                             b.mt2_prefix, b.totals, b.err);
+                             b.mt2_prefix, b.totals, masks, b.err);
   if (e != cudaSuccess) return e;
-  const size_t smem = static_cast<size_t>(E) * (BLK / 32) * sizeof(uint32_t);
-  if (smem > 48 * 1024) {
-    e = cudaFuncSetAttribute(scatter_kernel<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-    if (e != cudaSuccess) return e;
-  }
-  return launch_pdl(scatter_kernel<BLK>, dim3(nblk), dim3(BLK), smem, stream, ids, k, T, E,
-                    k_max, b.blk_off, b.offsets, b.perm, b.row_of, b.err);
+  int wpt, grid;
+  gather_shape(sizeof(Te) == 4 ? 0 : 1, T, d, num_sms, &wpt, &grid);
+  return launch_pdl(gather_scatter_kernel<Te>, dim3(grid), dim3(256), 0, stream, hidden, ids, k,
+                    static_cast<const uint32_t*>(masks), static_cast<const int32_t*>(b.blk_off),
+                    static_cast<const int32_t*>(b.offsets), E, k_max, cap_rows, T, d, wpt,
+                    b.perm, b.row_of, x_perm, b.err);
 }
 
-cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T, int E,
-                            int k_max, const DispatchBufs& b,
-                            cudaStream_t stream) {
+template <typename Te>
+static cudaError_t launch_gather(const Te* hidden, const int32_t* row_of, const int32_t* k,
+                                 int T, int k_max, int cap_rows, int d, Te* x_perm,
+                                 uint32_t* err, int num_sms, cudaStream_t stream) {
+  int wpt, grid;
+  gather_shape(sizeof(Te) == 4 ? 0 : 1, T, d, num_sms, &wpt, &grid);
+  return launch_pdl(gather_kernel<Te>, dim3(grid), dim3(256), 0, stream, hidden, row_of, k,
+                    k_max, cap_rows, T, d, wpt, x_perm, err);
+}
+
+template <typename Te>
+static cudaError_t dispatch_gather(const Te* hidden, const int32_t* ids, const int32_t* k,
+                                   int T, int E, int k_max, int cap_rows, int d,
+                                   const DispatchBufs& b, Te* x_perm, int num_sms,
+                                   cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
   if (dispatch_block(T) == kDispatchBlockSmall &&
       static_cast<size_t>((T + kDispatchBlockSmall - 1) / kDispatchBlockSmall) * E *
-              sizeof(int) <= kCountScanSmem)
-    return launch_dispatch_small(ids, k, T, E, k_max, b, stream);
-  if (dispatch_block(T) == kDispatchBlockSmall)
-    return launch_dispatch_blk<kDispatchBlockSmall>(ids, k, T, E, k_max, b, stream);
-  return launch_dispatch_blk<kDispatchBlock>(ids, k, T, E, k_max, b, stream);
+              sizeof(uint32_t) <= kCountScanSmem)
+    return launch_dispatch_small(hidden, ids, k, T, E, k_max, cap_rows, d, b, x_perm, num_sms,
+                                 stream);
+  const cudaError_t e =
+      dispatch_block(T) == kDispatchBlockSmall
+          ? launch_dispatch_blk<kDispatchBlockSmall>(ids, k, T, E, k_max, b, stream)
+          : launch_dispatch_blk<kDispatchBlock>(ids, k, T, E, k_max, b, stream);
+  if (e != cudaSuccess) return e;
+  return launch_gather(hidden, b.row_of, k, T, k_max, cap_rows, d, x_perm, b.err, num_sms,
+                       stream);
 }
 
-cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* row_of,
-                               const int32_t* k, int T, int k_max, int cap_rows,
-                               int d, void* x_perm, uint32_t* err, int num_sms,
-                               cudaStream_t stream) {
-  if (T == 0) return cudaSuccess;
-  // warps per token: enough warps for 16 per SM, each segment whole vectors
-  const int row_vecs = d * (dtype == 0 ? 4 : 2) / 16;
-  int wpt = 1;
-  while (wpt < 8 && static_cast<int64_t>(T) * wpt < 16LL * num_sms &&
-         row_vecs % (2 * wpt) == 0)
-    wpt *= 2;
-  const int64_t warps = static_cast<int64_t>(T) * wpt;
-  int grid = static_cast<int>((warps + 7) / 8);
-  if (grid > 16 * num_sms) grid = 16 * num_sms;
+cudaError_t launch_dispatch_gather(int dtype, const void* hidden, const int32_t* ids,
+                                   const int32_t* k, int T, int E, int k_max, int cap_rows,
+                                   int d, const DispatchBufs& b, void* x_perm, int num_sms,
+                                   cudaStream_t stream) {
   if (dtype == 0)
-    return launch_pdl(gather_kernel<float>, dim3(grid), dim3(256), 0, stream,
-                      static_cast<const float*>(hidden), row_of, k, k_max, cap_rows, T, d,
-                      wpt, static_cast<float*>(x_perm), err);
-  return launch_pdl(gather_kernel<__nv_bfloat16>, dim3(grid), dim3(256), 0, stream,
-                    static_cast<const __nv_bfloat16*>(hidden), row_of, k, k_max, cap_rows, T,
-                    d, wpt, static_cast<__nv_bfloat16*>(x_perm), err);
+    return dispatch_gather(static_cast<const float*>(hidden), ids, k, T, E, k_max, cap_rows, d,
+                           b, static_cast<float*>(x_perm), num_sms, stream);
+  return dispatch_gather(static_cast<const __nv_bfloat16*>(hidden), ids, k, T, E, k_max,
+                         cap_rows, d, b, static_cast<__nv_bfloat16*>(x_perm), num_sms, stream);
 }
 
 }  // namespace rx

@@ -107,14 +107,12 @@ inline int64_t dispatch_blocks_alloc(int T) {
   return (ts + kDispatchBlockSmall - 1) / kDispatchBlockSmall +
          (T + kDispatchBlock - 1) / kDispatchBlock;
 }
-cudaError_t launch_dispatch(const int32_t* ids, const int32_t* k, int T,
-                            int E, int k_max, const DispatchBufs& b,
-                            cudaStream_t stream);
-// X_perm[row_of[t, j]] = X[t] for j < k_t.
-cudaError_t launch_gather_rows(int dtype, const void* hidden, const int32_t* row_of,
-                               const int32_t* k, int T, int k_max, int cap_rows,
-                               int d, void* x_perm, uint32_t* err, int num_sms,
-                               cudaStream_t stream);
+// The pair layout (counts, offsets, tile prefixes, perm, row_of) and the
+// gathered rows X_perm[row_of[t, j]] = X[t] for j < k_t.
+cudaError_t launch_dispatch_gather(int dtype, const void* hidden, const int32_t* ids,
+                                   const int32_t* k, int T, int E, int k_max, int cap_rows,
+                                   int d, const DispatchBufs& b, void* x_perm, int num_sms,
+                                   cudaStream_t stream);
 
 // ---- experts: SIMT grouped GEMMs (experts_simt.cu) ------------------------
 // Grouped mode: rows [offsets[e], offsets[e+1]) use expert e; dense mode

@@ -441,9 +441,8 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
                        I32(L.offsets),   I32(L.mt_prefix), I32(L.mt2_prefix),
                        I32(L.perm),      I32(L.row_of),    totals,
                        err};
-    RX_CUDA(rx::launch_dispatch(I32(L.ids), k, T, E, k_max, b, s));
-    RX_CUDA(rx::launch_gather_rows(dtype, hidden, I32(L.row_of), k, T, k_max, cap, d,
-                                   xperm, err, sms, s));
+    RX_CUDA(rx::launch_dispatch_gather(dtype, hidden, I32(L.ids), k, T, E, k_max, cap, d, b,
+                                       xperm, sms, s));
   }
   const bool up = (stages & REFLEX_STAGE_EXPERT_UP) != 0;
   const bool down = (stages & REFLEX_STAGE_EXPERT_DOWN) != 0;
