@@ -77,16 +77,16 @@ def step_launches(dtype: str, T: int, d: int, E: int, shared_inter: int,
     or (bf16, renormalised weights, >= 128 experts, T E >= 2048 x 256,
     d % 128 == 0) the norm
     kernel, the score GEMM and the screened selection; count + scan in one
-    CTA, then the gather, which also places the pairs (short batches whose
-    block masks fit in shared memory), or count, scan, scatter and gather; the
-    gate/up and down GEMMs (and the shared expert's two); the combine.
+    CTA (short batches whose block masks fit in shared memory) or count and
+    scan, then the gather, which also places the pairs; the gate/up and down
+    GEMMs (and the shared expert's two); the combine.
     Memsets are not kernels."""
     n = 1
     screen = (dtype == "bf16" and flags & B.REFLEX_FLAG_RENORM_TOPK and
               not flags & B.REFLEX_FLAG_EXACT_SCORES and d % 128 == 0 and E >= 128 and
               T * E >= 2048 * 256)
     n += 3 if screen else 2
-    n += 1 if T <= 4096 and (T + 31) // 32 * E * 4 <= 160 * 1024 else 3
+    n += 1 if T <= 4096 and (T + 31) // 32 * E * 4 <= 160 * 1024 else 2
     n += 1 + 2 + (2 if shared_inter else 0) + 1
     return n
 

@@ -10,14 +10,11 @@
 //   scan    per expert, exclusive prefix over blocks; per-expert totals;
 //           exclusive prefix over experts = offsets, and over the 128- and
 //           256-row tile counts = tile prefixes for the grouped GEMMs;
-//   scatter rebuilds the block's masks; the row of pair (t, j) is
-//           offsets[e] + block prefix + popcount of lower tokens' bits.
-// A fourth launch gathers X rows into pair order (one warp per token: the
-// hidden row is read once and written to each of its pair rows).  Short
-// batches take two launches: count and scan in one CTA (32-token blocks,
-// one mask word per block and expert, kept in global memory), then the
-// gather, whose warps place their token's pairs from those masks as scatter
-// does.
+//   gather  the row of pair (t, j) is offsets[e] + block prefix + popcount
+//           of the lower tokens' bits in the block's masks (kept in global
+//           memory by count); X rows are copied into pair order on the way.
+// Short batches whose masks fit in one CTA's shared memory take two: count
+// and scan in one CTA, then the gather.
 #include "common.cuh"
 #include "internal.h"
 
@@ -57,12 +54,14 @@ template <int BLK>
 __global__ void __launch_bounds__(BLK)
     count_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ k,
                  int T, int E, int k_max, int32_t* __restrict__ blk_count,
-                 uint32_t* __restrict__ err) {
+                 uint32_t* __restrict__ blk_mask, uint32_t* __restrict__ err) {
   constexpr int kBlk = BLK, kWords = BLK / 32;
   extern __shared__ uint32_t mask[];
   grid_dep_wait();
   grid_dep_launch();
   build_masks<BLK>(mask, ids, k, T, E, k_max, err);
+  uint32_t* gm = blk_mask + static_cast<int64_t>(blockIdx.x) * E * kWords;
+  for (int i = threadIdx.x; i < E * kWords; i += kBlk) gm[i] = mask[i];
   for (int e = threadIdx.x; e < E; e += kBlk) {
     int c = 0;
 #pragma unroll
@@ -212,101 +211,16 @@ __global__ void __launch_bounds__(1024)
   }
 }
 
-template <int BLK>
-__global__ void __launch_bounds__(BLK)
-    scatter_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ k,
-                   int T, int E, int k_max,
-                   const int32_t* __restrict__ blk_off,
-                   const int32_t* __restrict__ offsets,
-                   int32_t* __restrict__ perm, int32_t* __restrict__ row_of,
-                   uint32_t* __restrict__ err) {
-  constexpr int kBlk = BLK, kWords = BLK / 32;
-  extern __shared__ uint32_t mask[];
-  grid_dep_wait();
-  grid_dep_launch();
-  build_masks<BLK>(mask, ids, k, T, E, k_max, nullptr);
-  const int t = blockIdx.x * kBlk + threadIdx.x;
-  if (t >= T) return;
-  const int kt = clamp_k(k[t], k_max < E ? k_max : E);
-  const int w = threadIdx.x >> 5;
-  const uint32_t below = (1u << (threadIdx.x & 31)) - 1u;
-  for (int j = 0; j < k_max; ++j) {
-    const int64_t o = static_cast<int64_t>(t) * k_max + j;
-    int pos = -1;
-    if (j < kt) {
-      const int e = ids[o];
-      if (e >= 0 && e < E) {
-        int local = __popc(mask[e * kWords + w] & below);
-        for (int ww = 0; ww < w; ++ww) local += __popc(mask[e * kWords + ww]);
-        pos = offsets[e] + blk_off[static_cast<int64_t>(blockIdx.x) * E + e] + local;
-        perm[pos] = static_cast<int32_t>(o);
-      }
-    }
-    row_of[o] = pos;
-  }
-}
-
-// Token-order gather: W warps per token (W = 1 for long batches), each
-// reading one 1/W segment of the token's hidden row once (up to 8 16-byte
-// vectors per lane in flight) and writing it to each of the token's k_t pair
-// rows, so every hidden row crosses HBM once however many experts selected
-// it.  Short batches split rows across warps so that every SM gets work.
-template <typename Te>
-__global__ void __launch_bounds__(256)
-    gather_kernel(const Te* __restrict__ x, const int32_t* __restrict__ row_of,
-                  const int32_t* __restrict__ k, int k_max, int cap_rows, int T,
-                  int d, int wpt, Te* __restrict__ xp, uint32_t* __restrict__ err) {
-  constexpr int kVecElems = 16 / sizeof(Te);  // elements per 16-byte vector
-  constexpr int kMaxVec = 8;                  // vectors per lane per pass
-  grid_dep_wait();
-  grid_dep_launch();
-  const int lane = threadIdx.x & 31;
-  const int warps = gridDim.x * 8;
-  const int row_vecs = d / kVecElems;
-  const int seg_vecs = row_vecs / wpt;        // vectors of one warp's segment
-  const int units = T * wpt;
-  for (int u = blockIdx.x * 8 + (threadIdx.x >> 5); u < units; u += warps) {
-    const int t = u / wpt;
-    const int v0 = (u % wpt) * seg_vecs;
-    int kt = k[t];
-    kt = kt < 1 ? 1 : (kt > k_max ? k_max : kt);
-    int my_row = -1;
-    if (lane < kt) {
-      my_row = row_of[static_cast<int64_t>(t) * k_max + lane];
-      if (my_row >= cap_rows) {
-        set_err(err, kErrIndex);
-        my_row = -1;
-      }
-    }
-    const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(t) * d) + v0;
-    for (int base = 0; base < seg_vecs; base += 32 * kMaxVec) {
-      uint4 v[kMaxVec];
-#pragma unroll
-      for (int i = 0; i < kMaxVec; ++i) {
-        const int q = base + lane + 32 * i;
-        if (q < seg_vecs) v[i] = __ldg(src + q);
-      }
-      for (int j = 0; j < kt; ++j) {
-        const int r = __shfl_sync(0xffffffffu, my_row, j);
-        if (r < 0) continue;
-        uint4* dst = reinterpret_cast<uint4*>(xp + static_cast<int64_t>(r) * d) + v0;
-#pragma unroll
-        for (int i = 0; i < kMaxVec; ++i) {
-          const int q = base + lane + 32 * i;
-          if (q < seg_vecs) dst[q] = v[i];
-        }
-      }
-    }
-  }
-}
-
-// Short batches: the scatter step inside the gather.  Lane j of a warp of
-// token t places pair (t, j) at offsets[e] + block prefix + the popcount of
-// the lower tokens' bits in its block's mask word of expert e (the same row
-// as scatter_kernel), the warp of the row's first segment writes perm and
-// row_of, and every warp copies its segment of the hidden row to the pair
-// rows as gather_kernel does.
-template <typename Te>
+// Token-order gather with the scatter step.  W warps per token (W = 1 for
+// long batches), each reading one 1/W segment of the token's hidden row
+// once (up to 8 16-byte vectors per lane in flight) and writing it to each
+// of the token's k_t pair rows, so every hidden row crosses HBM once however
+// many experts selected it; short batches split rows across warps so that
+// every SM gets work.  Lane j of a warp of token t places pair (t, j) at
+// offsets[e] + block prefix + the popcount of the lower tokens' bits in its
+// block's KW mask words of expert e (the pairs of expert e in token order);
+// the warp of the row's first segment writes perm and row_of.
+template <typename Te, int KW>
 __global__ void __launch_bounds__(256)
     gather_scatter_kernel(const Te* __restrict__ x, const int32_t* __restrict__ ids,
                           const int32_t* __restrict__ k, const uint32_t* __restrict__ blk_mask,
@@ -336,9 +250,24 @@ __global__ void __launch_bounds__(256)
       if (lane < kt) {
         const int e = ids[o];
         if (e >= 0 && e < E) {
-          const int64_t bi = static_cast<int64_t>(t / kDispatchBlockSmall) * E + e;
-          const uint32_t below = (1u << (t % kDispatchBlockSmall)) - 1u;
-          my_row = offsets[e] + blk_off[bi] + __popc(blk_mask[bi] & below);
+          const int tb = t % (32 * KW);  // token within its block
+          const int64_t bi = static_cast<int64_t>(t / (32 * KW)) * E + e;
+          const uint32_t below = (1u << (tb & 31)) - 1u;
+          int local;
+          if constexpr (KW == 1) {
+            local = __popc(blk_mask[bi] & below);
+          } else {
+            static_assert(KW == 8, "32- or 256-token blocks");
+            const uint4* mv = reinterpret_cast<const uint4*>(blk_mask + bi * KW);
+            const uint4 m0 = mv[0], m1 = mv[1];
+            const uint32_t m[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+            const int w = tb >> 5;
+            local = 0;
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              local += i < w ? __popc(m[i]) : (i == w ? __popc(m[i] & below) : 0);
+          }
+          my_row = offsets[e] + blk_off[bi] + local;
           if (my_row < 0 || my_row >= cap_rows) {
             set_err(err, kErrIndex);
             my_row = -1;
@@ -389,67 +318,53 @@ void gather_shape(int dtype, int T, int d, int num_sms, int* wpt_out, int* grid_
 
 }  // namespace
 
+// count and scan over BLK-token blocks (the gather places the pairs)
 template <int BLK>
 cudaError_t launch_dispatch_blk(const int32_t* ids, const int32_t* k, int T, int E, int k_max,
                                 const DispatchBufs& b, cudaStream_t stream) {
   const int nblk = (T + BLK - 1) / BLK;
   const size_t smem = static_cast<size_t>(E) * (BLK / 32) * sizeof(uint32_t);
   if (smem > 48 * 1024) {
-    cudaError_t e1 = cudaFuncSetAttribute(count_kernel<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    cudaError_t e2 = cudaFuncSetAttribute(scatter_kernel<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const cudaError_t e1 = cudaFuncSetAttribute(
+        count_kernel<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e1 != cudaSuccess) return e1;
-    if (e2 != cudaSuccess) return e2;
   }
   cudaError_t e = launch_pdl(count_kernel<BLK>, dim3(nblk), dim3(BLK), smem, stream, ids, k, T,
-                             E, k_max, b.blk_count, b.err);
+                             E, k_max, b.blk_count, b.blk_mask, b.err);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(scan_kernel, dim3(1), dim3(1024), 0, stream, b.blk_count, nblk, E, b.blk_off,
-                 b.counts, b.offsets, b.mt_prefix, b.mt2_prefix, b.totals);
-  if (e != cudaSuccess) return e;
-  return launch_pdl(scatter_kernel<BLK>, dim3(nblk), dim3(BLK), smem, stream, ids, k, T, E,
-                    k_max, b.blk_off, b.offsets, b.perm, b.row_of, b.err);
+  return launch_pdl(scan_kernel, dim3(1), dim3(1024), 0, stream, b.blk_count, nblk, E,
+                    b.blk_off, b.counts, b.offsets, b.mt_prefix, b.mt2_prefix, b.totals);
 }
 
 // Short batches whose block masks fit in shared memory: count + scan in one
-// CTA, then the gather, which also places the pairs.
+// CTA.
 constexpr size_t kCountScanSmem = 160 * 1024;
 
-template <typename Te>
-static cudaError_t launch_dispatch_small(const Te* hidden, const int32_t* ids, const int32_t* k,
-                                         int T, int E, int k_max, int cap_rows, int d,
-                                         const DispatchBufs& b, Te* x_perm, int num_sms,
-                                         cudaStream_t stream) {
-  constexpr int BLK = kDispatchBlockSmall;
-  const int nblk = (T + BLK - 1) / BLK;
+static cudaError_t launch_count_scan(const int32_t* ids, const int32_t* k, int T, int E,
+                                    int k_max, const DispatchBufs& b, cudaStream_t stream) {
+  const int nblk = (T + kDispatchBlockSmall - 1) / kDispatchBlockSmall;
   const size_t cs_smem = static_cast<size_t>(nblk) * E * sizeof(uint32_t);
   if (cs_smem > 48 * 1024) {
     const cudaError_t e = cudaFuncSetAttribute(
         count_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cs_smem);
     if (e != cudaSuccess) return e;
   }
-  // the block masks reuse the block-count buffer (one word per block and
-  // expert, which the short path does not otherwise use)
-  uint32_t* masks = reinterpret_cast<uint32_t*>(b.blk_count);
-  cudaError_t e = launch_pdl(count_scan_kernel, dim3(1), dim3(1024), cs_smem, stream, ids, k,
-                             T, E, k_max, nblk, b.blk_off, b.counts, b.offsets, b.mt_prefix,
-                             b.mt2_prefix, b.totals, masks, b.err);
-  if (e != cudaSuccess) return e;
-  int wpt, grid;
-  gather_shape(sizeof(Te) == 4 ? 0 : 1, T, d, num_sms, &wpt, &grid);
-  return launch_pdl(gather_scatter_kernel<Te>, dim3(grid), dim3(256), 0, stream, hidden, ids, k,
-                    static_cast<const uint32_t*>(masks), static_cast<const int32_t*>(b.blk_off),
-                    static_cast<const int32_t*>(b.offsets), E, k_max, cap_rows, T, d, wpt,
-                    b.perm, b.row_of, x_perm, b.err);
+  return launch_pdl(count_scan_kernel, dim3(1), dim3(1024), cs_smem, stream, ids, k, T, E,
+                    k_max, nblk, b.blk_off, b.counts, b.offsets, b.mt_prefix, b.mt2_prefix,
+                    b.totals, b.blk_mask, b.err);
 }
 
-template <typename Te>
-static cudaError_t launch_gather(const Te* hidden, const int32_t* row_of, const int32_t* k,
-                                 int T, int k_max, int cap_rows, int d, Te* x_perm,
-                                 uint32_t* err, int num_sms, cudaStream_t stream) {
+template <typename Te, int KW>
+static cudaError_t launch_gather_scatter(const Te* hidden, const int32_t* ids, const int32_t* k,
+                                         int T, int E, int k_max, int cap_rows, int d,
+                                         const DispatchBufs& b, Te* x_perm, int num_sms,
+                                         cudaStream_t stream) {
   int wpt, grid;
   gather_shape(sizeof(Te) == 4 ? 0 : 1, T, d, num_sms, &wpt, &grid);
-  return launch_pdl(gather_kernel<Te>, dim3(grid), dim3(256), 0, stream, hidden, row_of, k,
-                    k_max, cap_rows, T, d, wpt, x_perm, err);
+  return launch_pdl(gather_scatter_kernel<Te, KW>, dim3(grid), dim3(256), 0, stream, hidden,
+                    ids, k, static_cast<const uint32_t*>(b.blk_mask),
+                    static_cast<const int32_t*>(b.blk_off), static_cast<const int32_t*>(b.offsets),
+                    E, k_max, cap_rows, T, d, wpt, b.perm, b.row_of, x_perm, b.err);
 }
 
 template <typename Te>
@@ -458,18 +373,20 @@ static cudaError_t dispatch_gather(const Te* hidden, const int32_t* ids, const i
                                    const DispatchBufs& b, Te* x_perm, int num_sms,
                                    cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
-  if (dispatch_block(T) == kDispatchBlockSmall &&
-      static_cast<size_t>((T + kDispatchBlockSmall - 1) / kDispatchBlockSmall) * E *
-              sizeof(uint32_t) <= kCountScanSmem)
-    return launch_dispatch_small(hidden, ids, k, T, E, k_max, cap_rows, d, b, x_perm, num_sms,
-                                 stream);
-  const cudaError_t e =
-      dispatch_block(T) == kDispatchBlockSmall
-          ? launch_dispatch_blk<kDispatchBlockSmall>(ids, k, T, E, k_max, b, stream)
-          : launch_dispatch_blk<kDispatchBlock>(ids, k, T, E, k_max, b, stream);
+  cudaError_t e;
+  if (dispatch_block(T) == kDispatchBlockSmall) {
+    e = static_cast<size_t>((T + kDispatchBlockSmall - 1) / kDispatchBlockSmall) * E *
+                    sizeof(uint32_t) <= kCountScanSmem
+            ? launch_count_scan(ids, k, T, E, k_max, b, stream)
+            : launch_dispatch_blk<kDispatchBlockSmall>(ids, k, T, E, k_max, b, stream);
+    if (e != cudaSuccess) return e;
+    return launch_gather_scatter<Te, 1>(hidden, ids, k, T, E, k_max, cap_rows, d, b, x_perm,
+                                        num_sms, stream);
+  }
+  e = launch_dispatch_blk<kDispatchBlock>(ids, k, T, E, k_max, b, stream);
   if (e != cudaSuccess) return e;
-  return launch_gather(hidden, b.row_of, k, T, k_max, cap_rows, d, x_perm, b.err, num_sms,
-                       stream);
+  return launch_gather_scatter<Te, kDispatchBlock / 32>(hidden, ids, k, T, E, k_max, cap_rows,
+                                                        d, b, x_perm, num_sms, stream);
 }
 
 cudaError_t launch_dispatch_gather(int dtype, const void* hidden, const int32_t* ids,

@@ -95,6 +95,7 @@ struct DispatchBufs {
   int32_t* row_of;     // [T*k_max]
   int32_t* totals;     // header: total_pairs, total_mtiles, total_mtiles2
   uint32_t* err;
+  uint32_t* blk_mask;  // [nblk, E, BLK / 32] token bits of each block and expert
 };
 constexpr int kDispatchBlock = 256;       // tokens per dispatch block, large batches
 constexpr int kDispatchBlockSmall = 32;   // tokens per dispatch block up to 4096 tokens
@@ -109,6 +110,12 @@ inline int64_t dispatch_blocks_alloc(int T) {
 }
 // The pair layout (counts, offsets, tile prefixes, perm, row_of) and the
 // gathered rows X_perm[row_of[t, j]] = X[t] for j < k_t.
+// mask words for either block size (monotonic in T, like the block counts)
+inline int64_t dispatch_mask_words_alloc(int T) {
+  const int ts = T < kDispatchSmallT ? T : kDispatchSmallT;
+  return (ts + kDispatchBlockSmall - 1) / kDispatchBlockSmall +
+         static_cast<int64_t>(T + kDispatchBlock - 1) / kDispatchBlock * (kDispatchBlock / 32);
+}
 cudaError_t launch_dispatch_gather(int dtype, const void* hidden, const int32_t* ids,
                                    const int32_t* k, int T, int E, int k_max, int cap_rows,
                                    int d, const DispatchBufs& b, void* x_perm, int num_sms,

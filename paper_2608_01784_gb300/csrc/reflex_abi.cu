@@ -23,7 +23,7 @@ size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 // Byte offsets of every workspace region (all 256-byte aligned).
 struct Layout {
-  size_t hdr, z, wnorm, ids, alpha, blk_count, blk_off, counts, offsets, mt_prefix,
+  size_t hdr, z, wnorm, ids, alpha, blk_count, blk_mask, blk_off, counts, offsets, mt_prefix,
       mt2_prefix, perm, row_of, xperm, amid, ash, ysh, total;
   int64_t cap_rows;
   int nblk;
@@ -60,6 +60,7 @@ Layout make_layout(int32_t dtype, int32_t T, int32_t d, int32_t E,
   L.ids = take(cap * 4);
   L.alpha = take(cap * 4);
   L.blk_count = take(static_cast<size_t>(nblk) * E * 4);
+  L.blk_mask = take(static_cast<size_t>(rx::dispatch_mask_words_alloc(T)) * E * 4);
   L.blk_off = take(static_cast<size_t>(nblk) * E * 4);
   L.counts = take(static_cast<size_t>(E) * 4);
   L.offsets = take(static_cast<size_t>(E + 1) * 4);
@@ -440,7 +441,7 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
     rx::DispatchBufs b{I32(L.blk_count), I32(L.blk_off),   I32(L.counts),
                        I32(L.offsets),   I32(L.mt_prefix), I32(L.mt2_prefix),
                        I32(L.perm),      I32(L.row_of),    totals,
-                       err};
+                       err,              reinterpret_cast<uint32_t*>(ws + L.blk_mask)};
     RX_CUDA(rx::launch_dispatch_gather(dtype, hidden, I32(L.ids), k, T, E, k_max, cap, d, b,
                                        xperm, sms, s));
   }

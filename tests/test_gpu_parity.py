@@ -307,6 +307,8 @@ def test_screened_and_exact_routing_agree_on_the_whole_layer():
     (4096, 256, 256, 512, 0, 6, "random"),  # 1-SM 256-wide tiles, ~48 rows per group
     (4096, 256, 4, 128, 0, 4, "random"),   # CTA-pair (2-SM) GEMMs, ragged groups
     (2048, 512, 8, 256, 0, 4, "max"),      # CTA-pair GEMMs, several n-tiles
+    (4096, 256, 512, 64, 0, 8, "random"),  # block masks past one CTA: 32-token count + scan
+    (5000, 256, 16, 128, 0, 4, "random"),  # 256-token dispatch blocks, ragged last block
 ])
 @pytest.mark.parametrize("simt", [False, True])
 def test_forward_bf16_small(T, d, E, inter, shared, kmax, kmode, simt):
