@@ -52,7 +52,7 @@ METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
 # (profiles/grouped_gemm_llada_moe_T1024.md,
 # profiles/grouped_gemm_pair_llada2_mini_T8192.md); workloads without a
 # capture of the current kernel report null.
-NCU_TRAFFIC_BYTES = {"llada_moe": 561247744, "llada2_mini": 1407363048}
+NCU_TRAFFIC_BYTES = {"llada_moe": 561284352, "llada2_mini": 1407363048}
 
 
 def parse():
