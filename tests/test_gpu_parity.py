@@ -420,19 +420,27 @@ def test_forward_count_out_of_range_flagged():
     assert (rec["ids"][5] >= 0).sum() == cfg.k_max   # clamped, still routed
 
 
-def test_forward_stages_compose():
-    cfg = CFG["llada_moe"]
+# Stages run one per call on one workspace give the bits of one call with
+# every stage (1-SM tiles; CTA-pair tiles with the shared expert; the
+# residual added)
+@pytest.mark.parametrize("name,extra", [
+    ("llada_moe", 0),
+    ("llada2_mini", 0),
+    ("llada_moe", B.REFLEX_FLAG_RESIDUAL),
+])
+def test_forward_stages_compose(name, extra):
+    cfg = CFG[name]
     layer = W.make_layer(cfg, 2)
     k = _k_for(cfg, 2)
     gl = G.GpuLayer(cfg, layer)
-    full, _, _ = gl.forward(k)
+    full, _, _ = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | extra)
     kd = torch.from_numpy(k).cuda()
     out = torch.empty_like(gl.dev["hidden"])
     for st in (B.REFLEX_STAGE_ROUTE, B.REFLEX_STAGE_DISPATCH,
                B.REFLEX_STAGE_EXPERT_UP, B.REFLEX_STAGE_EXPERT_DOWN,
                B.REFLEX_STAGE_COMBINE):
         gl.moe.forward(gl.dev["hidden"], kd, out=out,
-                       flags=B.REFLEX_FLAG_RENORM_TOPK | st)
+                       flags=B.REFLEX_FLAG_RENORM_TOPK | extra | st)
     torch.cuda.synchronize()
     assert np.array_equal(G.to_f32(out), full)
 
