@@ -8,7 +8,7 @@
 // The CTAs are persistent (a few per SM) and walk the tokens in groups; the
 // pair rows, weights and count of the next group are copied into shared
 // memory with cp.async while the current group is summed, so each token costs
-// one round trip for its rows (up to 8 slots in flight per thread) instead of
+// one round trip per 4 slots (their rows loaded back to back) instead of
 // a chain of metadata loads, barriers and row loads.  Sums are fp32 in slot
 // order j = 0, 1, ..., then rounded once to the output type.
 #include "common.cuh"
@@ -19,8 +19,8 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kMaxK = 32;
-constexpr int kBatch = 8;        // slots whose rows are loaded back to back
-constexpr int kCtasPerSm = 4;
+constexpr int kBatch = 4;        // slots whose rows are loaded back to back
+constexpr int kCtasPerSm = 6;
 
 // 8 raw elements: loaded as stored, widened exactly to fp32 when summed.
 template <typename Te>
