@@ -1028,13 +1028,15 @@ cudaError_t logits_dispatch(const __nv_bfloat16* h, const __nv_bfloat16* w, int 
                             int d, int E, float* z, uint32_t* zw, int nz, uint32_t* err,
                             int num_sms, cudaStream_t s, const L2Prefetch& pf) {
   const int64_t per_sm = static_cast<int64_t>(T) * E / (num_sms > 0 ? num_sms : 1);
-  // whole rows resident: 16 x 32 tiles, one CTA per SM, for about 300-640
-  // chains per SM (1024 x 64 scores: 20.8 -> 18.1 us; fewer chains favour
-  // the ring kernel's smaller tiles, more chains need a second wave)
-  using Res = ResCfg<4, 2, 2, 2, 2>;
+  // whole rows resident: 16 x 32 tiles, one CTA of 8 warps per SM (2 x 1
+  // chains per thread), for about 300-640 chains per SM (1024 x 64 scores:
+  // 20.8 -> 18.1 us; 8 warps of 2 x 1 instead of 4 of 2 x 2: step -0.6 us;
+  // fewer chains favour the ring kernel's smaller tiles, more chains need a
+  // second wave)
+  using Res = ResCfg<4, 2, 1, 2, 4>;
   if (per_sm > 300 && per_sm <= 640 && d % kResChunkK == 0 &&
       d / kResChunkK <= kResMaxChunks && Res::smem(d) <= 227 * 1024)
-    return launch_logits_res<4, 2, 2, 2, 2>(h, w, T, d, E, z, zw, nz, err, pf, s);
+    return launch_logits_res<4, 2, 1, 2, 4>(h, w, T, d, E, z, zw, nz, err, pf, s);
   if (per_sm <= 216) return launch_logits_mx<4, 1, 1, 4, 1, 8>(h, w, T, d, E, z, zw, nz, s);
   if (per_sm <= 1080) return launch_logits_mx<4, 1, 2, 4, 1, 8>(h, w, T, d, E, z, zw, nz, s);
   if (per_sm <= 4300) return launch_logits_mx<4, 2, 2, 2, 2, 4, 64>(h, w, T, d, E, z, zw, nz, s);
