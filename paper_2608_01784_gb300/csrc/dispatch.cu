@@ -71,30 +71,49 @@ __global__ void __launch_bounds__(BLK)
 }
 
 // Exclusive scan of one value per thread over a block of 1024 threads.
-__device__ int block_exclusive_scan(int v, int* s_warp, int* total) {
+// Exclusive scans of three values per thread over a block of 1024 threads
+// (one pass: two block barriers for all three).
+struct Scan3 {
+  int a, b, c;
+};
+__device__ Scan3 block_exclusive_scan3(Scan3 v, int (*s_warp)[32], Scan3* total) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  int x = v;
+  Scan3 x = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, x, o);
-    if (lane >= o) x += y;
+    const int ya = __shfl_up_sync(0xffffffffu, x.a, o);
+    const int yb = __shfl_up_sync(0xffffffffu, x.b, o);
+    const int yc = __shfl_up_sync(0xffffffffu, x.c, o);
+    if (lane >= o) {
+      x.a += ya;
+      x.b += yb;
+      x.c += yc;
+    }
   }
-  if (lane == 31) s_warp[wid] = x;
+  if (lane == 31) {
+    s_warp[0][wid] = x.a;
+    s_warp[1][wid] = x.b;
+    s_warp[2][wid] = x.c;
+  }
   __syncthreads();
-  if (wid == 0) {
-    int s = s_warp[lane];
+  if (wid < 3) {
+    int s = s_warp[wid][lane];
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int y = __shfl_up_sync(0xffffffffu, s, o);
       if (lane >= o) s += y;
     }
-    s_warp[lane] = s;  // inclusive prefix of warp totals
+    s_warp[wid][lane] = s;  // inclusive prefix of warp totals
   }
   __syncthreads();
-  const int before = wid > 0 ? s_warp[wid - 1] : 0;
-  *total = s_warp[31];
-  __syncthreads();
-  return before + x - v;
+  Scan3 r;
+  r.a = (wid > 0 ? s_warp[0][wid - 1] : 0) + x.a - v.a;
+  r.b = (wid > 0 ? s_warp[1][wid - 1] : 0) + x.b - v.b;
+  r.c = (wid > 0 ? s_warp[2][wid - 1] : 0) + x.c - v.c;
+  total->a = s_warp[0][31];
+  total->b = s_warp[1][31];
+  total->c = s_warp[2][31];
+  return r;
 }
 
 __global__ void __launch_bounds__(1024)
@@ -102,7 +121,7 @@ __global__ void __launch_bounds__(1024)
                 int32_t* __restrict__ blk_off, int32_t* __restrict__ counts,
                 int32_t* __restrict__ offsets, int32_t* __restrict__ mt_prefix,
                 int32_t* __restrict__ mt2_prefix, int32_t* __restrict__ totals) {
-  __shared__ int s_warp[32];
+  __shared__ int s_warp3[3][32];
   grid_dep_wait();
   grid_dep_launch();
   const int e = threadIdx.x;  // E <= 1024
@@ -123,13 +142,14 @@ __global__ void __launch_bounds__(1024)
     }
     counts[e] = run;
   }
-  int total_pairs, total_tiles;
-  const int off = block_exclusive_scan(e < E ? run : 0, s_warp, &total_pairs);
-  const int tiles = e < E ? (run + kTileM - 1) / kTileM : 0;
-  const int toff = block_exclusive_scan(tiles, s_warp, &total_tiles);
-  int total_tiles2;  // 256-row tiles of the CTA-pair GEMM
-  const int tiles2 = e < E ? (run + 2 * kTileM - 1) / (2 * kTileM) : 0;
-  const int toff2 = block_exclusive_scan(tiles2, s_warp, &total_tiles2);
+  // pairs, 128-row tiles and 256-row tiles (CTA-pair GEMM) per expert
+  Scan3 tot;
+  const Scan3 pre = block_exclusive_scan3(
+      Scan3{e < E ? run : 0, e < E ? (run + kTileM - 1) / kTileM : 0,
+            e < E ? (run + 2 * kTileM - 1) / (2 * kTileM) : 0},
+      s_warp3, &tot);
+  const int off = pre.a, toff = pre.b, toff2 = pre.c;
+  const int total_pairs = tot.a, total_tiles = tot.b, total_tiles2 = tot.c;
   if (e < E) {
     offsets[e] = off;
     mt_prefix[e] = toff;
@@ -159,7 +179,7 @@ __global__ void __launch_bounds__(1024)
                       int32_t* __restrict__ totals, uint32_t* __restrict__ blk_mask,
                       uint32_t* __restrict__ err) {
   extern __shared__ uint32_t s_mask[];  // [nblk][E]: bit = token of the block
-  __shared__ int s_warp[32];
+  __shared__ int s_warp3[3][32];
   grid_dep_wait();
   grid_dep_launch();
   for (int i = threadIdx.x; i < nblk * E; i += 1024) s_mask[i] = 0u;
@@ -190,12 +210,13 @@ __global__ void __launch_bounds__(1024)
     }
     counts[e] = run;
   }
-  int total_pairs, total_tiles, total_tiles2;
-  const int off = block_exclusive_scan(e < E ? run : 0, s_warp, &total_pairs);
-  const int tiles = e < E ? (run + kTileM - 1) / kTileM : 0;
-  const int toff = block_exclusive_scan(tiles, s_warp, &total_tiles);
-  const int tiles2 = e < E ? (run + 2 * kTileM - 1) / (2 * kTileM) : 0;
-  const int toff2 = block_exclusive_scan(tiles2, s_warp, &total_tiles2);
+  Scan3 tot;
+  const Scan3 pre = block_exclusive_scan3(
+      Scan3{e < E ? run : 0, e < E ? (run + kTileM - 1) / kTileM : 0,
+            e < E ? (run + 2 * kTileM - 1) / (2 * kTileM) : 0},
+      s_warp3, &tot);
+  const int off = pre.a, toff = pre.b, toff2 = pre.c;
+  const int total_pairs = tot.a, total_tiles = tot.b, total_tiles2 = tot.c;
   if (e < E) {
     offsets[e] = off;
     mt_prefix[e] = toff;
@@ -244,6 +265,15 @@ __global__ void __launch_bounds__(256)
     const int seg = u % wpt;
     const int v0 = seg * seg_vecs;
     const int kt = clamp_k(k[t], kcap);
+    // the row segment's first vectors do not depend on the pair rows: their
+    // loads overlap the position lookups
+    const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(t) * d) + v0;
+    uint4 v[kMaxVec];
+#pragma unroll
+    for (int i = 0; i < kMaxVec; ++i) {
+      const int q = lane + 32 * i;
+      if (q < seg_vecs) v[i] = __ldg(src + q);
+    }
     int my_row = -1;
     if (lane < k_max) {
       const int64_t o = static_cast<int64_t>(t) * k_max + lane;
@@ -279,13 +309,13 @@ __global__ void __launch_bounds__(256)
         if (my_row >= 0) perm[my_row] = static_cast<int32_t>(o);
       }
     }
-    const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(t) * d) + v0;
     for (int base = 0; base < seg_vecs; base += 32 * kMaxVec) {
-      uint4 v[kMaxVec];
+      if (base > 0) {
 #pragma unroll
-      for (int i = 0; i < kMaxVec; ++i) {
-        const int q = base + lane + 32 * i;
-        if (q < seg_vecs) v[i] = __ldg(src + q);
+        for (int i = 0; i < kMaxVec; ++i) {
+          const int q = base + lane + 32 * i;
+          if (q < seg_vecs) v[i] = __ldg(src + q);
+        }
       }
       for (int j = 0; j < kt; ++j) {
         const int r = __shfl_sync(0xffffffffu, my_row, j);
