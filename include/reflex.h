@@ -227,7 +227,9 @@ typedef struct {
 
 /* Bytes of workspace reflex_moe_forward needs for these shapes (0 if the
  * shapes are invalid).  Sized for the worst case T * k_max pairs, so the
- * forward never reads back the realised sum of k. */
+ * forward never reads back the realised sum of k.  Never decreases as T
+ * grows (other shapes fixed): a workspace sized for T serves every smaller
+ * batch. */
 size_t reflex_moe_workspace_size(int32_t dtype, int32_t T, int32_t d,
                                  int32_t E, int32_t inter,
                                  int32_t shared_inter, int32_t k_max);
@@ -261,6 +263,9 @@ size_t reflex_moe_workspace_size(int32_t dtype, int32_t T, int32_t d,
  *                   error word gets REFLEX_EKRANGE and the count is clamped).
  *   flags           REFLEX_FLAG_* | REFLEX_STAGE_* (see above).
  *   workspace       >= reflex_moe_workspace_size(...) bytes, 256-B aligned.
+ *   ws_bytes        the workspace's size in bytes; smaller than
+ *                   reflex_moe_workspace_size(...) for this call's shapes:
+ *                   REFLEX_EWORKSPACE, nothing enqueued.
  *   out             [T, d] output.
  *   rec             HOST struct, nullable: receives device pointers into the
  *                   workspace (no copy is made).

@@ -120,14 +120,11 @@ class MoELayer:
             raise ValueError("more tokens than the workspace was sized for")
         if out is None:
             out = torch.empty((T, self.d), dtype=self.tdtype, device=hidden.device)
-        ws_bytes = B.reflex_moe_workspace_size(self.dtype, T, self.d, self.E,
-                                               self.inter, self.shared_inter,
-                                               self.k_max)
         B.reflex_moe_forward(self.dtype, hidden, self.w["w_router"],
                              self.w["w_gate_up"], self.w["w_down"],
                              self.w.get("shared_gate_up"), self.w.get("shared_down"),
                              self.shared_inter, k, T, self.d, self.E, self.inter,
-                             self.k_max, flags, self.ws, ws_bytes, out, self.rec,
+                             self.k_max, flags, self.ws, self.ws_bytes, out, self.rec,
                              stream, check)
         self._T = T
         return out
@@ -149,16 +146,13 @@ class MoELayer:
         k_out = torch.empty(T, dtype=torch.int32, device=dev) if k_out is None else k_out
         k_sum = torch.zeros(1, dtype=torch.int64, device=dev) if k_sum is None else k_sum
         status = torch.zeros(1, dtype=torch.int32, device=dev) if status is None else status
-        ws_bytes = B.reflex_moe_workspace_size(self.dtype, T, self.d, self.E,
-                                               self.inter, self.shared_inter,
-                                               self.k_max)
         B.reflex_step(state["conf1"], state["conf2"], state["hist_len"], state["masked"],
                       state["block_id"], state["seq_offsets"], state["active_block"],
                       nseq, params, k_out, k_sum, status, self.dtype, hidden,
                       self.w["w_router"], self.w["w_gate_up"], self.w["w_down"],
                       self.w.get("shared_gate_up"), self.w.get("shared_down"),
                       self.shared_inter, T, self.d, self.E, self.inter, self.k_max,
-                      flags, self.ws, ws_bytes, out, self.rec, stream, check)
+                      flags, self.ws, self.ws_bytes, out, self.rec, stream, check)
         self._T = T
         return out, k_out, k_sum, status
 

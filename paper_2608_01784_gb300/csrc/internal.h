@@ -77,6 +77,20 @@ inline int screen_splits(int T, int E, int d) {
   while (s < 16 && mt * nt * s * 2 <= 152 && nkb % (2 * s) == 0) s *= 2;
   return s;
 }
+// Rows of the workspace's score region for the screen GEMM's slices: s T,
+// and never fewer than for a smaller batch (s falls as T adds tiles, and a
+// workspace sized for a batch must serve every smaller one).  A batch of m
+// full 128-row tiles has the most rows among those of m tiles; beyond 152
+// tiles s = 1.
+inline int64_t screen_z_rows(int T, int E, int d) {
+  int64_t rows = static_cast<int64_t>(screen_splits(T, E, d)) * T;
+  const int64_t mt = (T + 127) / 128;
+  for (int64_t m = 1; m < mt && m <= 152; ++m) {
+    const int64_t r = screen_splits(static_cast<int>(m * 128), E, d) * m * 128;
+    if (r > rows) rows = r;
+  }
+  return rows;
+}
 // ids/alpha [T, k_max] from z and the counts k.
 cudaError_t launch_router_select(const float* z, const int32_t* k, int T,
                                  int E, int k_max, bool renorm, int32_t* ids,

@@ -54,8 +54,8 @@ Layout make_layout(int32_t dtype, int32_t T, int32_t d, int32_t E,
   };
   L.hdr = take(sizeof(WsHeader));
   // bf16: room for the screen GEMM's split-K slices of the scores
-  const int zslices = dtype == REFLEX_DTYPE_F32 ? 1 : rx::screen_splits(T, E, d);
-  L.z = take(static_cast<size_t>(zslices) * T * E * 4);
+  const int64_t zrows = dtype == REFLEX_DTYPE_F32 ? T : rx::screen_z_rows(T, E, d);
+  L.z = take(static_cast<size_t>(zrows) * E * 4);
   L.wnorm = take(static_cast<size_t>(E) * 4);
   L.ids = take(cap * 4);
   L.alpha = take(cap * 4);

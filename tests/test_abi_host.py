@@ -78,6 +78,26 @@ def test_workspace_size(lib):
     assert ws(7, 1024, 2048, 64, 1024, 0, 12) == 0    # dtype
 
 
+def test_workspace_size_never_shrinks_with_more_tokens(lib):
+    # a workspace sized for a batch serves every smaller one (MoELayer sizes
+    # it once for max_tokens), across the switch from 32- to 256-token
+    # dispatch blocks at 4096 tokens and the router-screen regions
+    from paper_2608_01784_gb300 import _binding as B
+    ws = B.reflex_moe_workspace_size
+    # every T up to 12000 (the score region's split count falls at 128-row
+    # tile boundaries such as 512 -> 513 tokens with 256 experts), then a
+    # sample up to 65536
+    Ts = list(range(0, 12001)) + list(range(12001, 65537, 997)) + [65536]
+    for dtype, d, E, inter, shared in [(1, 2048, 64, 1024, 0), (1, 2048, 256, 512, 512),
+                                       (1, 2048, 128, 1024, 0), (0, 256, 8, 128, 0),
+                                       (1, 512, 160, 256, 0)]:
+        prev = 0
+        for T in Ts:
+            cur = ws(dtype, T, d, E, inter, shared, 12)
+            assert cur >= prev, (dtype, d, E, T, prev, cur)
+            prev = cur
+
+
 def test_host_rejections_enqueue_nothing(lib):
     from paper_2608_01784_gb300 import _binding as B
     p = B.reflex_default_params()
