@@ -409,6 +409,27 @@ def test_forward_without_renorm():
     assert rel <= G.F32_REL_L2 and mx <= G.F32_MAX_ABS
 
 
+def test_smaller_batch_in_a_larger_workspace():
+    # a layer sized for 513 tokens runs 512 (256 experts: the score region's
+    # split count falls from 512 to 513 tokens) and matches a layer sized
+    # for 512 bit for bit
+    T, d, E, inter, kmax = 512, 2048, 256, 128, 8
+    cfg, layer = _bf16_case(T, d, E, inter, 0, kmax, seed=41, weight_std=0.02)
+    dl = api.layer_to_device(layer, cfg.dtype)
+    k = torch.from_numpy(np.random.default_rng(41).integers(1, kmax + 1, T)
+                         .astype(np.int32)).cuda()
+    outs = []
+    for max_tokens in (T, T + 1):
+        moe = api.MoELayer(dl, dtype="bf16", d=d, E=E, inter=inter, shared_inter=0,
+                           k_max=kmax, max_tokens=max_tokens)
+        assert moe.ws_bytes >= B.reflex_moe_workspace_size(B.REFLEX_DTYPE_BF16, T, d, E,
+                                                           inter, 0, kmax)
+        outs.append(moe.forward(dl["hidden"], k).clone())
+        torch.cuda.synchronize()
+        assert moe.status() == B.REFLEX_OK
+    assert torch.equal(outs[0].view(torch.int16), outs[1].view(torch.int16))
+
+
 def test_forward_count_out_of_range_flagged():
     cfg = CFG["tiny_fp32"]
     layer = W.make_layer(cfg, 0)
