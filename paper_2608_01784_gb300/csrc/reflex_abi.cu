@@ -218,7 +218,7 @@ cudaError_t launch_alloc(const AllocCall& c, int32_t T, cudaStream_t s, bool alo
 
 extern "C" {
 
-int reflex_abi_version(void) { return 111; }
+int reflex_abi_version(void) { return 112; }
 
 const char* reflex_status_string(int s) {
   switch (s) {
