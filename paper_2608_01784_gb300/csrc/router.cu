@@ -40,16 +40,8 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// 8 raw elements -> fp32 (exact widening).
-__device__ __forceinline__ void widen8(const uint8_t* p, float* f, const __nv_bfloat16*) {
-  const uint4 v = *reinterpret_cast<const uint4*>(p);
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    f[2 * i] = __uint_as_float(w[i] << 16);
-    f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
-  }
-}
+// 8 raw fp32 elements (the fp32 score kernels; bf16 scores use the mixed-
+// precision fma on raw operands).
 __device__ __forceinline__ void widen8(const uint8_t* p, float* f, const float*) {
   const float4 a = *reinterpret_cast<const float4*>(p);
   const float4 b = *reinterpret_cast<const float4*>(p + 16);
@@ -801,7 +793,7 @@ __global__ void __launch_bounds__(256)
 // lane), the expert row from L2.  (A ring keeping 8-16 expert-row loads in
 // flight per lane made short batches faster but cost occupancy at 8192 and
 // more tokens, where the screen is used.)
-constexpr int kRing = 16;  // d must be a multiple of 8 kRing
+constexpr int kScreenDMultiple = 128;  // d of the screened path (as tested)
 __device__ __forceinline__ float chain_bf16(const uint4* __restrict__ hs,
                                             const __nv_bfloat16* __restrict__ we, int d) {
   const uint4* wv = reinterpret_cast<const uint4*>(we);
@@ -1075,7 +1067,7 @@ cudaError_t launch_router_screen_select(const __nv_bfloat16* h, const __nv_bfloa
                                         int d, int k_max, int32_t* ids, float* alpha,
                                         uint32_t* err, cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
-  if (d % (8 * kRing) != 0 || E > 1024 || k_splits < 1) return cudaErrorInvalidValue;
+  if (d % kScreenDMultiple != 0 || E > 1024 || k_splits < 1) return cudaErrorInvalidValue;
   const size_t smem = static_cast<size_t>(kScreenWarps) * d * 2;  // bf16 token rows
   const double u = 1.0 / 16777216.0;
   const double gamma = d * u / (1.0 - d * u);
