@@ -171,3 +171,19 @@ def test_step_host_rejections(lib):
     lib.reflex_default_params(ctypes.byref(bad))
     bad.q = 0.75                                         # q outside (0, 1/2]
     assert step(params=ctypes.byref(bad)) == B.REFLEX_EINVAL
+
+
+def test_step_launch_counts_of_the_bench_layers():
+    # the kernels of one reflex_step as the ncu launch lists show them:
+    # LLaDA-MoE layer (count, scores, selection, count + scan, gather, two
+    # GEMMs, combine), LLaDA2.0-mini layer (count, norms, score GEMM,
+    # screened selection, count, scan, gather, four GEMMs, combine), 32 x 1024
+    # layer (count, scores, selection, count, scan, gather, two GEMMs, combine)
+    from paper_2608_01784_gb300 import _binding as B
+    from paper_2608_01784_gb300 import api
+    assert api.step_launches("bf16", 1024, 2048, 64, 0) == 8
+    assert api.step_launches("bf16", 8192, 2048, 256, 512) == 12
+    assert api.step_launches("bf16", 32768, 2048, 64, 0) == 9
+    # exact scores: the screen's three kernels become scores + selection
+    exact = B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_FLAG_EXACT_SCORES
+    assert api.step_launches("bf16", 8192, 2048, 256, 512, flags=exact) == 11
