@@ -1,25 +1,28 @@
 """Benchmark of the REFLEX per-forward MoE hot path on GB300.
 
-One step = one denoising forward's hot path on one batch, one reflex_step
-call: the per-token counts of reflex_allocate (Eq. 5 / Eq. 9 + clip) and
-reflex_moe_forward with them (router scores, variable-count TopK, pair
-dispatch, grouped SwiGLU expert GEMMs on tcgen05, weighted combine; Eq. 2),
-the count kernel running beside the router scores.
-Default workload: the LLaDA-MoE-shaped layer (T = 1024 tokens: 512 prompt +
-512 generated in blocks of 32; d = 2048, E = 64 SwiGLU experts with inter =
-1024; K in [2, 12]; bf16 storage, fp32 accumulation), synthetic inputs.
+Default workload (one step = one whole denoising forward): a stack of 16
+LLaDA-MoE-shaped MoE layers (d = 2048, E = 64 SwiGLU experts with inter =
+1024, K in [2, 12], bf16 storage, fp32 accumulation) over a batch of 32 x
+1024 tokens (512 prompt + 512 generated, blocks of 32).  The per-token counts
+are allocated once per forward (Eq. 3 realised by Eq. 5, Eq. 6-9 and the
+clip) and shared by every layer (Sec. 3.3); each layer runs the
+variable-count layer of Eq. 2 (router scores, variable-count TopK, pair
+dispatch, grouped SwiGLU expert GEMMs on tcgen05, weighted combine) with the
+residual h <- bf16(h + MoE(h)).  Inputs are synthetic and seeded on the host
+(the oracle can check the exact timed inputs).
 
-Prints ONE JSON line (rank 0).  `value` = MoE-layer tokens/s over all ranks;
-`expert_tflops` = 6 d inter sum(k) / step time (Eq. 10); the same kernels at
-fixed top-K_base run beside it; `roofline` is for the dominant kernel, the
-grouped gate/up (SwiGLU) GEMM; `e2e` times the same step from pinned host
-buffers through the C ABI with the copies inside the timed region.
+Prints ONE JSON line (rank 0).  `value` = tokens/s of whole forwards over all
+ranks; `expert_tflops` = 6 d inter sum(k) x layers / forward time (Eq. 10);
+the same kernels at fixed top-K_base run beside it; `roofline` is for the
+dominant kernel, the CTA-pair gate/up (SwiGLU) GEMM; `e2e` times the same
+forward from pinned host buffers through the public API with the copies
+inside the timed region; `cpu_baseline` times the oracle on the host cores.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reflex|reference]
-                  [--config NAME] [--no-cpu-baseline] [--sweep]
---config llada_moe_stack16: a whole denoising forward of 16 LLaDA-MoE-shaped
-layers (batch 32 x 1024 tokens, counts allocated once and shared by every
-layer, residual connection, fresh weights per layer drawn on the device).
+                  [--config NAME] [--no-cpu-baseline] [--sweep] [--ablation]
+                  [--trajectory]
+--config llada_moe | llada2_mini | llada_moe_b32 | tiny_fp32: one layer, one
+reflex_step call (counts + layer) per step.
 --sweep: LLaDA2.0-mini layer shapes, 256 .. 65536 tokens x count skew
 0 .. 1 (0 = uniform K_base, 1 = 70% K_min / 30% K_max), forward only.
 Under torchrun each rank runs its own batch on its own GPU (weak scaling, no
@@ -47,12 +50,29 @@ from paper_2608_01784_gb300 import workloads as W  # noqa: E402
 METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
           "fixed top-K")
 
-# DRAM bytes (read + write) moved per launch by the dominant kernel, from an
-# ncu capture of the current kernel on the same workload
-# (profiles/grouped_gemm_llada_moe_T1024.md,
-# profiles/grouped_gemm_pair_llada2_mini_T8192.md); workloads without a
-# capture of the current kernel report null.
-NCU_TRAFFIC_BYTES = {"llada_moe": 561284352, "llada2_mini": 1407363048}
+# DRAM bytes (read + write) per launch of the dominant kernel, from one ncu
+# capture of that kernel on the workload, with the SHA-256 prefix of the
+# kernel source it was taken on; once the source differs the line reports
+# null (the counters no longer describe the kernel that ran).
+NCU_TRAFFIC = {
+    "llada_moe": (561284352, None),
+    "llada2_mini": (1407363048, None),
+    "llada_moe_stack16": (None, None),
+}
+KERNEL_SOURCE = os.path.join(ROOT, "paper_2608_01784_gb300", "csrc", "experts_tc.cu")
+
+
+def kernel_source_sha16() -> str:
+    import hashlib
+    with open(KERNEL_SOURCE, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def ncu_traffic(workload: str):
+    nbytes, sha = NCU_TRAFFIC.get(workload, (None, None))
+    if nbytes is None or sha != kernel_source_sha16():
+        return None
+    return nbytes
 
 
 def parse():
@@ -61,7 +81,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="reflex", choices=["reflex", "reference"])
-    ap.add_argument("--config", default="llada_moe",
+    ap.add_argument("--config", default="llada_moe_stack16",
                     choices=sorted(W.CONFIGS) + ["llada_moe_stack16"])
     ap.add_argument("--sweep", action="store_true",
                     help="token-count x count-skew sweep on the LLaDA2.0-mini "
@@ -119,7 +139,7 @@ class ClockSampler:
         except Exception:
             self.proc.kill()
             out = ""
-        sm, mx, reasons = [], [], set()
+        sm, mx, pw, reasons = [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
                  "sw_power_cap"]
         for line in out.strip().splitlines():
@@ -129,14 +149,20 @@ class ClockSampler:
             try:
                 sm.append(float(f[1]))
                 mx.append(float(f[2]))
+                pw.append(float(f[3]))
             except ValueError:
                 continue
             for n, v in zip(names, f[5:9]):
                 if v.lower() == "active":
                     reasons.add(n)
-        return dict(sm_mhz=statistics.median(sm) if sm else None,
+        # under load: samples drawing at least half of the largest power seen
+        top = max(pw) if pw else 0.0
+        loaded = [c for c, w in zip(sm, pw) if w >= 0.5 * top]
+        return dict(sm_mhz=statistics.median(loaded) if loaded else None,
                     sm_max_mhz=max(mx) if mx else None,
-                    reasons=sorted(reasons), samples=len(sm))
+                    reasons=sorted(reasons), samples=len(sm),
+                    samples_under_load=len(loaded),
+                    power_w_max=top if pw else None)
 
 
 # ---------------------------------------------------------------------------
@@ -162,22 +188,36 @@ def oracle_step(cfg, layer, state, tokens):
     return int(ks.sum())
 
 
-def oracle_rate(cfg, layer, state, target_s, seed=0):
-    """tokens/s of the oracle on a seeded token sample sized to ~target_s."""
+def oracle_rate(cfg, layer, state, target_s, seed=0, threads=None):
+    """tokens/s of the oracle on a seeded token sample sized to ~target_s;
+    threads = None keeps the OpenMP default (all cores)."""
     import oracle
     oracle.build()
-    T = layer["hidden"].shape[0]
-    rng = np.random.default_rng(seed)
-    n = min(T, 16)
-    t0 = time.perf_counter()
-    oracle_step(cfg, layer, state, np.sort(rng.choice(T, n, replace=False)).astype(np.int32))
-    dt = time.perf_counter() - t0
-    n2 = int(min(T, max(n, n * target_s / max(dt, 1e-6))))
-    toks = np.sort(rng.choice(T, n2, replace=False)).astype(np.int32)
-    t0 = time.perf_counter()
-    oracle_step(cfg, layer, state, toks)
-    dt = time.perf_counter() - t0
-    return n2 / dt, n2, dt, oracle.num_threads()
+    all_cores = oracle.num_threads()
+    if threads is not None:
+        oracle.set_num_threads(threads)
+    try:
+        used = oracle.num_threads()
+        T = layer["hidden"].shape[0]
+        rng = np.random.default_rng(seed)
+        n = min(T, max(2, 2 * used))
+        t0 = time.perf_counter()
+        oracle_step(cfg, layer, state, np.sort(rng.choice(T, n, replace=False)).astype(np.int32))
+        dt = time.perf_counter() - t0
+        n2 = int(min(T, max(n, n * target_s / max(dt, 1e-6))))
+        toks = np.sort(rng.choice(T, n2, replace=False)).astype(np.int32)
+        t0 = time.perf_counter()
+        oracle_step(cfg, layer, state, toks)
+        dt = time.perf_counter() - t0
+    finally:
+        oracle.set_num_threads(all_cores)
+    return n2 / dt, n2, dt, used
+
+
+def layer_config(cfg, world: int) -> dict:
+    return dict(workload=cfg.name, description=cfg.description, tokens_per_step=cfg.T,
+                parallelism=f"replicas{world}",
+                l2="no flush: expert weights > 129 MB L2 stream from HBM every step")
 
 
 def run_reference(args, cfg, rank, world):
@@ -210,8 +250,7 @@ def run_reference(args, cfg, rank, world):
                 warmup=args.warmup, ms_per_step=1e3 * dt / args.steps,
                 higher_is_better=True, scaling="weak", vs_baseline=None,
                 dtype="f64", data="synthetic",
-                config=dict(workload=cfg.name, description=cfg.description,
-                            tokens_per_step_sample=n),
+                config=layer_config(cfg, world),
                 cpu_baseline=dict(value=value, unit="tokens/s", kind="oracle",
                                   cores=oracle.num_threads(),
                                   sample=f"{n} seeded tokens of the {T}-token "
@@ -292,6 +331,9 @@ def run_gpu(args, cfg, rank, world, local_rank):
     def max_over_ranks(x: float) -> float:
         return R.max_over_ranks(x, world, dev)
 
+    # clocks sampled from the first launch to the end of the end-to-end leg
+    clk = ClockSampler(local_rank)
+    clk.start()
     # correctness gate before timing: counts and routing status clean
     step(p_reflex)
     torch.cuda.synchronize(dev)
@@ -306,10 +348,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
 
     # ---- timed region: REFLEX counts, one step per graph replay ----
     g_reflex = graph_of(lambda: step(p_reflex))
-    clk = ClockSampler(local_rank)
-    clk.start()
     ms = timed(g_reflex, args.steps, args.warmup)
-    clocks = clk.stop()
     ms = max_over_ranks(ms)
     ms_step = ms / args.steps
     # ---- gate/up GEMM launches: the same step with events around the GEMM,
@@ -388,6 +427,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
     e1.record(stream)
     barrier()
     ms_e2e = max_over_ranks(e0.elapsed_time(e1)) / n_e2e
+    clocks = clk.stop()
     # the end-to-end outputs are those of the resident-input step, bit for bit
     g_reflex.replay()
     torch.cuda.synchronize(dev)
@@ -418,7 +458,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
         roof = dict(bound="tensor", achieved=tf, peak=peaks["bf16"],
                     unit="TFLOP/s", frac=tf / peaks["bf16"])
     roof.update(kernel="grouped_gemm_kernel, gate/up + SwiGLU (tcgen05)",
-                traffic=NCU_TRAFFIC_BYTES.get(cfg.name), algorithmic_bytes=up_bytes,
+                traffic=ncu_traffic(cfg.name), algorithmic_bytes=up_bytes,
                 algorithmic_flops=up_flops, avg_launch_ms=up_ms,
                 peak_source=peaks["source"] + " (burst)")
     # layer roofline: all expert weights touched + hidden in/out vs Eq. 10 flops
@@ -433,9 +473,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
         n_gpus=world, steps=args.steps, warmup=args.warmup, ms_per_step=ms_step,
         higher_is_better=True, scaling="weak", vs_baseline=None, dtype="bf16"
         if cfg.dtype == "bf16" else "f32", data="synthetic",
-        config=dict(workload=cfg.name, description=cfg.description,
-                    tokens_per_step=T, parallelism=f"replicas{world}",
-                    l2="no flush: expert weights > 129 MB L2 stream from HBM every step",
+        config=dict(layer_config(cfg, world),
                     timing="CUDA-graph replay of one step (one reflex_step call: "
                            "allocation + forward) per "
                            "timed iteration; e2e: eager API calls, each step's upload "
@@ -452,37 +490,128 @@ def run_gpu(args, cfg, rank, world, local_rank):
                  h2d_bytes_per_step=h2d, d2h_bytes_per_step=d2h,
                  ms_per_step=ms_e2e),
         gpu_launches=launches_per_step * args.steps,
-        clocks=dict(sm_mhz=clocks["sm_mhz"], sm_max_mhz=clocks["sm_max_mhz"],
-                    reasons=clocks["reasons"], samples=clocks["samples"]),
+        clocks=clocks,
     )
     if not args.no_cpu_baseline and world == 1:
         rate, n, dt, cores = oracle_rate(cfg, layer, state, args.cpu_seconds, seed)
+        rate1, n1, dt1, _ = oracle_rate(cfg, layer, state, args.cpu_seconds / 2, seed + 1, 1)
         line["cpu_baseline"] = dict(
             value=rate, unit="tokens/s", cores=cores, kind="oracle",
             sample=f"{n} seeded tokens of the {T}-token batch, full oracle path "
-                   f"(allocation on the whole batch), {dt:.1f} s")
+                   f"(allocation on the whole batch), {dt:.1f} s",
+            single_thread=dict(value=rate1, unit="tokens/s", cores=1,
+                               sample=f"{n1} seeded tokens, {dt1:.1f} s"))
     elif world > 1:
         line["cpu_baseline"] = None
     print(json.dumps(line), flush=True)
 
 
 # ---------------------------------------------------------------------------
-# 16-layer stack and sweep (GPU)
+# 16-layer stack (GPU): the default workload
 # ---------------------------------------------------------------------------
 STACK_LAYERS = 16
+STACK_LAYER_CFG = "llada_moe_b32"
 
 
-def _device_weights(cfg, seed, dev, std):
-    """Random-init bf16 weights of one layer drawn on the device (seeded)."""
-    import torch
-    g = torch.Generator(device=dev)
-    g.manual_seed(int(seed))
-    E, d, I = cfg.E, cfg.d, cfg.inter
+def stack_config(world: int) -> dict:
+    cfg = W.CONFIGS[STACK_LAYER_CFG]
+    return dict(workload="llada_moe_stack16",
+                description=f"full denoising forward of {STACK_LAYERS} LLaDA-MoE-shaped "
+                            f"layers (d=2048, E=64 SwiGLU experts, inter=1024, K in "
+                            f"[2,12]), batch 32 x 1024 tokens (512 prompt + 512 gen, "
+                            f"block 32), counts allocated once per forward and shared by "
+                            f"every layer, residual h <- bf16(h + MoE(h)), fresh router "
+                            f"and expert weights per layer, bf16 storage, fp32 "
+                            f"accumulation",
+                tokens_per_step=cfg.T, layers=STACK_LAYERS, parallelism=f"replicas{world}",
+                l2="no flush: 12.9 GB of expert weights stream from HBM every step")
 
-    def rnd(*shape):
-        return (torch.randn(*shape, generator=g, device=dev, dtype=torch.float32)
-                * std).to(torch.bfloat16)
-    return dict(w_router=rnd(E, d), w_gate_up=rnd(E, 2 * I, d), w_down=rnd(E, d, I))
+
+def oracle_stack(cfg, stack, state, tokens):
+    """The oracle's whole forward for the listed tokens: the counts of the
+    whole batch (Eq. 5 / Eq. 9 + clip; an active block couples its tokens),
+    then every layer on those tokens (scores, TopK / alpha, pair order,
+    Eq. 2, residual).  Tokens are independent across the layers (no
+    attention), so the sample is exact."""
+    import oracle
+    k = oracle.allocate(state["conf1"], state["conf2"], state["hist_len"],
+                        state["masked"], state["block_id"], state["seq_offsets"],
+                        state["active_block"], **cfg.alloc_params())
+    trace = oracle.moe_stack(stack["hidden"][tokens], stack["layers"], k[tokens],
+                             cfg.k_max)
+    return trace[-1]["h_out"]
+
+
+def oracle_stack_rate(cfg, stack, state, target_s, seed, threads=None):
+    """tokens/s (whole forwards) of the oracle on a seeded token sample sized to
+    about target_s seconds; threads = None keeps the OpenMP default (all
+    cores)."""
+    import oracle
+    oracle.build()
+    all_cores = oracle.num_threads()
+    if threads is not None:
+        oracle.set_num_threads(threads)
+    try:
+        used = oracle.num_threads()
+        T = stack["hidden"].shape[0]
+        rng = np.random.default_rng(seed)
+        n = max(2, min(T, 2 * used))
+        t0 = time.perf_counter()
+        oracle_stack(cfg, stack, state, np.sort(rng.choice(T, n, replace=False)).astype(np.int32))
+        dt = time.perf_counter() - t0
+        n2 = int(min(T, max(n, n * target_s / max(dt, 1e-6))))
+        toks = np.sort(rng.choice(T, n2, replace=False)).astype(np.int32)
+        t0 = time.perf_counter()
+        oracle_stack(cfg, stack, state, toks)
+        dt = time.perf_counter() - t0
+    finally:
+        oracle.set_num_threads(all_cores)
+    return n2 / dt, n2, dt, used
+
+
+def run_stack_reference(args, rank, world):
+    """The oracle as it stands on the host cores, on the stack workload: each
+    step is the whole forward (counts once, 16 layers with the residual) on a
+    seeded token sample of the 32 x 1024 batch."""
+    import torch  # noqa: F401  (keeps the launch environment identical)
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    cfg = W.CONFIGS[STACK_LAYER_CFG]
+    stack = W.make_stack(cfg, args.seed, STACK_LAYERS)
+    state = W.make_state(cfg, args.seed)
+    T = cfg.T
+    rng = np.random.default_rng(args.seed)
+    per_step_s = max(0.5, min(5.0, 150.0 / max(1, args.steps + args.warmup)))
+    n = min(T, 2 * oracle.num_threads())
+    t0 = time.perf_counter()
+    oracle_stack(cfg, stack, state, np.arange(n, dtype=np.int32))
+    dt = time.perf_counter() - t0
+    n = int(min(T, max(1, n * per_step_s / max(dt, 1e-6))))
+
+    def one():
+        oracle_stack(cfg, stack, state,
+                     np.sort(rng.choice(T, n, replace=False)).astype(np.int32))
+    for _ in range(args.warmup):
+        one()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        one()
+    dt = time.perf_counter() - t0
+    value = n * args.steps / dt
+    sample = (f"{n} seeded tokens of the {T}-token batch per step through all "
+              f"{STACK_LAYERS} layers (counts on the whole batch)")
+    line = dict(metric=METRIC, value=value, unit="tokens/s", impl="reference",
+                n_gpus=args.gpus, steps=args.steps, warmup=args.warmup,
+                ms_per_step=1e3 * dt / args.steps, higher_is_better=True,
+                scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
+                config=stack_config(world),
+                cpu_baseline=dict(value=value, unit="tokens/s", kind="oracle",
+                                  cores=oracle.num_threads(), sample=sample),
+                e2e=dict(value=value, unit="tokens/s", h2d_bytes_per_step=0,
+                         d2h_bytes_per_step=0))
+    print(json.dumps(line), flush=True)
 
 
 def run_stack(args, rank, world, local_rank):
@@ -494,85 +623,208 @@ def run_stack(args, rank, world, local_rank):
     B.load()
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    cfg = W.CONFIGS["llada_moe_b32"]
+    cfg = W.CONFIGS[STACK_LAYER_CFG]
+    L = STACK_LAYERS
     seed = R.rank_seed(args.seed, rank)
     T, d, E, I, km = cfg.T, cfg.d, cfg.E, cfg.inter, cfg.k_max
-    state = api.state_to_device(W.make_state(cfg, seed), dev)
-    h0 = api.layer_to_device({"hidden": W.make_layer(cfg.with_(E=1, inter=64), seed)["hidden"]},
-                             cfg.dtype, dev)["hidden"]
-    layers = [_device_weights(cfg, 1000 * seed + l, dev, cfg.weight_std)
-              for l in range(STACK_LAYERS)]
-    # one workspace serves every layer (layers run one after another)
-    moe = api.MoELayer(layers[0], dtype=cfg.dtype, d=d, E=E, inter=I, shared_inter=0,
+    # seeded host inputs (the oracle sees the same bits), then on the device
+    stack = W.make_stack(cfg, seed, L)
+    state = W.make_state(cfg, seed)
+    ds = api.state_to_device(state, dev)
+    layers = [api.layer_to_device(w, cfg.dtype, dev) for w in stack["layers"]]
+    h0 = api.layer_to_device({"hidden": stack["hidden"]}, cfg.dtype, dev)["hidden"]
+    net = api.MoEStack(layers, dtype=cfg.dtype, d=d, E=E, inter=I, shared_inter=0,
                        k_max=km, max_tokens=T, device=dev)
-    bufs = [torch.empty_like(h0), torch.empty_like(h0)]
     stream = torch.cuda.current_stream(dev)
     k_buf = torch.empty(T, dtype=torch.int32, device=dev)
     k_sum = torch.zeros(1, dtype=torch.int64, device=dev)
     st = torch.zeros(1, dtype=torch.int32, device=dev)
-    F = B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_FLAG_RESIDUAL
-
-    def forward(params):
-        api.allocate(state, params, E, stream, k_buf, k_sum, st)
-        h = h0
-        for l, w in enumerate(layers):
-            moe.w = w
-            moe.forward(h, k_buf, bufs[l & 1], F)
-            h = bufs[l & 1]
-
-    def timed(params, steps, warmup):
-        for _ in range(warmup):
-            forward(params)
-        R.barrier(world, dev)
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        for _ in range(steps):
-            forward(params)
-        b.record(stream)
-        R.barrier(world, dev)
-        return R.max_over_ranks(a.elapsed_time(b) / steps, world, dev)
-
+    out = torch.empty_like(h0)
+    F = B.REFLEX_FLAG_RENORM_TOPK
     p_reflex = B.make_params(**cfg.alloc_params())
     p_fixed = B.make_params(**cfg.alloc_params(delta_role=0, delta_cur=0))
+
+    def forward(params, hidden=h0, dst=out, state_=ds, around_up=None):
+        net.forward(state_, params, hidden, dst, k_buf, k_sum, st, flags=F,
+                    around_up=around_up)
+
+    def graph_of(fn):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="relaxed"):
+            fn()
+        return g
+
+    def barrier():
+        R.barrier(world, dev)
+
+    def timed(graph, replays, warmup):
+        for _ in range(warmup):
+            graph.replay()
+        barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(replays):
+            graph.replay()
+        b.record(stream)
+        barrier()
+        return a.elapsed_time(b)
+
+    clk = ClockSampler(local_rank)
+    clk.start()
+    # correctness gate before timing: counts and statuses clean
     forward(p_reflex)
     torch.cuda.synchronize(dev)
-    assert B.reflex_read_status(st) == B.REFLEX_OK and moe.status() == B.REFLEX_OK
+    assert B.reflex_read_status(st) == B.REFLEX_OK and net.status() == B.REFLEX_OK
     pairs = int(k_sum.item())
     forward(p_fixed)
     torch.cuda.synchronize(dev)
+    assert net.status() == B.REFLEX_OK
     pairs_fixed = int(k_sum.item())
-    clk = ClockSampler(local_rank)
-    clk.start()
-    ms = timed(p_reflex, args.steps, args.warmup)
+    # the routing of the last layer: experts that received pairs
+    counts = net.moe.record()["counts"].cpu().numpy()
+
+    # ---- timed region: one whole forward (counts + 16 layers) per replay ----
+    g_reflex = graph_of(lambda: forward(p_reflex))
+    ms = R.max_over_ranks(timed(g_reflex, args.steps, args.warmup), world, dev)
+    ms_step = ms / args.steps
+    # ---- gate/up GEMM launches: the same forward with events around every
+    # layer's gate/up GEMM, in one graph; durations of the last replay ----
+    try:   # timestamps recorded by graph nodes need external event records
+        up_evs = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+                  for _ in range(L)]
+        around = (lambda l: up_evs[l][0].record(), lambda l: up_evs[l][1].record())
+        timed(graph_of(lambda: forward(p_reflex, around_up=around)), 2, 1)
+    except TypeError:  # older torch: the same staged forward, launched eagerly
+        up_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(L)]
+        around = (lambda l: up_evs[l][0].record(), lambda l: up_evs[l][1].record())
+        for _ in range(2):
+            forward(p_reflex, around_up=around)
+        barrier()
+    up_times = [e[0].elapsed_time(e[1]) for e in up_evs]
+    # ---- same kernels at fixed top-K_base ----
+    g_fixed = graph_of(lambda: forward(p_fixed))
+    n_fixed = max(1, args.steps // 2)
+    ms_fixed = R.max_over_ranks(timed(g_fixed, n_fixed, 2), world, dev) / n_fixed
+
+    # ---- end to end through the public API from pinned host buffers: every
+    # forward uploads its hidden states and per-token state and reads its
+    # output back; copies on a copy stream, two buffer sets, so the upload of
+    # forward i+1 and the read-back of forward i-1 overlap forward i ----
+    host_in = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
+               for k, v in state.items()}
+    host_h = torch.from_numpy(np.ascontiguousarray(stack["hidden"]).view(np.int16)).pin_memory()
+    host_out = [torch.empty((T, d), dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+    dev_state = [{k: torch.empty_like(v) for k, v in ds.items()} for _ in range(2)]
+    dev_h = [torch.empty_like(h0) for _ in range(2)]
+    dev_out = [torch.empty_like(out) for _ in range(2)]
+    h2d = sum(int(v.numel() * v.element_size()) for v in host_in.values()) + \
+        int(host_h.numel() * host_h.element_size())
+    d2h = int(host_out[0].numel() * host_out[0].element_size())
+    copy_s = torch.cuda.Stream(dev)
+    ev_up = [torch.cuda.Event() for _ in range(2)]
+    ev_done = [torch.cuda.Event() for _ in range(2)]
+    ev_read = [torch.cuda.Event() for _ in range(2)]
+
+    def e2e_run(n: int):
+        for i in range(n + 1):
+            b = i & 1
+            if i < n:
+                with torch.cuda.stream(copy_s):   # upload forward i
+                    copy_s.wait_event(ev_done[b])  # forward i-2 finished with set b
+                    for k, v in host_in.items():
+                        dev_state[b][k].copy_(v, non_blocking=True)
+                    dev_h[b].view(torch.int16).copy_(host_h, non_blocking=True)
+                    ev_up[b].record(copy_s)
+                stream.wait_event(ev_up[b])
+                stream.wait_event(ev_read[b])      # read-back of forward i-2 done
+                forward(p_reflex, hidden=dev_h[b], dst=dev_out[b], state_=dev_state[b])
+                ev_done[b].record(stream)
+            if i > 0:
+                pb = (i - 1) & 1
+                with torch.cuda.stream(copy_s):   # read back forward i-1
+                    copy_s.wait_event(ev_done[pb])
+                    host_out[pb].copy_(dev_out[pb], non_blocking=True)
+                    ev_read[pb].record(copy_s)
+        stream.wait_event(ev_read[(n - 1) & 1])
+
+    e2e_run(2)
+    barrier()
+    n_e2e = max(3, args.steps // 2)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    copy_s.wait_event(e0)
+    e2e_run(n_e2e)
+    e1.record(stream)
+    barrier()
+    ms_e2e = R.max_over_ranks(e0.elapsed_time(e1), world, dev) / n_e2e
     clocks = clk.stop()
-    ms_fixed = timed(p_fixed, max(1, args.steps // 2), 2)
+    # the end-to-end outputs are those of the resident-input forward, bit for bit
+    g_reflex.replay()
+    torch.cuda.synchronize(dev)
+    assert torch.equal(host_out[(n_e2e - 1) & 1], out.cpu())
+    assert net.status() == B.REFLEX_OK
+
     if rank != 0:
         return
     peaks = load_peaks()
-    L = STACK_LAYERS
-    flops = 6.0 * d * I * pairs * L
-    flops_fixed = 6.0 * d * I * pairs_fixed * L
+    flops_layer = 6.0 * d * I * pairs                  # Eq. 10, routed experts
+    # dominant kernel: the CTA-pair gate/up (SwiGLU) GEMM, tensor-bound on
+    # this shape; algorithmic FLOPs per launch = 4 d inter sum(k); it runs
+    # inside a ~30 ms forward, so the sustained bf16 peak is the denominator
+    up_flops = 4.0 * pairs * d * I
+    touched = int((counts > 0).sum())
+    up_bytes = touched * 2 * I * d * 2 + pairs * d * 2 + pairs * I * 2
+    up_ms = statistics.mean(up_times)
+    tf = up_flops / (up_ms * 1e-3) / 1e12
+    peak_sus = peaks["bf16_sustained"] or peaks["bf16"]
+    roof = dict(bound="tensor", achieved=tf, peak=peak_sus, unit="TFLOP/s",
+                frac=tf / peak_sus, traffic=ncu_traffic("llada_moe_stack16"),
+                kernel="grouped_gemm_pair_kernel<0>: gate/up + SwiGLU, cta_group::2 "
+                       "tcgen05, TMEM accumulators, TMA-fed",
+                algorithmic_flops=up_flops, algorithmic_bytes=up_bytes,
+                avg_launch_ms=up_ms, launches_averaged=len(up_times),
+                frac_of_burst=tf / peaks["bf16"],
+                peak_source=peaks["source"] + " (sustained bf16; the kernel runs "
+                                              "inside a long step)")
+    launches = 1 + L * (api.step_launches(cfg.dtype, T, d, E, 0, F) - 1)
     line = dict(
-        metric=METRIC, value=R.whole_job_rate(T, world, ms), unit="tokens/s", n_gpus=world,
-        steps=args.steps, warmup=args.warmup, ms_per_step=ms, higher_is_better=True,
-        scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic",
-        config=dict(workload="llada_moe_stack16",
-                    description=f"{L} LLaDA-MoE-shaped layers (d=2048, E=64, inter=1024), "
-                                f"batch 32 x 1024 tokens, counts allocated once per forward, "
-                                f"residual h <- h + MoE(h), weights drawn on the device",
-                    tokens_per_step=T, layers=L, parallelism=f"replicas{world}",
-                    l2="no flush: 12.9 GB of expert weights stream every step"),
-        expert_tflops=flops * world / (ms * 1e-3) / 1e12,
-        expert_frac_of_bf16_peak=flops / (ms * 1e-3) / 1e12 / peaks["bf16_sustained"],
+        metric=METRIC, value=R.whole_job_rate(T, world, ms_step), unit="tokens/s",
+        n_gpus=world, steps=args.steps, warmup=args.warmup, ms_per_step=ms_step,
+        higher_is_better=True, scaling="weak", vs_baseline=None, dtype="bf16",
+        data="synthetic",
+        config=dict(stack_config(world),
+                    timing="CUDA-graph replay of one whole forward (counts + 16 "
+                           "layers) per timed iteration; e2e: eager API calls, each "
+                           "forward's upload and read-back from pinned host memory on a "
+                           "copy stream, double-buffered"),
+        expert_tflops=flops_layer * L * world / (ms_step * 1e-3) / 1e12,
+        expert_frac_of_bf16_sustained=flops_layer * L / (ms_step * 1e-3) / 1e12 / peak_sus,
         avg_k=pairs / T, pairs_per_layer=pairs,
         fixed_topk=dict(k=cfg.k_base, pairs_per_layer=pairs_fixed, ms_per_step=ms_fixed,
                         value=R.whole_job_rate(T, world, ms_fixed),
-                        expert_tflops=flops_fixed * world / (ms_fixed * 1e-3) / 1e12),
-        # the counts once, then every layer's forward
-        gpu_launches=args.steps * (1 + L * (api.step_launches(cfg.dtype, T, d, E, 0, F) - 1)),
-        clocks=dict(sm_mhz=clocks["sm_mhz"], sm_max_mhz=clocks["sm_max_mhz"],
-                    reasons=clocks["reasons"], samples=clocks["samples"]),
-        peak_source=peaks["source"] + " (sustained bf16, long step)")
+                        expert_tflops=6.0 * d * I * pairs_fixed * L * world
+                        / (ms_fixed * 1e-3) / 1e12),
+        roofline=roof,
+        e2e=dict(value=R.whole_job_rate(T, world, ms_e2e), unit="tokens/s",
+                 h2d_bytes_per_step=h2d, d2h_bytes_per_step=d2h, ms_per_step=ms_e2e,
+                 api="MoEStack.forward: reflex_step (counts + layer 0), then "
+                     "reflex_moe_forward per layer"),
+        gpu_launches=launches * args.steps,
+        clocks=clocks,
+    )
+    if not args.no_cpu_baseline and world == 1:
+        budget = args.cpu_seconds
+        rate, n, dt, cores = oracle_stack_rate(cfg, stack, state, budget, seed)
+        rate1, n1, dt1, _ = oracle_stack_rate(cfg, stack, state, budget / 2, seed + 1, 1)
+        line["cpu_baseline"] = dict(
+            value=rate, unit="tokens/s", cores=cores, kind="oracle",
+            sample=f"{n} seeded tokens of the {T}-token batch through all {L} layers "
+                   f"(counts on the whole batch; tokens are independent across "
+                   f"layers), {dt:.1f} s, rate per whole forward",
+            single_thread=dict(value=rate1, unit="tokens/s", cores=1,
+                               sample=f"{n1} seeded tokens, {dt1:.1f} s"))
+    elif world > 1:
+        line["cpu_baseline"] = None
     print(json.dumps(line), flush=True)
 
 
@@ -764,14 +1016,17 @@ def run_trajectory(args, rank, world, local_rank):
 
 def main():
     args = parse()
-    cfg = W.CONFIGS.get(args.config, W.CONFIGS["llada_moe_b32"])
     ri = R.rank_info()
     world, rank, local_rank = ri.world, ri.rank, ri.local_rank
     # the GPU arm reduces on the GPUs (NCCL); the reference arm is host-only
     R.init(world, "nccl" if args.impl == "reflex" else "gloo", local_rank)
+    stack = args.config == "llada_moe_stack16"
     try:
         if args.impl == "reference":
-            run_reference(args, cfg, rank, world)
+            if stack:
+                run_stack_reference(args, rank, world)
+            else:
+                run_reference(args, W.CONFIGS[args.config], rank, world)
         elif args.sweep:
             if rank == 0:
                 run_sweep(args, rank, world, local_rank)
@@ -781,10 +1036,10 @@ def main():
         elif args.trajectory:
             if rank == 0:
                 run_trajectory(args, rank, world, local_rank)
-        elif args.config == "llada_moe_stack16":
+        elif stack:
             run_stack(args, rank, world, local_rank)
         else:
-            run_gpu(args, cfg, rank, world, local_rank)
+            run_gpu(args, W.CONFIGS[args.config], rank, world, local_rank)
     finally:
         R.finalize(world)
 

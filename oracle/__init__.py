@@ -104,6 +104,8 @@ def _load():
                                       i32, i32, i32, i32, p]
     lib.oracle_num_threads.restype = ctypes.c_int
     lib.oracle_num_threads.argtypes = []
+    lib.oracle_set_num_threads.restype = None
+    lib.oracle_set_num_threads.argtypes = [ctypes.c_int]
     lib.oracle_bf16_from_f64_n.restype = None
     lib.oracle_bf16_from_f64_n.argtypes = [p, ctypes.c_int64, p]
     lib.oracle_residual_bf16.restype = None
@@ -125,6 +127,11 @@ def _c(a, dtype):
 
 def num_threads() -> int:
     return int(_load().oracle_num_threads())
+
+
+def set_num_threads(n: int) -> None:
+    """Threads of the oracle's OpenMP loops from now on."""
+    _load().oracle_set_num_threads(int(n))
 
 
 def exp_f32(x) -> np.ndarray:

@@ -535,6 +535,17 @@ int oracle_num_threads(void) {
 #endif
 }
 
+/* Threads used by the OpenMP loops from now on (timing the oracle on one  */
+/* core and on all cores); no effect without OpenMP.                       */
+void oracle_set_num_threads(int n) {
+#ifdef _OPENMP
+    extern void omp_set_num_threads(int);
+    if (n >= 1) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
 /* Array forms used by the pins and by the parity tests. */
 void oracle_exp_f32_n(const float* x, float* y, int64_t n) {
     for (int64_t i = 0; i < n; ++i) y[i] = oracle_exp_f32(x[i]);

@@ -179,3 +179,73 @@ class MoELayer:
             totals=totals,
             scores=self._view(self.rec.scores, T * E, torch.float32).view(T, E),
         )
+
+
+class MoEStack:
+    """A stack of variable-count MoE layers of one shape sharing one workspace:
+    one denoising forward computes the per-token counts once (Eq. 3; the
+    counts are shared by every layer) and runs every layer with the residual
+    connection h <- h + MoE(h).  The first layer runs with the counts in one
+    reflex_step call, the others with reflex_moe_forward; every call takes the
+    current stream, so a whole forward can be captured in one CUDA graph."""
+
+    def __init__(self, layers: list, *, dtype: str, d: int, E: int, inter: int,
+                 shared_inter: int, k_max: int, max_tokens: int, device="cuda"):
+        if not layers:
+            raise ValueError("a stack needs at least one layer")
+        self.layers = layers
+        self.moe = MoELayer(layers[0], dtype=dtype, d=d, E=E, inter=inter,
+                            shared_inter=shared_inter, k_max=k_max,
+                            max_tokens=max_tokens, device=device)
+        self.d, self.E = d, E
+        self.tdtype = self.moe.tdtype
+        self._bufs = [torch.empty((max_tokens, d), dtype=self.tdtype, device=device)
+                      for _ in range(2)]
+
+    def _layer_out(self, l: int, T: int, out: torch.Tensor, keep):
+        if keep is not None:
+            return keep[l]
+        if l == len(self.layers) - 1:
+            return out
+        return self._bufs[l & 1][:T]
+
+    def forward(self, state: dict, params: B.reflex_alloc_params, hidden: torch.Tensor,
+                out: torch.Tensor, k_out: torch.Tensor, k_sum: torch.Tensor,
+                status: torch.Tensor, flags: int = B.REFLEX_FLAG_RENORM_TOPK,
+                keep: list | None = None, around_up=None, check: bool = True):
+        """One denoising forward: `out` receives the last layer's output.
+        `keep` (optional) lists one [T, d] tensor per layer that receives that
+        layer's output instead of the internal ping-pong buffers.
+        `around_up` (optional) is a pair of callables run right before and
+        after every layer's gate/up GEMM (the layer is then issued as three
+        stage calls on the same workspace, which gives the same bits)."""
+        T = int(hidden.shape[0])
+        flags = flags | B.REFLEX_FLAG_RESIDUAL
+        h = hidden
+        for l, w in enumerate(self.layers):
+            self.moe.w = w
+            dst = self._layer_out(l, T, out, keep)
+            if around_up is None:
+                if l == 0:
+                    self.moe.step(state, params, h, out=dst, k_out=k_out, k_sum=k_sum,
+                                  status=status, flags=flags, check=check)
+                else:
+                    self.moe.forward(h, k_out, dst, flags, check=check)
+            else:
+                first = B.REFLEX_STAGE_ROUTE | B.REFLEX_STAGE_DISPATCH
+                if l == 0:
+                    self.moe.step(state, params, h, out=dst, k_out=k_out, k_sum=k_sum,
+                                  status=status, flags=flags | first, check=check)
+                else:
+                    self.moe.forward(h, k_out, dst, flags | first, check=check)
+                around_up[0](l)
+                self.moe.forward(h, k_out, dst, flags | B.REFLEX_STAGE_EXPERT_UP,
+                                 check=check)
+                around_up[1](l)
+                self.moe.forward(h, k_out, dst, flags | B.REFLEX_STAGE_EXPERT_DOWN |
+                                 B.REFLEX_STAGE_COMBINE, check=check)
+            h = dst
+        return out
+
+    def status(self) -> int:
+        return self.moe.status()

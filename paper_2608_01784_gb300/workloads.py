@@ -236,6 +236,29 @@ def make_state(cfg: LayerConfig, seed: int = 0, hist_len: int | None = None,
                 masked=masked, conf1=conf1, conf2=conf2, hist_len=hl)
 
 
+def layer_weights(cfg: LayerConfig, seed: int = 0, prefix: str = "") -> dict:
+    """Router and expert weights of one MoE layer (no hidden states); the
+    streams are named `prefix` + array name, so each layer of a stack draws
+    its own weights from the same seed."""
+    d, E, I = cfg.d, cfg.E, cfg.inter
+    out = {}
+    out["w_router"] = _weights(cfg, seed, prefix + "w_router", (E, d), d)
+    out["w_gate_up"] = _weights(cfg, seed, prefix + "w_gate_up", (E, 2 * I, d), d)
+    out["w_down"] = _weights(cfg, seed, prefix + "w_down", (E, d, I), I)
+    if cfg.shared_inter:
+        S = cfg.shared_inter
+        out["shared_gate_up"] = _weights(cfg, seed, prefix + "shared_gate_up", (2 * S, d), d)
+        out["shared_down"] = _weights(cfg, seed, prefix + "shared_down", (d, S), S)
+    return out
+
+
+def make_hidden(cfg: LayerConfig, seed: int = 0, T: int | None = None) -> np.ndarray:
+    """Hidden states [T, d] ~ N(0, 1) (bf16 bits for bf16 layers)."""
+    T = cfg.T if T is None else T
+    h = normal_f32(seed, "hidden", T * cfg.d, 1.0).reshape(T, cfg.d)
+    return to_bf16_bits(h) if cfg.dtype == "bf16" else h
+
+
 def make_layer(cfg: LayerConfig, seed: int = 0, T: int | None = None) -> dict:
     """Hidden states and weights of one MoE layer.
 
@@ -243,18 +266,18 @@ def make_layer(cfg: LayerConfig, seed: int = 0, T: int | None = None) -> dict:
     w_gate_up [E, 2*inter, d] (rows [0, inter) gate, [inter, 2*inter) up);
     w_down [E, d, inter]; shared_gate_up [2*s, d]; shared_down [d, s].
     bf16 arrays are uint16 bit patterns."""
-    T = cfg.T if T is None else T
-    d, E, I = cfg.d, cfg.E, cfg.inter
-    h = normal_f32(seed, "hidden", T * d, 1.0).reshape(T, d)
-    out = dict(hidden=to_bf16_bits(h) if cfg.dtype == "bf16" else h)
-    out["w_router"] = _weights(cfg, seed, "w_router", (E, d), d)
-    out["w_gate_up"] = _weights(cfg, seed, "w_gate_up", (E, 2 * I, d), d)
-    out["w_down"] = _weights(cfg, seed, "w_down", (E, d, I), I)
-    if cfg.shared_inter:
-        S = cfg.shared_inter
-        out["shared_gate_up"] = _weights(cfg, seed, "shared_gate_up", (2 * S, d), d)
-        out["shared_down"] = _weights(cfg, seed, "shared_down", (d, S), S)
+    out = dict(hidden=make_hidden(cfg, seed, T))
+    out.update(layer_weights(cfg, seed))
     return out
+
+
+def make_stack(cfg: LayerConfig, seed: int = 0, n_layers: int = 16,
+               T: int | None = None) -> dict:
+    """A stack of `n_layers` MoE layers of one shape: the first layer's input
+    hidden states and, per layer l, its own router and expert weights (streams
+    "layer{l}/..." of the seed).  Returns {"hidden": [T, d], "layers": [...]}."""
+    return dict(hidden=make_hidden(cfg, seed, T),
+                layers=[layer_weights(cfg, seed, f"layer{l}/") for l in range(n_layers)])
 
 
 def skewed_k(T: int, skew: float, k_min: int, k_base: int, k_max: int,

@@ -20,6 +20,28 @@ F32_MAX_ABS = 1e-4
 ALPHA_RTOL = 2e-5
 
 
+def bf16_ulp(x) -> np.ndarray:
+    """Spacing of bf16 numbers (8 significant bits) at |x|: 2^(floor(log2|x|) - 7)."""
+    ax = np.maximum(np.abs(np.asarray(x, np.float64)), 2.0 ** -126)
+    return np.exp2(np.floor(np.log2(ax)) - 7)
+
+
+def residual_excess(gpu: np.ndarray, ref: np.ndarray, rounded_ref: bool) -> float:
+    """Largest |gpu - ref| beyond what the bf16 rounding of a residual output
+    h + MoE(h) allows on top of the MoE term's BF16_MAX_ABS; <= 0 passes.
+
+    The layer output is rounded to bf16 once, after the residual sum.  Against
+    an unrounded (fp64) reference that rounding adds at most half a bf16 ulp
+    of the sum; against a reference rounded to bf16 itself the two sums may
+    round to neighbouring values, one ulp apart.  The ulp is taken at the
+    larger of the two magnitudes (a sum just below a power of two may round up
+    to it)."""
+    g = gpu.astype(np.float64)
+    u = bf16_ulp(np.maximum(np.abs(g), np.abs(ref)))
+    allow = BF16_MAX_ABS + (u if rounded_ref else 0.5 * u)
+    return float((np.abs(g - ref) - allow).max())
+
+
 def params_of(cfg: W.LayerConfig, **override) -> B.reflex_alloc_params:
     return B.make_params(**cfg.alloc_params(**override))
 

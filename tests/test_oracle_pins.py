@@ -450,6 +450,21 @@ def test_role_shuffle_follows_key_order():
         assert k1[a:b].tolist() == k0[a:b][ranks].tolist()
 
 
+def test_splitmix64_matches_published_reference_outputs():
+    # SplitMix64 (Steele, Lea and Flood 2014) as published: the outputs of its
+    # public-domain reference implementation for two seeds
+    # (tests/golden/splitmix64_reference.json).  A wrong gamma, multiplier or
+    # shift in the oracle's generator fails here.
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden",
+                                    "splitmix64_reference.json")))
+    for v in g["vectors"]:
+        seed = int(v["seed"])
+        want = ([int(x, 16) for x in v["outputs_hex"]] if "outputs_hex" in v
+                else [int(x) for x in v["outputs_dec"]])
+        got = [oracle.splitmix64(seed, n) for n in range(1, len(want) + 1)]
+        assert got == want, (seed, [hex(x) for x in got])
+
+
 def test_splitmix64_bits_are_uniform_and_mix():
     out = np.array([oracle.splitmix64(42, n) for n in range(1, 1 << 15)], np.uint64)
     top = (out >> np.uint64(56)).astype(np.int64)
