@@ -55,9 +55,9 @@ METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
 # kernel source it was taken on; once the source differs the line reports
 # null (the counters no longer describe the kernel that ran).
 NCU_TRAFFIC = {
-    "llada_moe": (561284352, None),
+    "llada_moe": (561284352, "7507f281c153b35d"),
     "llada2_mini": (1407363048, None),
-    "llada_moe_stack16": (None, None),
+    "llada_moe_stack16": (1636404224, "7507f281c153b35d"),
 }
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2608_01784_gb300", "csrc", "experts_tc.cu")
 
@@ -127,6 +127,7 @@ class ClockSampler:
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
                  "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            time.sleep(1.0)   # nvidia-smi takes a moment before its first sample
         except Exception:
             self.proc = None
 

@@ -269,6 +269,8 @@ size_t reflex_moe_workspace_size(int32_t dtype, int32_t T, int32_t d,
  *   out             [T, d] output.
  *   rec             HOST struct, nullable: receives device pointers into the
  *                   workspace (no copy is made).
+ * T == 0 launches no kernel; the workspace header (error word, totals) is
+ * cleared in stream order, so reflex_moe_status reports this call.
  * Shape rules: T >= 0, d % 64 == 0, 1 <= E <= 1024, 1 <= k_max <= 32,
  * inter % 64 == 0, shared_inter % 64 == 0.  The bf16 tcgen05 path also needs
  * d % 256 == 0 and inter, shared_inter % 128 == 0 (else REFLEX_EUNSUPPORTED
@@ -329,8 +331,9 @@ int reflex_step(const float* conf_prev1, const float* conf_prev2, const uint8_t*
  * library until the process exits).  Nothing is allocated or freed.
  *   ids_out    [T, k_max] int32, alpha_out [T, k_max] fp32: same meaning and
  *              values as the ids / alpha of reflex_route_record.
- *   dev_status nullable device error word (cleared, then OR-ed as for the
- *              forward; read it with reflex_read_status).
+ *   dev_status nullable device error word: cleared with a 4-byte memset in
+ *              stream order before this call's kernels (also when T == 0),
+ *              then OR-ed with error bits; read it with reflex_read_status.
  * Returns REFLEX_EWORKSPACE when T * E > REFLEX_NOALLOC_MAX_SCORES, and
  * REFLEX_EINVAL for the shape errors of reflex_moe_forward.  The first call
  * on each device looks up the array's address; make it before any stream

@@ -334,8 +334,11 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
     rec->scores = reinterpret_cast<float*>(ws + L.z);
   }
   if (T == 0) {
+    // no kernel of the layer runs: the header (error word, totals) still
+    // describes this call
+    cudaStream_t s0 = static_cast<cudaStream_t>(stream);
+    RX_CUDA(cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s0));
     if (ac != nullptr) {
-      cudaStream_t s0 = static_cast<cudaStream_t>(stream);
       RX_CUDA(clear_alloc_outputs(*ac, s0));
       RX_CUDA(launch_alloc(*ac, 0, s0, false));
     }

@@ -18,8 +18,12 @@
 //     any stream capture starts.
 //   - All calls share the one array and it keeps whatever the last call
 //     wrote.  Nothing in it needs to start at zero: each call writes every
-//     score it later reads.  Calls whose GPU work overlaps in time (for
-//     example on two streams at once) race on the array; serialise them.
+//     score it later reads (a score tile whose bounded wait expires writes
+//     -inf, never the previous call's values, and flags REFLEX_ETIMEOUT).
+//     Calls whose GPU work overlaps in time (for example on two streams at
+//     once) race on the array; serialise them.
+//   - The caller's status word is cleared with a 4-byte memset in stream
+//     order before the kernels, also when T == 0.
 #include <mutex>
 
 #include "common.cuh"
@@ -67,18 +71,26 @@ extern "C" int reflex_route_noalloc(int32_t dtype, const void* hidden,
   if (T < 0 || d <= 0 || d % 64 != 0 || E < 1 || E > 1024) return REFLEX_EINVAL;
   if (k_max < 1 || k_max > 32) return REFLEX_EINVAL;
   if (static_cast<int64_t>(T) * E > REFLEX_NOALLOC_MAX_SCORES) return REFLEX_EWORKSPACE;
-  if (T == 0) return REFLEX_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint32_t* err = reinterpret_cast<uint32_t*>(dev_status);
+  if (T == 0) {
+    // nothing to route; the status word still reports this call only
+    if (err != nullptr && cudaMemsetAsync(err, 0, sizeof(uint32_t), s) != cudaSuccess)
+      return REFLEX_ECUDA;
+    return REFLEX_OK;
+  }
   if (hidden == nullptr || w_router == nullptr || k == nullptr ||
       ids_out == nullptr || alpha_out == nullptr)
     return REFLEX_EINVAL;
   float* z = nullptr;
   int sms = 0;
   if (!device_setup(&z, &sms)) return REFLEX_ECUDA;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  uint32_t* err = reinterpret_cast<uint32_t*>(dev_status);
-  // the router clears the error word before select may set bits in it
-  if (rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z, err, err ? 1 : 0, err,
-                               sms, s) != cudaSuccess)
+  // the status word is cleared in stream order before any kernel of this
+  // call can set a bit in it (a 4-byte memset allocates nothing)
+  if (err != nullptr && cudaMemsetAsync(err, 0, sizeof(uint32_t), s) != cudaSuccess)
+    return REFLEX_ECUDA;
+  if (rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z, nullptr, 0, err, sms,
+                               s) != cudaSuccess)
     return REFLEX_ECUDA;
   if (rx::launch_router_select(z, k, T, E, k_max, (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
                                ids_out, alpha_out, err, s) != cudaSuccess)

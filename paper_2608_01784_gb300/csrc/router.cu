@@ -649,6 +649,11 @@ __global__ void __launch_bounds__(ResCfg<LY, TM, TN, WT, WE>::NT, 1)
   uint8_t* rows = smem_r + kResBarBytes;
   grid_dep_wait();
   grid_dep_launch();
+  // CTA (0, 0) clears the header words when it starts; a wait of another
+  // CTA can only expire (and set an error bit) kResWaitNs after that CTA
+  // started, and the grid is at most two waves of CTAs that start within
+  // microseconds of each other, so the clear comes first.  Callers that need
+  // the order guaranteed clear the word in stream order and pass nz = 0.
   if (zw != nullptr && blockIdx.x == 0 && blockIdx.y == 0)
     for (int i = threadIdx.x; i < nz; i += blockDim.x) zw[i] = 0u;
   const int pitch = 2 * d + 16;
@@ -705,10 +710,11 @@ __global__ void __launch_bounds__(ResCfg<LY, TM, TN, WT, WE>::NT, 1)
     }
   }
   if (!ok) {
-    // every copy into this CTA's shared memory must land before it exits
+    // every copy into this CTA's shared memory must land before it exits;
+    // the thread's scores are incomplete and are stored as -inf (never left
+    // as whatever an earlier call wrote there)
     set_err(err, kErrTimeout);
     for (int c = 0; c < nch; ++c) mbar_wait(&bars[c], 0u, nullptr, kResDrainNs);
-    return;
   }
 #pragma unroll
   for (int i = 0; i < TM; ++i) {
@@ -717,7 +723,7 @@ __global__ void __launch_bounds__(ResCfg<LY, TM, TN, WT, WE>::NT, 1)
 #pragma unroll
     for (int j = 0; j < TN; ++j) {
       const int e = e0 + re + LX * j;
-      if (e < E) z[static_cast<int64_t>(t) * E + e] = acc[i][j];
+      if (e < E) z[static_cast<int64_t>(t) * E + e] = ok ? acc[i][j] : -INFINITY;
     }
   }
 }
@@ -817,7 +823,8 @@ __device__ __forceinline__ float chain_bf16(const uint4* __restrict__ hs,
 // The same chain with 32-byte expert-row loads (two in flight per lane):
 // half the load instructions and L1 requests of the 16-byte form, whose
 // warp loads each touch a different row per lane (LLaDA2.0-mini routing
-// 113.6 -> 107.6 us).  Needs the row 32-byte aligned and d % 16 == 0.
+// 113.6 -> 107.6 us).  Needs the row 32-byte aligned and d % 32 == 0 (the
+// loop takes the 32-byte steps in pairs; the screened path has d % 128 == 0).
 __device__ __forceinline__ float chain_bf16_wide(const uint4* __restrict__ hs,
                                                  const __nv_bfloat16* __restrict__ we, int d) {
   const uint32_t* wp = reinterpret_cast<const uint32_t*>(we);

@@ -131,10 +131,11 @@ def test_host_rejections_enqueue_nothing(lib):
     # shared expert declared without weights
     assert fw(1, 1, 1, 1, 1, None, None, 128, 1, 4, 256, 8, 128, 4, 1, 256,
               1 << 30, 1, None, None) == B.REFLEX_EINVAL
-    # T = 0 is a no-op that still fills the record
+    # T = 0 launches no kernel; it fills the record and clears the workspace
+    # header with a memset, which needs a device (none here: ECUDA)
     rec = B.reflex_route_record()
     assert fw(1, None, None, None, None, None, None, 0, None, 0, 256, 8, 128, 4,
-              1, 256, 1 << 20, None, ctypes.byref(rec), None) == B.REFLEX_OK
+              1, 256, 1 << 20, None, ctypes.byref(rec), None) == B.REFLEX_ECUDA
     assert rec.ids == 3 * 256            # after the header, scores and expert norms
     assert lib.reflex_selftest_wait_timeout(None, 10, None) == B.REFLEX_EINVAL
     assert lib.reflex_read_status(None, None) == B.REFLEX_EINVAL

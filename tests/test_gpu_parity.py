@@ -296,6 +296,102 @@ def test_screened_and_exact_routing_agree_on_the_whole_layer():
     assert np.array_equal(out_s.view(np.uint32), out_e.view(np.uint32))
 
 
+# Adversarial inputs for the screen's one assumption (the tensor cores' fp32
+# accumulation errs by at most 2^-12 sum_k |h_k w_k|): rows whose products
+# cancel (sum |h w| far above |z|), bf16 inputs spread over many binary
+# orders of magnitude, d = 4096, and the most K slices the screen takes
+# (2: from 2048 x 256 scores on, the tile count leaves no room for more).
+# Ids, weights and selected scores must stay bit-exact; every tensor-core
+# estimate left in the record is checked against the assumed bound and the
+# largest observed ratio is printed (TC_ERROR_RATIO).
+def _cancelling_case(T, d, E, seed):
+    rng = np.random.default_rng(seed)
+    x = rng.standard_normal((T, d // 2)).astype(np.float32)
+    y = (0.02 * rng.standard_normal((E, d // 2))).astype(np.float32)
+    eps = (0.005 * rng.standard_normal((E, d // 2))).astype(np.float32)
+    xb = W.bf16_bits_to_f32(W.to_bf16_bits(x))
+    yb = W.bf16_bits_to_f32(W.to_bf16_bits(y))
+    h = np.concatenate([xb, xb], axis=1)                    # [x, x]
+    w = np.concatenate([yb, -yb + eps], axis=1)             # [y, -y + eps]
+    return W.to_bf16_bits(h), W.to_bf16_bits(w)
+
+
+def _wide_exponent_case(T, d, E, seed):
+    rng = np.random.default_rng(seed)
+
+    def spread(shape, lo, hi):
+        mant = rng.uniform(1.0, 2.0, shape)
+        sign = rng.choice([-1.0, 1.0], shape)
+        return (sign * mant * np.exp2(rng.integers(lo, hi + 1, shape))).astype(np.float32)
+    return W.to_bf16_bits(spread((T, d), -24, 8)), W.to_bf16_bits(spread((E, d), -30, 0))
+
+
+@pytest.mark.parametrize("kind,T,E,d", [
+    ("cancel", 4096, 128, 2048),     # 2 K slices
+    ("cancel", 2048, 256, 4096),     # 2 K slices, d = 4096
+    ("wide", 2048, 256, 2048),       # 2 K slices
+    ("wide", 4096, 256, 4096),       # 1 slice, d = 4096
+    ("gauss", 2048, 256, 4096),      # 2 K slices, d = 4096
+])
+def test_screened_routing_adversarial_inputs(kind, T, E, d):
+    kmax = 8
+    if kind == "cancel":
+        hb, wb = _cancelling_case(T, d, E, 41)
+    elif kind == "wide":
+        hb, wb = _wide_exponent_case(T, d, E, 43)
+    else:
+        _, lay = _bf16_case(T, d, E, 128, 0, kmax, seed=45)
+        hb, wb = lay["hidden"], lay["w_router"]
+    cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=47)
+    layer = dict(layer, hidden=hb, w_router=wb)
+    k = np.random.default_rng(T + E).integers(1, kmax + 1, T).astype(np.int32)
+    gl = G.GpuLayer(cfg, layer)
+    _, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE)
+    assert status == B.REFLEX_OK
+    z = oracle.router_logits(hb, wb)
+    ids, alpha = oracle.select(z, k, kmax)
+    assert np.array_equal(rec["ids"], ids)
+    valid = ids >= 0
+    np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
+    rows = np.repeat(np.arange(T), kmax).reshape(T, kmax)[valid]
+    assert np.array_equal(rec["scores"][rows, ids[valid]].view(np.uint32),
+                          z[rows, ids[valid]].view(np.uint32))
+    # the tensor-core estimates (entries not recomputed with the chain)
+    hf = _bf16_floats(hb).astype(np.float64)
+    wf = _bf16_floats(wb).astype(np.float64)
+    exact = hf @ wf.T
+    absdot = np.abs(hf) @ np.abs(wf).T
+    est = rec["scores"].view(np.uint32) != z.view(np.uint32)
+    assert est.sum() > T                     # most scores stayed estimates
+    ratio = np.abs(rec["scores"].astype(np.float64) - exact)[est] / absdot[est]
+    worst = float(ratio.max())
+    print(f"TC_ERROR_RATIO kind={kind} T={T} E={E} d={d} max={worst:.3e} "
+          f"(2^-12 = {2.0 ** -12:.3e}) median={float(np.median(ratio)):.3e} "
+          f"estimates={int(est.sum())} cancellation={float(np.median(absdot / (np.abs(exact) + 1e-30))):.1f}")
+    assert worst <= 2.0 ** -12
+
+
+def test_screened_routing_router_rows_16_byte_aligned():
+    # a router matrix that starts 16 bytes past a 32-byte boundary: the
+    # recheck reads expert rows with 16-byte loads instead of 32-byte ones
+    T, E, d, kmax = 4096, 256, 2048, 8
+    cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=51)
+    gl = G.GpuLayer(cfg, layer)
+    flat = torch.empty(E * d + 8, dtype=torch.bfloat16, device="cuda")
+    w_off = flat[8:].view(E, d)
+    w_off.copy_(gl.dev["w_router"])
+    assert w_off.data_ptr() % 32 == 16
+    gl.moe.w = dict(gl.moe.w, w_router=w_off)
+    k = np.random.default_rng(52).integers(1, kmax + 1, T).astype(np.int32)
+    _, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE)
+    assert status == B.REFLEX_OK
+    z = oracle.router_logits(layer["hidden"], layer["w_router"])
+    ids, alpha = oracle.select(z, k, kmax)
+    assert np.array_equal(rec["ids"], ids)
+    valid = ids >= 0
+    np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
+
+
 @pytest.mark.parametrize("T,d,E,inter,shared,kmax,kmode", [
     (96, 256, 8, 128, 0, 4, "random"),     # one partial m-tile per expert
     (1000, 256, 4, 128, 0, 4, "max"),      # 8 m-tiles per expert, ragged tail

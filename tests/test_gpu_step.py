@@ -124,6 +124,17 @@ def test_step_zero_tokens():
     assert int(k_sum.item()) == 0 and B.reflex_read_status(st) == B.REFLEX_OK
 
 
+def test_forward_zero_tokens_clears_a_stale_error():
+    cfg, layer, dl, moe = _setup("llada_moe", 1)
+    k = torch.full((cfg.T,), cfg.k_max + 3, dtype=torch.int32, device="cuda")
+    moe.forward(dl["hidden"], k)                 # counts out of range: flagged
+    torch.cuda.synchronize()
+    assert moe.status() == B.REFLEX_EKRANGE
+    moe.forward(dl["hidden"][:0], k[:0])
+    torch.cuda.synchronize()
+    assert moe.status() == B.REFLEX_OK
+
+
 def test_step_graph_replay():
     cfg, layer, dl, moe = _setup("llada_moe", 2)
     p = G.params_of(cfg)
