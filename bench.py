@@ -900,6 +900,27 @@ ABLATIONS = [  # (name, allocation overrides): REFLEX and its App. C ablations
     ("uncertainty_only", dict(signal=4)),
     ("fixed_topk", dict(delta_role=0, delta_cur=0)),
 ]
+# The threshold-based comparison methods of App. B on the same kernels (count
+# bounds [1, 12]; low / high thresholds per model family as the paper sets
+# them): Top-p mass p and the Expert-Threshold router weight.
+RULE_SETTINGS = {
+    "llada_moe": dict(top_p=(0.15, 0.20), expert_thr=(0.0215, 0.0190)),
+    "llada_moe_b32": dict(top_p=(0.15, 0.20), expert_thr=(0.0215, 0.0190)),
+    "llada2_mini": dict(top_p=(0.25, 0.325), expert_thr=(0.0270, 0.0220)),
+}
+
+
+def rule_ablations(cfg_name: str):
+    r = RULE_SETTINGS.get(cfg_name)
+    if r is None:
+        return []
+    out = []
+    for tag, v in zip(("low", "high"), r["top_p"]):
+        out.append((f"top_p_{tag}", dict(count_rule=1, rule_threshold=v, k_min=1, k_max=12)))
+    for tag, v in zip(("low", "high"), r["expert_thr"]):
+        out.append((f"expert_threshold_{tag}",
+                    dict(count_rule=2, rule_threshold=v, k_min=1, k_max=12)))
+    return out
 
 
 def run_ablation(args, rank, world, local_rank):
@@ -941,12 +962,22 @@ def run_ablation(args, rank, world, local_rank):
         torch.cuda.synchronize(dev)
         return a.elapsed_time(b) / steps
 
-    for name, over in ABLATIONS:
+    for name, over in ABLATIONS + rule_ablations(cfg.name):
         params = [B.make_params(**cfg.alloc_params(**over, shuffle_seed=args.seed + i))
                   for i in range(steps)]
+        rule = over.get("count_rule", 0)
+        scores = None
+        if rule:   # the score rules' counts from the layer's own router scores
+            moe.forward(dl["hidden"], k_buf, out, F | B.REFLEX_STAGE_ROUTE |
+                        B.REFLEX_FLAG_EXACT_SCORES)
+            scores = moe.record()["scores"].clone()
 
         def alloc(i):
-            api.allocate(ds, params[i % steps], E, stream, k_buf, k_sum, st)
+            if rule:
+                api.allocate(None, params[i % steps], E, stream, k_buf, k_sum, st,
+                             router_scores=scores)
+            else:
+                api.allocate(ds, params[i % steps], E, stream, k_buf, k_sum, st)
 
         def step(i):
             moe.step(ds, params[i % steps], dl["hidden"], out=out, k_out=k_buf,
@@ -961,6 +992,9 @@ def run_ablation(args, rank, world, local_rank):
         ms = timed(step)
         line = dict(ablation=name, workload=cfg.name, tokens=T, avg_k=pairs / T,
                     pairs=pairs, alloc_us=1e3 * ms_alloc, ms_per_step=ms,
+                    count_rule=("reflex" if not rule else
+                                "top_p" if rule == 1 else "expert_threshold"),
+                    rule_threshold=over.get("rule_threshold"),
                     tokens_per_s=T / (ms * 1e-3),
                     expert_tflops=6.0 * d * I * pairs / (ms * 1e-3) / 1e12)
         print(json.dumps(line), flush=True)

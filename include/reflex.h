@@ -102,7 +102,37 @@ typedef struct {
                            Sequences longer than 4096 tokens are left as
                            they are and flag REFLEX_ECAPACITY.              */
     uint64_t shuffle_seed; /* seed of the shuffle's splitmix64 stream       */
+    int32_t count_rule; /* where the counts come from: REFLEX_RULE_*        */
+    float rule_threshold; /* p of REFLEX_RULE_TOP_P, or the router-weight
+                           threshold of REFLEX_RULE_EXPERT_THRESHOLD      */
 } reflex_alloc_params;
+
+/* Count rules.  REFLEX_RULE_REFLEX (0, the default) is the allocation of
+ * Sec. 4.2-4.3 above.  The other two are the threshold-based comparison
+ * methods of App. B, which take each token's count from its router scores
+ * z_t instead of its refinement state (the paper runs them with the count
+ * bounds [1, 12], i.e. k_min = 1, k_max = 12):
+ *   TOP_P             the smallest prefix of the router-ranked experts
+ *                     (scores descending, lower index first on ties) whose
+ *                     cumulative routing mass reaches rule_threshold;
+ *   EXPERT_THRESHOLD  the number of experts whose routing mass exceeds
+ *                     rule_threshold;
+ * either clipped to [k_min, min(k_max, E)].  The routing mass is the
+ * softmax of z_t over all E experts, and the decision is taken in fp32 in
+ * this order, so that the counts are reproducible bit for bit:
+ *   m = max_e z_e;  u_e = exp(z_e - m) (the library's Cody-Waite exp, the
+ *   one of the FPS sigmoids);  S = the sum of the u_e, lane l of 32 adding
+ *   u_l, u_{l+32}, ... in ascending order, then the 32 lane sums combined by
+ *   s_l <- s_l + s_{l xor o} for o = 16, 8, 4, 2, 1;
+ *   TOP_P: c_j = c_{j-1} + u_(j) over the ranks j = 1, 2, ... (c_0 = 0),
+ *   k = the smallest j with c_j / S >= rule_threshold;
+ *   EXPERT_THRESHOLD: k = #{e : u_e / S > rule_threshold}.
+ * The score rules read every router score, so a forward that takes its
+ * counts from them computes every score with the canonical chain (as with
+ * REFLEX_FLAG_EXACT_SCORES). */
+#define REFLEX_RULE_REFLEX 0
+#define REFLEX_RULE_TOP_P 1
+#define REFLEX_RULE_EXPERT_THRESHOLD 2
 
 /* Rank keys for the FGER groups (Sec. 4.3; signal ablation of App. C).  The
  * top floor(q |J_h|) tokens by (key desc, position asc) gain delta_cur, the
@@ -130,16 +160,19 @@ typedef struct {
 
 /* Fills the Sec. 5.1 defaults: k_base 8, delta_role 4, delta_cur 2, q 0.25,
  * theta 0.9, w_cf 0.30 (LLaDA-MoE; 0.25 for LLaDA2.0-mini), v_ref 0.01,
- * tau 0.05, the clip [k_min, k_max] = [2, 12], signal FPS, no shuffle. */
+ * tau 0.05, the clip [k_min, k_max] = [2, 12], signal FPS, no shuffle,
+ * count rule REFLEX (rule_threshold 0). */
 void reflex_default_params(reflex_alloc_params* p);
 
 /*
  * reflex_allocate — per-token expert counts k_i for one denoising forward
  * (Eq. 3 realised by Eq. 5 and Eq. 9, Sec. 4.2-4.3).
  *
- *   router_scores  [T, E] fp32, nullable.  Accepted for the shape of the
- *                  allocation problem; REFLEX's rule does not read it (the
- *                  router only ranks experts, Sec. 3.3).
+ *   router_scores  [T, E] fp32.  REFLEX's rule does not read it (the router
+ *                  only ranks experts, Sec. 3.3) and it may be NULL; the
+ *                  score rules (p->count_rule TOP_P or EXPERT_THRESHOLD)
+ *                  take the counts from it alone (E experts per row), and
+ *                  then every state array below may be NULL.
  *   conf_prev1     [T] fp32  c_i^{t-1}, the latest confidence observation.
  *   conf_prev2     [T] fp32  c_i^{t-2}; read only where hist_len >= 2.
  *   hist_len       [T] u8    number of past observations (0, 1, >= 2).
@@ -160,8 +193,10 @@ void reflex_default_params(reflex_alloc_params* p);
  * REFLEX_ECAPACITY in dev_status and leaves them at K_cur, clipped).
  * Host errors: REFLEX_EINVAL for null required pointers, T < 0, B < 1, or
  * parameters violating 1 <= k_min <= k_max, k_base >= 1, delta_* >= 0,
- * 0 < q <= 0.5, w_cf > 0, tau > 0.  Counts below k_min (or above k_max)
- * produced by Eq. 5 / Eq. 9 are clipped.
+ * 0 < q <= 0.5, w_cf > 0, tau > 0, an unknown count_rule, or (score rules)
+ * a missing router_scores, E outside [1, 1024] or a non-finite
+ * rule_threshold.  Counts below k_min (or above k_max) produced by Eq. 5 /
+ * Eq. 9 are clipped.
  */
 int reflex_allocate(const float* router_scores, const float* conf_prev1,
                     const float* conf_prev2, const uint8_t* hist_len,
@@ -306,6 +341,11 @@ int reflex_moe_forward(int32_t dtype, const void* hidden, const void* w_router,
  * returns its status before anything is launched.  The REFLEX_STAGE_* bits of
  * flags select the forward's stages as for reflex_moe_forward; the counts are
  * computed in every case.
+ * With a score rule (p->count_rule TOP_P or EXPERT_THRESHOLD) the counts come
+ * from the forward's own router scores: the TopK selection derives each k_i
+ * from z_i (as reflex_allocate with those scores would), writes it to k_out
+ * and selects with it; the state arrays are not read (they may be NULL), and
+ * the ROUTE stage must be among the selected stages (else REFLEX_EINVAL).
  */
 int reflex_step(const float* conf_prev1, const float* conf_prev2, const uint8_t* hist_len,
                 const uint8_t* masked, const int32_t* block_id, const int32_t* seq_offsets,

@@ -13,6 +13,8 @@ file's header lists which paper passage each function follows:
                       Expert Reallocation (forecast, Eq. 6-8, Eq. 9) + clip.
 * ``router_logits``   router scores of Sec. 3.2 (sequential fp32 fma chain).
 * ``select``          TopK of Eq. 2 and the normalised router weight.
+* ``rule_counts``     the Top-p and Expert-Threshold counts of the
+                      threshold-based comparison methods (App. B).
 * ``permutation``     (expert, token)-ordered pair list that executes Eq. 2.
 * ``moe_tokens``      Eq. 2 with SwiGLU experts (+ shared expert), fp64.
 * ``moe_stack``       a stack of such layers with the residual update
@@ -97,6 +99,8 @@ def _load():
     lib.oracle_router_logits.argtypes = [i32, p, p, i32, i32, i32, p]
     lib.oracle_select.restype = ctypes.c_int
     lib.oracle_select.argtypes = [p, p, i32, i32, i32, i32, p, p]
+    lib.oracle_rule_counts.restype = ctypes.c_int
+    lib.oracle_rule_counts.argtypes = [p, i32, i32, i32, f32, i32, i32, p]
     lib.oracle_permutation.restype = ctypes.c_int64
     lib.oracle_permutation.argtypes = [p, p, i32, i32, i32, p, p, p]
     lib.oracle_moe_tokens.restype = None
@@ -251,6 +255,25 @@ def select(z: np.ndarray, k: np.ndarray, k_max: int, renorm: bool = True):
     if rc != 0:
         raise ValueError("oracle_select: some k_t outside [1, min(k_max, E)]")
     return ids, alpha
+
+
+RULE_TOP_P = 1
+RULE_EXPERT_THRESHOLD = 2
+
+
+def rule_counts(z: np.ndarray, rule: int, threshold: float, k_min: int = 1,
+                k_max: int = 12) -> np.ndarray:
+    """Counts of the threshold-based comparison methods (App. B) from router
+    scores z [T, E]: rule 1 = Top-p (threshold p), 2 = Expert-Threshold
+    routing; clipped to [k_min, min(k_max, E)].  int32 [T]."""
+    z = _c(z, np.float32)
+    T, E = z.shape
+    k = np.empty(T, np.int32)
+    rc = _load().oracle_rule_counts(_ptr(z), T, E, int(rule), float(threshold),
+                                    int(k_min), int(k_max), _ptr(k))
+    if rc != 0:
+        raise ValueError("oracle_rule_counts: invalid rule or bounds")
+    return k
 
 
 def permutation(ids: np.ndarray, k: np.ndarray, E: int):

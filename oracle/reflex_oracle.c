@@ -30,6 +30,11 @@
  *                        contract the GPU router also follows).
  *   oracle_select        TopK_e(r, k_i) of Eq. 2 (ties: lower expert index)
  *                        and the normalised router weight alpha in fp64.
+ *   oracle_rule_counts   the counts of the threshold-based comparison
+ *                        methods (App. B): Top-p (smallest router-ranked
+ *                        prefix whose routing mass reaches p) and Expert-
+ *                        Threshold routing (experts whose routing mass
+ *                        exceeds a threshold), clipped to the count bounds.
  *   oracle_permutation   token-expert pairs sorted by (expert, token): the
  *                        per-expert row ranges that execute Eq. 2 sparsely.
  *   oracle_moe_tokens    Eq. 2 for a list of tokens: sum over selected experts
@@ -426,6 +431,83 @@ int oracle_select(const float* z, const int32_t* k, int32_t T, int32_t E,
             }
         }
     }
+    free(order);
+    return OR_OK;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Score-based count rules of the threshold-based comparison methods        */
+/* (App. B): the count of token t comes from its router scores z_t alone.   */
+/* The routing mass is the softmax of z_t over the E experts; the decision  */
+/* is taken in fp32 in this order (the order the GPU follows):             */
+/*   m   = max_e z_e                                                        */
+/*   u_e = exp_f32(z_e - m)                          (oracle_exp_f32)      */
+/*   S   : 32 lane sums s_l = ((0 + u_l) + u_{l+32}) + ..., l = 0 .. 31,    */
+/*         then for o = 16, 8, 4, 2, 1 every s_l <- s_l + s_{l xor o};      */
+/*         S = s_0                                                          */
+/*   rule 1, Top-p: ranks j = 1, 2, ... by (z desc, e asc);                 */
+/*         c_j = c_{j-1} + u_(j), c_0 = 0; k = the smallest j with          */
+/*         c_j / S >= thr (E when no j reaches it)                         */
+/*   rule 2, Expert threshold: k = #{e : u_e / S > thr}                    */
+/* then k is clipped to [k_min, min(k_max, E)] (the paper: [1, 12]).       */
+/* Returns OR_EINVAL for an unknown rule or bounds.                        */
+/* ------------------------------------------------------------------------ */
+int oracle_rule_counts(const float* z, int32_t T, int32_t E, int32_t rule,
+                       float thr, int32_t k_min, int32_t k_max, int32_t* k_out) {
+    if (E < 1 || (rule != 1 && rule != 2) || k_min < 1 || k_max < k_min) return OR_EINVAL;
+    int32_t kcap = k_max < E ? k_max : E;
+    int32_t klo = k_min < kcap ? k_min : kcap;
+    float* u = (float*)malloc(sizeof(float) * (size_t)E);
+    int32_t* order = (int32_t*)malloc(sizeof(int32_t) * (size_t)E);
+    for (int32_t t = 0; t < T; ++t) {
+        const float* zt = z + (int64_t)t * E;
+        float m = zt[0];
+        for (int32_t e = 1; e < E; ++e)
+            if (zt[e] > m) m = zt[e];
+        for (int32_t e = 0; e < E; ++e) u[e] = oracle_exp_f32(zt[e] - m);
+        float lane[32];
+        for (int32_t l = 0; l < 32; ++l) {
+            float acc = 0.0f;
+            for (int32_t e = l; e < E; e += 32) acc = acc + u[e];
+            lane[l] = acc;
+        }
+        for (int32_t o = 16; o > 0; o >>= 1) {
+            float nxt[32];
+            for (int32_t l = 0; l < 32; ++l) nxt[l] = lane[l] + lane[l ^ o];
+            for (int32_t l = 0; l < 32; ++l) lane[l] = nxt[l];
+        }
+        float S = lane[0];
+        int32_t k;
+        if (rule == 2) {
+            k = 0;
+            for (int32_t e = 0; e < E; ++e)
+                if (u[e] / S > thr) ++k;
+        } else {
+            /* rank order: repeatedly the best remaining expert */
+            for (int32_t e = 0; e < E; ++e) order[e] = e;
+            k = E;
+            float c = 0.0f;
+            for (int32_t j = 0; j < E; ++j) {
+                int32_t best = j;
+                for (int32_t q = j + 1; q < E; ++q) {
+                    int32_t eq = order[q], eb = order[best];
+                    if (zt[eq] > zt[eb] || (zt[eq] == zt[eb] && eq < eb)) best = q;
+                }
+                int32_t tmp = order[j];
+                order[j] = order[best];
+                order[best] = tmp;
+                c = c + u[order[j]];
+                if (c / S >= thr) {
+                    k = j + 1;
+                    break;
+                }
+            }
+        }
+        if (k < klo) k = klo;
+        if (k > kcap) k = kcap;
+        k_out[t] = k;
+    }
+    free(u);
     free(order);
     return OR_OK;
 }

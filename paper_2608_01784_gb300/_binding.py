@@ -33,6 +33,11 @@ REFLEX_SIGNAL_FRONTIER = 1
 REFLEX_SIGNAL_PROGRESS = 2
 REFLEX_SIGNAL_CONFIDENCE = 3
 REFLEX_SIGNAL_UNCERTAINTY = 4
+REFLEX_RULE_REFLEX = 0
+REFLEX_RULE_TOP_P = 1
+REFLEX_RULE_EXPERT_THRESHOLD = 2
+# the reflex_alloc_params layout above matches this ABI version
+ABI_VERSION = 113
 REFLEX_STAGE_ROUTE = 0x100
 REFLEX_STAGE_DISPATCH = 0x200
 REFLEX_STAGE_EXPERT_UP = 0x400
@@ -55,7 +60,8 @@ class reflex_alloc_params(ctypes.Structure):
                 ("theta", ctypes.c_float), ("w_cf", ctypes.c_float),
                 ("v_ref", ctypes.c_float), ("tau", ctypes.c_float),
                 ("signal", ctypes.c_int32), ("role_shuffle", ctypes.c_int32),
-                ("shuffle_seed", ctypes.c_uint64)]
+                ("shuffle_seed", ctypes.c_uint64), ("count_rule", ctypes.c_int32),
+                ("rule_threshold", ctypes.c_float)]
 
 
 class reflex_route_record(ctypes.Structure):
@@ -123,6 +129,9 @@ def load():
     lib.reflex_route_noalloc.restype = ctypes.c_int
     lib.reflex_route_noalloc.argtypes = [i32, P, P, P, i32, i32, i32, i32,
                                          ctypes.c_uint32, P, P, P, P]
+    if lib.reflex_abi_version() != ABI_VERSION:
+        raise ImportError(f"{_LIB_PATH} has ABI version {lib.reflex_abi_version()}, "
+                          f"this binding needs {ABI_VERSION}: rebuild it")
     _lib = lib
     return lib
 

@@ -36,18 +36,26 @@ def state_to_device(state: dict, device="cuda") -> dict:
 def allocate(state: dict, params: B.reflex_alloc_params, E: int = 0,
              stream=None, k_out: torch.Tensor | None = None,
              k_sum: torch.Tensor | None = None,
-             status: torch.Tensor | None = None):
+             status: torch.Tensor | None = None,
+             router_scores: torch.Tensor | None = None):
     """reflex_allocate on device state tensors -> (k int32 [T], k_sum int64 [1],
-    status int32 [1])."""
-    T = int(state["block_id"].numel())
-    nseq = int(state["active_block"].numel())
-    dev = state["block_id"].device
+    status int32 [1]).  With a score rule (params.count_rule) the counts come
+    from router_scores [T, E] fp32 and `state` may be None."""
+    if router_scores is not None:
+        T, E = int(router_scores.shape[0]), int(router_scores.shape[1])
+        dev = router_scores.device
+        nseq = 1
+    else:
+        T = int(state["block_id"].numel())
+        nseq = int(state["active_block"].numel())
+        dev = state["block_id"].device
     k_out = torch.empty(T, dtype=torch.int32, device=dev) if k_out is None else k_out
     k_sum = torch.zeros(1, dtype=torch.int64, device=dev) if k_sum is None else k_sum
     status = torch.zeros(1, dtype=torch.int32, device=dev) if status is None else status
-    B.reflex_allocate(None, state["conf1"], state["conf2"], state["hist_len"],
-                      state["masked"], state["block_id"], state["seq_offsets"],
-                      state["active_block"], T, nseq, E, params, k_out, k_sum,
+    st = state if state is not None else {}
+    B.reflex_allocate(router_scores, st.get("conf1"), st.get("conf2"), st.get("hist_len"),
+                      st.get("masked"), st.get("block_id"), st.get("seq_offsets"),
+                      st.get("active_block"), T, nseq, E, params, k_out, k_sum,
                       status, stream)
     return k_out, k_sum, status
 
@@ -71,7 +79,7 @@ def update_state(state: dict, conf_new: torch.Tensor, num_blocks: torch.Tensor,
 
 
 def step_launches(dtype: str, T: int, d: int, E: int, shared_inter: int,
-                  flags: int = B.REFLEX_FLAG_RENORM_TOPK) -> int:
+                  flags: int = B.REFLEX_FLAG_RENORM_TOPK, count_rule: int = 0) -> int:
     """Kernels one reflex_step call launches on the tcgen05 path, following the
     library's choices: the count kernel; the score kernel and the selection,
     or (bf16, renormalised weights, >= 128 experts, T E >= 2048 x 256,
@@ -80,11 +88,12 @@ def step_launches(dtype: str, T: int, d: int, E: int, shared_inter: int,
     CTA (short batches whose block masks fit in shared memory) or count and
     scan, then the gather, which also places the pairs; the gate/up and down
     GEMMs (and the shared expert's two); the combine.
-    Memsets are not kernels."""
-    n = 1
+    With a score count rule the selection derives the counts: no count
+    kernel and no screen.  Memsets are not kernels."""
+    n = 0 if count_rule else 1
     screen = (dtype == "bf16" and flags & B.REFLEX_FLAG_RENORM_TOPK and
               not flags & B.REFLEX_FLAG_EXACT_SCORES and d % 128 == 0 and E >= 128 and
-              T * E >= 2048 * 256)
+              T * E >= 2048 * 256 and not count_rule)
     n += 3 if screen else 2
     n += 1 if T <= 4096 and (T + 31) // 32 * E * 4 <= 160 * 1024 else 2
     n += 1 + 2 + (2 if shared_inter else 0) + 1

@@ -59,6 +59,45 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
+// ---- exp in fp32 from a published method ----------------------------------
+// Written from Cody & Waite's argument reduction with a degree-7 Taylor
+// polynomial, in separate IEEE operations (no contraction), so every call
+// gives the same bits on every launch: the FPS sigmoids of the count kernel
+// and the router-mass count rules of the selection take integer decisions
+// on it.
+__device__ __forceinline__ float pow2i(int e) {  // e in [-126, 127]
+  return __int_as_float((e + 127) << 23);
+}
+
+// e^x: x = k ln2 + r with k = nearest integer to x / ln2 (ties to even);
+// r = (x - k ln2_hi) - k ln2_lo (ln2_hi has 16 significant bits, so k ln2_hi
+// is exact); e^r by the Taylor series to r^7 in Horner form; the scale 2^k is
+// applied as two powers of two so that neither overflows and a subnormal
+// result is rounded once.
+__device__ __forceinline__ float exp_cw(float x) {
+  if (x != x) return x;
+  if (x >= 89.0f) return __int_as_float(0x7f800000);
+  if (x <= -104.0f) return 0.0f;
+  const float inv_ln2 = 1.44269502162933349609375f;
+  const float ln2_hi = 0.693145751953125f;
+  const float ln2_lo = 1.428606765330187045037746429443359375e-06f;
+  const float kf = rintf(__fmul_rn(x, inv_ln2));
+  const int k = static_cast<int>(kf);
+  float r = __fsub_rn(x, __fmul_rn(kf, ln2_hi));
+  r = __fsub_rn(r, __fmul_rn(kf, ln2_lo));
+  float p = 1.98412701138295233249664306640625e-04f;           // 1/7!
+  p = __fadd_rn(__fmul_rn(p, r), 1.388888922519981861114501953125e-03f);   // 1/6!
+  p = __fadd_rn(__fmul_rn(p, r), 8.333333767950534820556640625e-03f);      // 1/5!
+  p = __fadd_rn(__fmul_rn(p, r), 4.16666679084300994873046875e-02f);       // 1/4!
+  p = __fadd_rn(__fmul_rn(p, r), 1.6666667163372039794921875e-01f);        // 1/3!
+  p = __fadd_rn(__fmul_rn(p, r), 0.5f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  const int k1 = k >> 1;
+  const int k2 = k - k1;
+  return __fmul_rn(__fmul_rn(p, pow2i(k1)), pow2i(k2));
+}
+
 __device__ __forceinline__ void set_err(uint32_t* err, uint32_t bit) {
   if (err) atomicOr(err, bit);
 }

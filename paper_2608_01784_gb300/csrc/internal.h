@@ -15,6 +15,8 @@ struct AllocArgs {
   int signal;             // rank key of the Eq. 9 groups (REFLEX_SIGNAL_*)
   int role_shuffle;       // permute each sequence's final counts
   uint64_t shuffle_seed;  // splitmix64 seed of the permutation keys
+  int count_rule;         // REFLEX_RULE_*: 0 = this allocation, else a score rule
+  float rule_threshold;   // p of Top-p / the expert-threshold router weight
 };
 
 // ---- allocation (budget.cu) -----------------------------------------------
@@ -91,6 +93,15 @@ inline int64_t screen_z_rows(int T, int E, int d) {
   }
   return rows;
 }
+// The counts from the router scores (count rules 1 = Top-p, 2 = expert
+// threshold, threshold thr, clip [k_lo, min(k_hi, E)]) into k_out (and added
+// to k_sum, nullable, which the caller cleared), then ids / alpha [T, k_max]
+// as launch_router_select gives them for those counts; ids == nullptr:
+// counts only.
+cudaError_t launch_router_select_rule(const float* z, int T, int E, int k_hi, int k_lo,
+                                      int rule, float thr, int k_max, bool renorm,
+                                      int32_t* k_out, unsigned long long* k_sum,
+                                      int32_t* ids, float* alpha, cudaStream_t stream);
 // ids/alpha [T, k_max] from z and the counts k.
 cudaError_t launch_router_select(const float* z, const int32_t* k, int T,
                                  int E, int k_max, bool renorm, int32_t* ids,

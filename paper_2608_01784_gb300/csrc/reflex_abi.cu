@@ -12,6 +12,8 @@
 #include "internal.h"
 #include "reflex.h"
 
+static_assert(sizeof(reflex_alloc_params) == 64, "reflex_alloc_params layout (ABI 113)");
+
 namespace {
 
 using rx::WsHeader;
@@ -155,15 +157,16 @@ int map_err_bits(uint32_t bits) {
     if ((x) != cudaSuccess) return REFLEX_ECUDA;    \
   } while (0)
 
-// Argument checks of the allocation (reflex_allocate, reflex_step).
+bool score_rule(const reflex_alloc_params* p) {
+  return p->count_rule == REFLEX_RULE_TOP_P || p->count_rule == REFLEX_RULE_EXPERT_THRESHOLD;
+}
+
+// Argument checks of the allocation (reflex_allocate, reflex_step).  The
+// score rules read no refinement state: only the counts' output is needed.
 int check_alloc(const float* c1, const float* c2, const uint8_t* hl, const uint8_t* m,
                 const int32_t* bid, const int32_t* so, const int32_t* act, int32_t T,
                 int32_t B, const reflex_alloc_params* p, const int32_t* k_out) {
-  if (p == nullptr || T < 0 || B < 1) return REFLEX_EINVAL;
-  if (T > 0 && (c1 == nullptr || c2 == nullptr || hl == nullptr || m == nullptr ||
-                bid == nullptr || k_out == nullptr))
-    return REFLEX_EINVAL;
-  if (so == nullptr || act == nullptr) return REFLEX_EINVAL;
+  if (p == nullptr || T < 0) return REFLEX_EINVAL;
   if (p->k_min < 1 || p->k_min > p->k_max || p->k_base < 1 ||
       p->delta_role < 0 || p->delta_cur < 0)
     return REFLEX_EINVAL;
@@ -172,6 +175,17 @@ int check_alloc(const float* c1, const float* c2, const uint8_t* hl, const uint8
   if (p->signal < REFLEX_SIGNAL_FPS || p->signal > REFLEX_SIGNAL_UNCERTAINTY ||
       (p->role_shuffle != 0 && p->role_shuffle != 1))
     return REFLEX_EINVAL;
+  if (p->count_rule != REFLEX_RULE_REFLEX && !score_rule(p)) return REFLEX_EINVAL;
+  if (score_rule(p)) {
+    if (!std::isfinite(p->rule_threshold)) return REFLEX_EINVAL;
+    if (T > 0 && k_out == nullptr) return REFLEX_EINVAL;
+    return REFLEX_OK;
+  }
+  if (B < 1) return REFLEX_EINVAL;
+  if (T > 0 && (c1 == nullptr || c2 == nullptr || hl == nullptr || m == nullptr ||
+                bid == nullptr || k_out == nullptr))
+    return REFLEX_EINVAL;
+  if (so == nullptr || act == nullptr) return REFLEX_EINVAL;
   return REFLEX_OK;
 }
 
@@ -194,13 +208,15 @@ struct AllocCall {
 rx::AllocArgs alloc_args(const reflex_alloc_params* p) {
   return rx::AllocArgs{p->k_min, p->k_base,  p->k_max, p->delta_role, p->delta_cur,
                        p->q,     p->theta,   p->w_cf,  p->v_ref,      p->tau,
-                       p->signal, p->role_shuffle, p->shuffle_seed};
+                       p->signal, p->role_shuffle, p->shuffle_seed, p->count_rule,
+                       p->rule_threshold};
 }
 
 // The error word and the pair sum are stored outright by a single-sequence
-// count kernel; with several sequences each CTA adds its share to cleared words.
+// count kernel; with several sequences each CTA adds its share to cleared
+// words, and so does every warp of the score rules' selection.
 cudaError_t clear_alloc_outputs(const AllocCall& c, cudaStream_t s) {
-  if (c.B <= 1) return cudaSuccess;
+  if (c.B <= 1 && c.a.count_rule == REFLEX_RULE_REFLEX) return cudaSuccess;
   if (c.err) {
     const cudaError_t e = cudaMemsetAsync(c.err, 0, sizeof(int32_t), s);
     if (e != cudaSuccess) return e;
@@ -210,6 +226,7 @@ cudaError_t clear_alloc_outputs(const AllocCall& c, cudaStream_t s) {
 }
 
 cudaError_t launch_alloc(const AllocCall& c, int32_t T, cudaStream_t s, bool alongside) {
+  if (c.a.count_rule != REFLEX_RULE_REFLEX) return cudaSuccess;  // counts in the selection
   return rx::launch_budget(c.c1, c.c2, c.hl, c.m, c.bid, c.so, c.act, T, c.B, c.a, c.k_out,
                            c.k_sum, c.err, s, alongside);
 }
@@ -218,7 +235,7 @@ cudaError_t launch_alloc(const AllocCall& c, int32_t T, cudaStream_t s, bool alo
 
 extern "C" {
 
-int reflex_abi_version(void) { return 112; }
+int reflex_abi_version(void) { return 113; }
 
 const char* reflex_status_string(int s) {
   switch (s) {
@@ -249,6 +266,8 @@ void reflex_default_params(reflex_alloc_params* p) {
   p->signal = REFLEX_SIGNAL_FPS;
   p->role_shuffle = 0;
   p->shuffle_seed = 0;
+  p->count_rule = REFLEX_RULE_REFLEX;
+  p->rule_threshold = 0.0f;
 }
 
 int reflex_allocate(const float* router_scores, const float* conf_prev1,
@@ -258,12 +277,21 @@ int reflex_allocate(const float* router_scores, const float* conf_prev1,
                     int32_t T, int32_t B, int32_t E,
                     const reflex_alloc_params* p, int32_t* k_out,
                     int64_t* k_sum_out, int32_t* dev_status, void* stream) {
-  (void)router_scores;  // the REFLEX count rule does not read router scores
-  (void)E;
   const int chk = check_alloc(conf_prev1, conf_prev2, hist_len, masked, block_id,
                               seq_offsets, active_block, T, B, p, k_out);
   if (chk != REFLEX_OK) return chk;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (score_rule(p)) {
+    // the counts of the threshold-based rules come from the router scores
+    if (E < 1 || E > 1024 || (T > 0 && router_scores == nullptr)) return REFLEX_EINVAL;
+    if (dev_status != nullptr) RX_CUDA(cudaMemsetAsync(dev_status, 0, sizeof(int32_t), s));
+    if (k_sum_out != nullptr) RX_CUDA(cudaMemsetAsync(k_sum_out, 0, sizeof(int64_t), s));
+    RX_CUDA(rx::launch_router_select_rule(router_scores, T, E, p->k_max, p->k_min,
+                                          p->count_rule, p->rule_threshold, 1, true, k_out,
+                                          reinterpret_cast<unsigned long long*>(k_sum_out),
+                                          nullptr, nullptr, s));
+    return REFLEX_OK;
+  }
   const AllocCall c{conf_prev1, conf_prev2, hist_len, masked, block_id, seq_offsets,
                     active_block, B, alloc_args(p), k_out,
                     reinterpret_cast<unsigned long long*>(k_sum_out),
@@ -394,9 +422,11 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
   // routing 213 -> 113 us at 8192 tokens, layer 4.90 -> 4.35 ms at 65536;
   // below 2048 tokens, and with 64 experts at every size, the dense kernels
   // are faster).
+  // the score rules' counts need every score from the chain: no screen
+  const bool rule = ac != nullptr && ac->a.count_rule != REFLEX_RULE_REFLEX;
   const bool screen = dtype == REFLEX_DTYPE_BF16 && (flags & REFLEX_FLAG_RENORM_TOPK) &&
                       !(flags & REFLEX_FLAG_EXACT_SCORES) && d % 128 == 0 && E >= 128 &&
-                      static_cast<int64_t>(T) * E >= 2048 * 256;
+                      static_cast<int64_t>(T) * E >= 2048 * 256 && !rule;
   if ((stages & REFLEX_STAGE_ROUTE) && screen) {
     const int bn = rx::screen_bn(E), ks = rx::screen_splits(T, E, d);
     CUtensorMap mh, mw;
@@ -433,10 +463,19 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
     RX_CUDA(rx::launch_router_logits(dtype, hidden, w_router, T, d, E, z,
                                      reinterpret_cast<uint32_t*>(hdr),
                                      static_cast<int>(sizeof(WsHeader) / 4), err, sms, s, pf));
-    if (ac != nullptr) RX_CUDA(launch_alloc(*ac, T, s, true));
-    RX_CUDA(rx::launch_router_select(z, k, T, E, k_max,
-                                     (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
-                                     I32(L.ids), alpha, err, s));
+    if (rule) {
+      // k = ac->k_out: the selection writes the counts it derives
+      RX_CUDA(rx::launch_router_select_rule(z, T, E, ac->a.k_max < k_max ? ac->a.k_max : k_max,
+                                            ac->a.k_min,
+                                            ac->a.count_rule, ac->a.rule_threshold, k_max,
+                                            (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
+                                            ac->k_out, ac->k_sum, I32(L.ids), alpha, s));
+    } else {
+      if (ac != nullptr) RX_CUDA(launch_alloc(*ac, T, s, true));
+      RX_CUDA(rx::launch_router_select(z, k, T, E, k_max,
+                                       (flags & REFLEX_FLAG_RENORM_TOPK) != 0,
+                                       I32(L.ids), alpha, err, s));
+    }
   } else if (ac != nullptr) {
     RX_CUDA(launch_alloc(*ac, T, s, false));
   }
@@ -557,6 +596,11 @@ int reflex_step(const float* conf_prev1, const float* conf_prev2, const uint8_t*
                               seq_offsets, active_block, T, B, p, k_out);
   if (chk != REFLEX_OK) return chk;
   if (T > 0 && k_out == nullptr) return REFLEX_EINVAL;
+  // with a score rule the counts come out of the ROUTE stage
+  const uint32_t st_bits = flags & (REFLEX_STAGE_ROUTE | REFLEX_STAGE_DISPATCH |
+                                    REFLEX_STAGE_EXPERT_UP | REFLEX_STAGE_EXPERT_DOWN |
+                                    REFLEX_STAGE_COMBINE);
+  if (score_rule(p) && st_bits != 0 && !(st_bits & REFLEX_STAGE_ROUTE)) return REFLEX_EINVAL;
   const AllocCall c{conf_prev1, conf_prev2, hist_len, masked, block_id, seq_offsets,
                     active_block, B, alloc_args(p), k_out,
                     reinterpret_cast<unsigned long long*>(k_sum_out),

@@ -279,6 +279,129 @@ __global__ void __launch_bounds__(kSelWarps * 32)
   }
 }
 
+// Selection whose counts come from the router scores (the threshold-based
+// count rules, App. B): one warp per token derives k_t from the routing mass
+// softmax(z_t) in the fp32 order include/reflex.h states (exp_cw, lane sums
+// in ascending expert order, xor-butterfly over the lanes), writes it to
+// kout (and adds it to ksum), then selects TopK(z_t, k_t) and the weights as
+// select_kernel does.  rule 1 = Top-p (smallest prefix of ranks whose mass
+// reaches thr), rule 2 = expert threshold (experts whose mass exceeds thr);
+// either clipped to [k_lo, min(k_hi, E)].  ids == nullptr: counts only.
+template <int NPL>
+__global__ void __launch_bounds__(kSelWarps * 32)
+    select_rule_kernel(const float* __restrict__ z, int T, int E, int k_hi, int k_lo,
+                       int rule, float thr, int k_max, int renorm,
+                       int32_t* __restrict__ kout, unsigned long long* __restrict__ ksum,
+                       int32_t* __restrict__ ids, float* __restrict__ alpha) {
+  __shared__ float s_z[kSelWarps][32];
+  __shared__ int32_t s_e[kSelWarps][32];
+  grid_dep_wait();
+  grid_dep_launch();
+  const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = blockIdx.x * kSelWarps + wid;
+  if (t >= T) return;
+  const int kcap = k_hi < E ? k_hi : E;
+  const int klo = k_lo < kcap ? k_lo : kcap;
+  float zv[NPL];
+  unsigned long long key[NPL];
+  const float* zt = z + static_cast<int64_t>(t) * E;
+  float m = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    const int e = lane + 32 * i;
+    if (e < E) {
+      float v = zt[e];
+      v = (v == 0.0f) ? 0.0f : v;
+      zv[i] = v;
+      key[i] = (static_cast<unsigned long long>(order_bits(v)) << 32) |
+               static_cast<unsigned long long>(0xffffffffu - static_cast<uint32_t>(e));
+      m = fmaxf(m, v);
+    } else {
+      zv[i] = -INFINITY;
+      key[i] = 0ull;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  // u_e = exp(z_e - m); S = lane sums in ascending expert order, then the
+  // xor-butterfly (every lane ends with the same bits)
+  float u[NPL];
+  float S = 0.0f;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    u[i] = (lane + 32 * i < E) ? exp_cw(__fsub_rn(zv[i], m)) : 0.0f;
+    S = __fadd_rn(S, u[i]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) S = __fadd_rn(S, __shfl_xor_sync(0xffffffffu, S, o));
+  int kt = kcap;
+  if (rule == 2) {
+    int cnt = 0;
+#pragma unroll
+    for (int i = 0; i < NPL; ++i)
+      cnt += __popc(__ballot_sync(0xffffffffu,
+                                  lane + 32 * i < E && __fdiv_rn(u[i], S) > thr));
+    kt = cnt < klo ? klo : (cnt > kcap ? kcap : cnt);
+  }
+  float c = 0.0f;  // Top-p: mass of the ranks taken so far
+  // the ranks are needed to select, and by Top-p to count
+  const int rounds = (ids != nullptr || rule == 1) ? kt : 0;
+  for (int j = 0; j < rounds && j < kt; ++j) {
+    unsigned long long best = key[0];
+#pragma unroll
+    for (int i = 1; i < NPL; ++i) best = key[i] > best ? key[i] : best;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+      best = other > best ? other : best;
+    }
+    const int e = static_cast<int>(0xffffffffu - static_cast<uint32_t>(best & 0xffffffffull));
+    const float ze = from_order_bits(static_cast<uint32_t>(best >> 32));
+    if ((e & 31) == lane) {
+#pragma unroll
+      for (int i = 0; i < NPL; ++i)
+        if (i == (e >> 5)) key[i] = 0ull;
+    }
+    if (lane == 0) {
+      s_e[wid][j] = e;
+      s_z[wid][j] = ze;
+    }
+    if (rule == 1) {
+      c = __fadd_rn(c, exp_cw(__fsub_rn(ze, m)));
+      if (j + 1 >= klo && __fdiv_rn(c, S) >= thr) kt = j + 1;  // ends the loop
+    }
+  }
+  if (lane == 0) {
+    kout[t] = kt;
+    if (ksum != nullptr) atomicAdd(ksum, static_cast<unsigned long long>(kt));
+  }
+  if (ids == nullptr) return;
+  __syncwarp();
+  const float zmax = s_z[wid][0];
+  float all = 0.f;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i)
+    if (lane + 32 * i < E) all += expf(zv[i] - zmax);
+  const float mine = lane < kt ? expf(s_z[wid][lane] - zmax) : 0.f;
+  float sel = mine;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    all += __shfl_xor_sync(0xffffffffu, all, o);
+    sel += __shfl_xor_sync(0xffffffffu, sel, o);
+  }
+  const float denom = renorm ? sel : all;
+  for (int j = lane; j < k_max; j += 32) {
+    const int64_t o = static_cast<int64_t>(t) * k_max + j;
+    if (j < kt) {
+      ids[o] = s_e[wid][j];
+      alpha[o] = mine / denom;
+    } else {
+      ids[o] = -1;
+      alpha[o] = 0.f;
+    }
+  }
+}
+
 // Short-batch variant: too few (token, expert) chains to fill the GPU with
 // the widened-buffer tiles, so each CTA (4 warps) keeps 8 TM tokens x 64
 // experts, one 4-stage ring of 32-k raw chunks, and widens operands at use
@@ -1140,6 +1263,27 @@ cudaError_t launch_router_screen_select(const __nv_bfloat16* h, const __nv_bfloa
   if (E <= 512) return RX_SCREEN(16);
   return RX_SCREEN(32);
 #undef RX_SCREEN
+}
+
+cudaError_t launch_router_select_rule(const float* z, int T, int E, int k_hi, int k_lo,
+                                      int rule, float thr, int k_max, bool renorm,
+                                      int32_t* k_out, unsigned long long* k_sum,
+                                      int32_t* ids, float* alpha, cudaStream_t stream) {
+  if (T == 0) return cudaSuccess;
+  if (rule != 1 && rule != 2) return cudaErrorInvalidValue;
+  const dim3 grid((T + kSelWarps - 1) / kSelWarps);
+  const dim3 block(kSelWarps * 32);
+  const int r = renorm ? 1 : 0;
+#define RX_SEL_RULE(N)                                                                   \
+  launch_pdl(select_rule_kernel<N>, grid, block, 0, stream, z, T, E, k_hi, k_lo, rule, thr, \
+             k_max, r, k_out, k_sum, ids, alpha)
+  if (E <= 32) return RX_SEL_RULE(1);
+  if (E <= 64) return RX_SEL_RULE(2);
+  if (E <= 128) return RX_SEL_RULE(4);
+  if (E <= 256) return RX_SEL_RULE(8);
+  if (E <= 512) return RX_SEL_RULE(16);
+  return RX_SEL_RULE(32);
+#undef RX_SEL_RULE
 }
 
 cudaError_t launch_router_select(const float* z, const int32_t* k, int T,

@@ -48,7 +48,7 @@ def test_status_strings_and_version(lib):
     assert B.reflex_status_string(B.REFLEX_OK) == "ok"
     assert "workspace" in B.reflex_status_string(B.REFLEX_EWORKSPACE)
     assert B.reflex_status_string(999) == "unknown status"
-    assert B.reflex_abi_version() >= 112
+    assert B.reflex_abi_version() == B.ABI_VERSION == 113
 
 
 def test_default_params_are_the_paper_settings(lib):
@@ -61,7 +61,8 @@ def test_default_params_are_the_paper_settings(lib):
     # the ablation fields sit where the C struct has them (a layout mismatch
     # would show up as garbage here): FPS, no shuffle
     assert (p.signal, p.role_shuffle, p.shuffle_seed) == (B.REFLEX_SIGNAL_FPS, 0, 0)
-    assert ctypes.sizeof(B.reflex_alloc_params) == 56
+    assert (p.count_rule, p.rule_threshold) == (B.REFLEX_RULE_REFLEX, 0.0)
+    assert ctypes.sizeof(B.reflex_alloc_params) == 64
 
 
 def test_workspace_size(lib):
@@ -188,3 +189,43 @@ def test_step_launch_counts_of_the_bench_layers():
     # exact scores: the screen's three kernels become scores + selection
     exact = B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_FLAG_EXACT_SCORES
     assert api.step_launches("bf16", 8192, 2048, 256, 512, flags=exact) == 11
+
+
+def test_count_rule_host_rejections(lib):
+    # the score rules: every check returns before anything is launched
+    import ctypes
+    from paper_2608_01784_gb300 import _binding as B
+    for rule, thr in ((3, 0.2), (-1, 0.2), (B.REFLEX_RULE_TOP_P, float("nan")),
+                      (B.REFLEX_RULE_EXPERT_THRESHOLD, float("inf"))):
+        p = B.make_params(count_rule=rule, rule_threshold=thr)
+        assert lib.reflex_allocate(1, None, None, None, None, None, None, None, 4, 1, 8,
+                                   ctypes.byref(p), 1, None, None, None) == B.REFLEX_EINVAL
+    p = B.make_params(count_rule=B.REFLEX_RULE_TOP_P, rule_threshold=0.2)
+    # no score matrix, or an expert count outside [1, 1024]
+    assert lib.reflex_allocate(None, None, None, None, None, None, None, None, 4, 1, 8,
+                               ctypes.byref(p), 1, None, None, None) == B.REFLEX_EINVAL
+    for E in (0, 1025):
+        assert lib.reflex_allocate(1, None, None, None, None, None, None, None, 4, 1, E,
+                                   ctypes.byref(p), 1, None, None, None) == B.REFLEX_EINVAL
+    # nowhere to put the counts
+    assert lib.reflex_allocate(1, None, None, None, None, None, None, None, 4, 1, 8,
+                               ctypes.byref(p), None, None, None, None) == B.REFLEX_EINVAL
+
+    # reflex_step: the counts come out of the ROUTE stage, so a stage subset
+    # without it is rejected
+    def step(flags):
+        return lib.reflex_step(None, None, None, None, None, None, None, 1, ctypes.byref(p),
+                               1, None, None, 1, 1, 1, 1, 1, None, None, 0, 4, 256, 8, 128,
+                               4, flags, 256, 1 << 30, 1, None, None)
+    assert step(B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_DISPATCH) == B.REFLEX_EINVAL
+    assert step(B.REFLEX_STAGE_EXPERT_UP | B.REFLEX_STAGE_COMBINE) == B.REFLEX_EINVAL
+
+
+def test_default_params_count_rule_is_reflex(lib):
+    import ctypes
+    from paper_2608_01784_gb300 import _binding as B
+    p = B.reflex_alloc_params()
+    p.count_rule, p.rule_threshold = 9, 9.0
+    lib.reflex_default_params(ctypes.byref(p))
+    assert p.count_rule == B.REFLEX_RULE_REFLEX and p.rule_threshold == 0.0
+    assert ctypes.sizeof(B.reflex_alloc_params) == 64

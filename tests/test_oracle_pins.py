@@ -736,3 +736,94 @@ def test_stack_shares_counts_and_chains_inputs():
     zero = dict(layers[0], w_down=np.zeros_like(layers[0]["w_down"]))
     tr0 = oracle.moe_stack(h0, [zero], k, 2)
     assert np.array_equal(tr0[0]["h_out"], h0)
+
+
+# --------------------------------------------------------------------------
+# Score-based count rules of the threshold-based comparison methods (App. B):
+# Top-p = the smallest router-ranked prefix whose routing mass reaches p;
+# Expert-Threshold = the experts whose routing mass exceeds a threshold.
+# --------------------------------------------------------------------------
+def _softmax64(z):
+    z = np.asarray(z, np.float64)
+    e = np.exp(z - z.max(axis=1, keepdims=True))
+    return e / e.sum(axis=1, keepdims=True)
+
+
+@pytest.mark.parametrize("E", [8, 64])
+def test_rule_counts_uniform_scores_closed_form(E):
+    # equal scores: every expert has mass 1/E exactly (u_e = exp(0) = 1,
+    # S = E), so Top-p takes ceil(p E) experts and the threshold rule takes
+    # all of them below 1/E and none at or above it (then the clip)
+    z = np.full((1, E), 0.375, np.float32)
+    for j in (1, 3, E // 2, E):
+        p = j / E
+        assert oracle.rule_counts(z, 1, p, 1, E)[0] == j
+        assert oracle.rule_counts(z, 1, p - 0.5 / E, 1, E)[0] == j
+    assert oracle.rule_counts(z, 2, 0.99 / E, 1, 12)[0] == min(E, 12)
+    assert oracle.rule_counts(z, 2, 1.0 / E, 1, 12)[0] == 1
+    assert oracle.rule_counts(z, 2, 1.0 / E, 3, 12)[0] == 3
+
+
+def test_rule_counts_brute_force_over_subsets():
+    # E = 8: Top-p's count is the size of the smallest expert SUBSET whose
+    # mass reaches p (the top-j prefix is the heaviest j-subset), found by
+    # enumerating all 255 subsets in fp64; the threshold count is the number
+    # of experts above the threshold in fp64.  Tokens whose fp64 masses lie
+    # within 1e-5 of the threshold are left out (the oracle decides in fp32).
+    rng = np.random.default_rng(17)
+    T, E = 3000, 8
+    z = (rng.standard_normal((T, E)) * rng.uniform(0.2, 3.0, (T, 1))).astype(np.float32)
+    P = _softmax64(z)
+    masks = np.array([[(s >> e) & 1 for e in range(E)] for s in range(1, 1 << E)],
+                     np.float64)
+    sizes = masks.sum(axis=1)
+    mass = P @ masks.T                       # [T, 255] mass of every subset
+    checked = 0
+    for p in (0.15, 0.2, 0.5, 0.8, 0.95):
+        k = oracle.rule_counts(z, 1, p, 1, E)
+        ok = np.all(np.abs(mass - p) > 1e-5, axis=1)
+        want = np.where(mass >= p, sizes[None, :], E + 1).min(axis=1)
+        assert np.array_equal(k[ok], want[ok].astype(np.int32)), p
+        checked += int(ok.sum())
+    for thr in (0.05, 0.1, 0.125, 0.2, 0.4):
+        k = oracle.rule_counts(z, 2, thr, 1, E)
+        ok = np.all(np.abs(P - thr) > 1e-6, axis=1)
+        want = np.clip((P > thr).sum(axis=1), 1, E)
+        assert np.array_equal(k[ok], want[ok].astype(np.int32)), thr
+        checked += int(ok.sum())
+    assert checked > 0.99 * 10 * T
+
+
+def test_rule_counts_one_dominant_expert_and_monotone():
+    rng = np.random.default_rng(3)
+    z = np.zeros((1, 64), np.float32)
+    z[0, 17] = 12.0                          # mass 0.99..: one expert suffices
+    assert oracle.rule_counts(z, 1, 0.9, 1, 12)[0] == 1
+    assert oracle.rule_counts(z, 2, 0.01, 1, 12)[0] == 1
+    assert oracle.rule_counts(z, 1, 0.9, 2, 12)[0] == 2          # k_min clip
+    z = rng.standard_normal((500, 64)).astype(np.float32)
+    ps = [0.05, 0.15, 0.2, 0.3, 0.6, 0.9]
+    kp = np.stack([oracle.rule_counts(z, 1, p, 1, 12) for p in ps])
+    assert np.all(np.diff(kp, axis=0) >= 0)          # more mass, more experts
+    ts = [0.005, 0.0156, 0.019, 0.0215, 0.03, 0.08]
+    kt = np.stack([oracle.rule_counts(z, 2, t, 1, 12) for t in ts])
+    assert np.all(np.diff(kt, axis=0) <= 0)          # higher bar, fewer experts
+    assert kp.min() >= 1 and kp.max() <= 12 and kt.min() >= 1 and kt.max() <= 12
+    # p above the total mass: the upper clip
+    assert np.all(oracle.rule_counts(z, 1, 1.5, 1, 12) == 12)
+
+
+def test_rule_counts_route_the_selected_prefix():
+    # the count and the selection agree: the top-k ids of the oracle's
+    # selection with the Top-p counts carry at least mass p (fp64), and one
+    # fewer expert carries less (away from the boundary)
+    rng = np.random.default_rng(8)
+    z = (rng.standard_normal((400, 64)) * 1.5).astype(np.float32)
+    P = _softmax64(z)
+    k = oracle.rule_counts(z, 1, 0.3, 1, 64)
+    ids, _ = oracle.select(z, k, 64)
+    for t in range(z.shape[0]):
+        sel = ids[t, :k[t]]
+        m = P[t, sel].sum()
+        if abs(m - 0.3) > 1e-5 and abs(m - P[t, sel[-1]] - 0.3) > 1e-5:
+            assert m >= 0.3 and (k[t] == 1 or m - P[t, sel[-1]] < 0.3)
