@@ -42,6 +42,10 @@ constexpr int BM = kTileM;   // 128
 constexpr int BK = 64;       // 64 bf16 = 128 bytes = one swizzle row
 constexpr int UMMA_K = 16;
 constexpr int kThreads = 192;
+// scores mode: four more warps (6-9) that sum the squares of each A row from
+// the shared-memory stages while the MMAs read them (token norms for the
+// router screen's interval)
+constexpr int kThreadsScores = 320;
 constexpr int kRingBytes = 192 * 1024;  // TMA ring budget per CTA
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr uint64_t kDrainNs = 1000000000ull;
@@ -83,6 +87,8 @@ struct KParams {
   int defer_wait;
   // SwiGLU: map_b is the 3D {K, inter, 2 groups} map of tc_gate_up_3d
   int b3d;
+  // scores mode, k_splits == 1: sum of squares of every A row (fp32), nullable
+  float* norm_out;
 };
 
 // ---- PTX wrappers ---------------------------------------------------------
@@ -265,7 +271,7 @@ __device__ __forceinline__ bool decode_tile(const KParams& p, int t, Tile& o) {
 }
 
 template <int BN, int MODE>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(MODE == kModeScores ? kThreadsScores : kThreads, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap map_a,
                         const __grid_constant__ CUtensorMap map_b,
                         const KParams p) {
@@ -288,10 +294,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
+  const bool norms = MODE == kModeScores && p.norm_out != nullptr;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], norms ? 5 : 1);  // the MMA commit (+ 4 norm warps)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
@@ -419,6 +426,57 @@ __global__ void __launch_bounds__(kThreads, 1)
       // MMAs in flight must finish before TMEM is freed
       mma_commit(smem_addr(drain));
       mbar_wait(drain, 0, nullptr, kDrainNs);
+    }
+  } else if (MODE == kModeScores && warp >= 6) {
+    // ---------------- row norms (scores mode) ----------------
+    // warp 6 + q sums the squares of A rows 32 q .. 32 q + 31 of every tile,
+    // one row per lane, reading each stage as the MMAs do and releasing it
+    // on the stage's "empty" barrier next to the MMA commit
+    if (norms) {
+      const int r = (warp - 6) * 32 + lane;
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+        Tile tl;
+        const bool tile_ok = decode_tile(p, t, tl);
+        float ss = 0.f;
+        for (int kb = 0; kb < nk; ++kb) {
+          // every lane observes the stage's completion before reading it
+          const bool w = __all_sync(0xffffffffu,
+                                    mbar_wait(&full[stage], phase, abort_flag, kWaitNs));
+          if (!w) {
+            ok = false;
+            break;
+          }
+          // row r of the 128-byte-swizzled A stage: 16-byte chunk c at
+          // r * 128 + ((c ^ (r & 7)) << 4)
+          const uint8_t* rowp = sa + stage * C::kABytes + r * 128;
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const uint4 q = *reinterpret_cast<const uint4*>(rowp + ((c ^ (r & 7)) << 4));
+            const uint32_t wd[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const float lo = __uint_as_float(wd[i] << 16);
+              const float hi = __uint_as_float(wd[i] & 0xffff0000u);
+              ss = fmaf(lo, lo, ss);
+              ss = fmaf(hi, hi, ss);
+            }
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive1(smem_addr(&empty[stage]));
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (ok && tile_ok && r < tl.rows) p.norm_out[tl.row0 + r] = ss;
+      }
+      if (!ok && lane == 0) {
+        if (!*abort_flag) set_err(p.err, kErrTimeout);
+        *abort_flag = 1;
+      }
     }
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
@@ -559,6 +617,7 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.n_valid = 0;
   p.defer_wait = 0;
   p.b3d = MODE == kModeSwiGLU && a.b_gate_up_3d ? 1 : 0;
+  p.norm_out = nullptr;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);
@@ -583,7 +642,10 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
 // CTAs' epilogue warps arrive on the leader's "accumulator empty" barrier.
 // Every barrier wait is bounded, as in the 1-SM kernel.
 // ===========================================================================
-constexpr int kThreads2 = 192;
+// warps: 0 TMA producer, 1 MMA issuer (leader), 2-9 epilogue (two warps per
+// TMEM lane quarter, each draining half of the accumulator's columns)
+constexpr int kThreads2 = 320;
+constexpr int kEpiWarps2 = 8;
 
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
@@ -607,8 +669,12 @@ __device__ __forceinline__ void mbar_expect_tx_cluster(uint32_t cl_bar, uint32_t
                "r"(bytes)
                : "memory");
 }
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cl_bar) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cl_bar)
+// Arrival that orders nothing but the arriving thread's own progress: used to
+// hand a TMEM accumulator back once its last tcgen05.ld has completed
+// (tcgen05.wait::ld); the epilogue's global stores need not be visible to
+// the MMA issuer, so no release fence makes them drain first.
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t cl_bar) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cl_bar)
                : "memory");
 }
 // TMA tile load whose completion is counted on a barrier in either CTA of the pair.
@@ -656,8 +722,37 @@ struct Cfg2 {
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kStages = kRingBytes / kStageBytes;  // 6
   static constexpr int kTmemCols = 2 * BN;       // two accumulators
-  static constexpr int kSmemBytes = kStages * kStageBytes + 256 + 1024;
+  static constexpr int kStagingBytes = 32 * 128; // per epilogue warp: 32 rows x 128 B
+  static constexpr int kSmemBytes =
+      kStages * kStageBytes + 256 + kEpiWarps2 * kStagingBytes + 1024;
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
 };
+
+// The epilogue's bf16 rows reach global memory through a per-warp staging
+// tile: each thread writes its row's 128 bytes (16-byte chunk j at position
+// j ^ (row & 7), so the 32 rows' writes spread over the banks), then each
+// store instruction of the warp writes four whole 128-byte row segments
+// (lane l: row 4 i + l / 8, chunk l % 8).  Per-lane stores of 16 bytes to 32
+// different rows cost one L2 request per 16 bytes, as many requests as the
+// TMA loads of the main loop; this costs one per 128 bytes.
+__device__ __forceinline__ void stage_chunk(uint8_t* stg, int lane, int j, const uint4& v) {
+  *reinterpret_cast<uint4*>(stg + lane * 128 + ((j ^ (lane & 7)) << 4)) = v;
+}
+// rows [0, nrows) of the staging tile to out rows row_base + r, columns
+// col0 .. col0 + 63 (bf16), row stride ldo
+__device__ __forceinline__ void flush_staging(const uint8_t* stg, int lane,
+                                              __nv_bfloat16* out, int64_t row_base, int ldo,
+                                              int col0, int nrows) {
+  __syncwarp();
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int r = 4 * i + (lane >> 3), c = lane & 7;
+    const uint4 v = *reinterpret_cast<const uint4*>(stg + r * 128 + ((c ^ (r & 7)) << 4));
+    if (r < nrows)
+      *reinterpret_cast<uint4*>(out + (row_base + r) * ldo + col0 + 8 * c) = v;
+  }
+  __syncwarp();
+}
 
 template <int MODE>
 __global__ void __launch_bounds__(kThreads2, 1)
@@ -694,7 +789,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 8);  // 4 epilogue warps x 2 CTAs
+      mbar_init(&acc_empty[b], 2 * kEpiWarps2);  // every epilogue warp of both CTAs
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -813,8 +908,16 @@ __global__ void __launch_bounds__(kThreads2, 1)
     }
   } else if (warp >= 2) {
     // ---------------- epilogue (each CTA: its 128 rows) ----------------
+    // warp w drains TMEM lanes 32 (w % 4) .. +31 (its quarter of the rows)
+    // and one half of the columns: warps 2-5 the first, 6-9 the second.
+    // The TMEM loads of a half are issued two chunks at a time before one
+    // wait; once the last chunk is in registers the accumulator is handed
+    // back (relaxed arrive), and the conversion and stores of that chunk
+    // overlap the next tile's MMAs.
     const int quarter = warp & 3;
-    const int row = static_cast<int>(rank) * BM + quarter * 32 + lane;  // row within the 256
+    const int half = (warp - 2) >> 2;
+    const int wrow0 = static_cast<int>(rank) * BM + quarter * 32;  // warp's first row in the 256
+    uint8_t* stg = smem + kStages * C::kStageBytes + 256 + (warp - 2) * C::kStagingBytes;
     const uint32_t acc_empty_leader0 = map_to_rank(smem_addr(&acc_empty[0]), 0);
     const uint32_t acc_empty_leader1 = map_to_rank(smem_addr(&acc_empty[1]), 0);
     int lt = 0;
@@ -836,58 +939,71 @@ __global__ void __launch_bounds__(kThreads2, 1)
       tc_fence_after();
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                              static_cast<uint32_t>(ab * BN);
-      const bool store = tile_ok && row < tl.rows;
-      __nv_bfloat16* orow = p.out + static_cast<int64_t>(tl.row0 + (store ? row : 0)) * p.ldo;
+      // rows of this warp that belong to the tile (0 when the tile is bad)
+      const int nrows = tile_ok ? max(0, min(32, tl.rows - wrow0)) : 0;
+      const int64_t row_base = static_cast<int64_t>(tl.row0) + wrow0;
+      const uint32_t release_bar = ab ? acc_empty_leader1 : acc_empty_leader0;
+      auto hand_back = [&]() {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster_relaxed(release_bar);
+      };
       if (MODE == kModeSwiGLU) {
-#pragma unroll 1
-        for (int c = 0; c < BN / 2; c += 32) {
+        // output columns [64 half, +64): gate at c, up at BN/2 + c; both
+        // 32-column rounds fill one 128-byte staging row
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int c = half * 64 + 32 * r;
           uint32_t g[32], u[32];
           tmem_ld32(tbase + c, g);
           tmem_ld32(tbase + BN / 2 + c, u);
           tmem_ld_wait();
-          if (store) {
-            uint32_t packed[16];
+          if (r == 1) hand_back();
+          uint32_t packed[16];
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
-              const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
-              const float a0 = g0 / (1.0f + __expf(-g0)) * u0;
-              const float a1 = g1 / (1.0f + __expf(-g1)) * u1;
-              __nv_bfloat162 h2 = __floats2bfloat162_rn(a0, a1);
-              packed[i] = *reinterpret_cast<uint32_t*>(&h2);
-            }
-            uint4* dst = reinterpret_cast<uint4*>(orow + tl.n * (BN / 2) + c);
-#pragma unroll
-            for (int v = 0; v < 4; ++v)
-              dst[v] = make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
-                                  packed[4 * v + 3]);
+          for (int i = 0; i < 16; ++i) {
+            const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+            const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+            const float a0 = g0 / (1.0f + __expf(-g0)) * u0;
+            const float a1 = g1 / (1.0f + __expf(-g1)) * u1;
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(a0, a1);
+            packed[i] = *reinterpret_cast<uint32_t*>(&h2);
           }
+#pragma unroll
+          for (int v = 0; v < 4; ++v)
+            stage_chunk(stg, lane, 4 * r + v,
+                        make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
+                                   packed[4 * v + 3]));
         }
+        flush_staging(stg, lane, p.out, row_base, p.ldo, tl.n * (BN / 2) + half * 64, nrows);
       } else {
-#pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
-          uint32_t v32[32];
-          tmem_ld32(tbase + c, v32);
+        // columns [128 half, +128) in two rounds of 64 (one staging row each)
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int c = half * 128 + 64 * r;
+          uint32_t v0[32], v1[32];
+          tmem_ld32(tbase + c, v0);
+          tmem_ld32(tbase + c + 32, v1);
           tmem_ld_wait();
-          if (store) {
-            uint32_t packed[16];
+          if (r == 1) hand_back();
+          uint32_t packed[32];
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              __nv_bfloat162 h2 = __floats2bfloat162_rn(__uint_as_float(v32[2 * i]),
-                                                        __uint_as_float(v32[2 * i + 1]));
-              packed[i] = *reinterpret_cast<uint32_t*>(&h2);
-            }
-            uint4* dst = reinterpret_cast<uint4*>(orow + tl.n * BN + c);
-#pragma unroll
-            for (int v = 0; v < 4; ++v)
-              dst[v] = make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
-                                  packed[4 * v + 3]);
+          for (int i = 0; i < 16; ++i) {
+            __nv_bfloat162 h0 = __floats2bfloat162_rn(__uint_as_float(v0[2 * i]),
+                                                      __uint_as_float(v0[2 * i + 1]));
+            __nv_bfloat162 h1 = __floats2bfloat162_rn(__uint_as_float(v1[2 * i]),
+                                                      __uint_as_float(v1[2 * i + 1]));
+            packed[i] = *reinterpret_cast<uint32_t*>(&h0);
+            packed[16 + i] = *reinterpret_cast<uint32_t*>(&h1);
           }
+#pragma unroll
+          for (int v = 0; v < 8; ++v)
+            stage_chunk(stg, lane, v,
+                        make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
+                                   packed[4 * v + 3]));
+          flush_staging(stg, lane, p.out, row_base, p.ldo, tl.n * BN + c, nrows);
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(ab ? acc_empty_leader1 : acc_empty_leader0);
     }
   }
 
@@ -927,6 +1043,7 @@ cudaError_t launch_pair_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.n_valid = 0;
   p.defer_wait = 0;
   p.b3d = 0;
+  p.norm_out = nullptr;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   int pairs = a.num_sms / 2;
@@ -962,11 +1079,11 @@ cudaError_t launch_down_tc(const TcGemmArgs& a, int bn, cudaStream_t stream) {
 template <int BN>
 cudaError_t launch_scores_impl(const TcGemmArgs& a, int k_splits, float* out,
                                int64_t split_stride, int n_valid, bool defer_wait,
-                               cudaStream_t stream) {
+                               float* row_norms, cudaStream_t stream) {
   using C = Cfg<BN>;
   auto kernel = grouped_gemm_kernel<BN, kModeScores>;
   if (a.g.offsets != nullptr || k_splits < 1 || (a.K / BK) % k_splits != 0 ||
-      a.K % BK != 0 || n_valid < 1)
+      a.K % BK != 0 || n_valid < 1 || (row_norms != nullptr && k_splits != 1))
     return cudaErrorInvalidValue;
   cudaError_t e = cudaFuncSetAttribute(
       kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
@@ -989,11 +1106,12 @@ cudaError_t launch_scores_impl(const TcGemmArgs& a, int k_splits, float* out,
   p.n_valid = n_valid;
   p.defer_wait = defer_wait ? 1 : 0;
   p.b3d = 0;
+  p.norm_out = row_norms;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles * k_splits;
   if (max_tiles == 0) return cudaSuccess;
   const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);
-  return launch_pdl(kernel, dim3(grid), dim3(kThreads), C::kSmemBytes, stream, *a.map_a,
-                    *a.map_b, p);
+  return launch_pdl(kernel, dim3(grid), dim3(kThreadsScores), C::kSmemBytes, stream,
+                    *a.map_a, *a.map_b, p);
 }
 
 // SwiGLU loads gate and up halves as two boxes of bn/2 rows; down loads one
@@ -1002,11 +1120,13 @@ int tc_b_box_rows(bool swiglu, int bn) { return swiglu ? bn / 2 : bn; }
 
 cudaError_t launch_scores_tc(const TcGemmArgs& a, int bn, int k_splits, float* out,
                              int64_t split_stride, int n_valid, bool defer_wait,
-                             cudaStream_t stream) {
+                             cudaStream_t stream, float* row_norms) {
   if (bn == 64)
-    return launch_scores_impl<64>(a, k_splits, out, split_stride, n_valid, defer_wait, stream);
+    return launch_scores_impl<64>(a, k_splits, out, split_stride, n_valid, defer_wait,
+                                  row_norms, stream);
   if (bn == 128)
-    return launch_scores_impl<128>(a, k_splits, out, split_stride, n_valid, defer_wait, stream);
+    return launch_scores_impl<128>(a, k_splits, out, split_stride, n_valid, defer_wait,
+                                   row_norms, stream);
   return cudaErrorInvalidValue;
 }
 

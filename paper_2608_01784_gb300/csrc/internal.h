@@ -93,6 +93,17 @@ inline int64_t screen_z_rows(int T, int E, int d) {
   }
   return rows;
 }
+// Batched screen for E <= 64 (bf16, renormalised weights): z holds the
+// tensor-core estimates [T, E] (one K slice), hss the tokens' sums of
+// squares, nw the experts' norms (wnorm_kernel); map_h / map_w are 2D maps of
+// the hidden states [T, d] and the router weights [E, d] with 64 x 64 boxes
+// (128-byte swizzle).  Writes ids / alpha and the candidates' exact scores
+// into z.
+cudaError_t launch_router_screen_batch(const CUtensorMap* map_h, const CUtensorMap* map_w,
+                                       float* z, const float* hss, const float* nw,
+                                       const int32_t* k, int T, int E, int d, int k_max,
+                                       int32_t* ids, float* alpha, uint32_t* err,
+                                       cudaStream_t stream);
 // The counts from the router scores (count rules 1 = Top-p, 2 = expert
 // threshold, threshold thr, clip [k_lo, min(k_hi, E)]) into k_out (and added
 // to k_sum, nullable, which the caller cleared), then ids / alpha [T, k_max]
@@ -194,9 +205,11 @@ int tc_b_box_rows(bool swiglu, int bn);
 // (B tensor map box of bn rows); a.K / 64 must be a multiple of k_splits.
 // defer_wait: launched right behind a kernel that writes none of its inputs
 // or outputs (it then overlaps that kernel and waits for it before exiting).
+// row_norms (nullable, k_splits == 1 only): the sum of squares of every A
+// row (fp32, one per row), computed from the staged A tiles.
 cudaError_t launch_scores_tc(const TcGemmArgs& a, int bn, int k_splits, float* out,
                              int64_t split_stride, int n_valid, bool defer_wait,
-                             cudaStream_t stream);
+                             cudaStream_t stream, float* row_norms = nullptr);
 // CTA-pair (2-SM, cta_group::2) variants: 256 x 256 tiles, cluster of two
 // CTAs; A and B tensor maps both with boxes of 128 rows; needs
 // GroupRows::mt2_prefix in grouped mode.  n_total must be a multiple of 128

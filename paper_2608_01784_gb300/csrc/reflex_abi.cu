@@ -21,12 +21,14 @@ using rx::WsHeader;
 constexpr size_t kAlign = 256;
 // gate/up weight bytes handed to the L2 while the router scores run
 constexpr uint64_t kRouterL2Prefetch = 64ull << 20;
+// tokens from which layers with up to 64 experts screen their router scores
+constexpr int32_t kBatchScreenMinTokens = 8192;
 size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 // Byte offsets of every workspace region (all 256-byte aligned).
 struct Layout {
-  size_t hdr, z, wnorm, ids, alpha, blk_count, blk_mask, blk_off, counts, offsets, mt_prefix,
-      mt2_prefix, perm, row_of, xperm, amid, ash, ysh, total;
+  size_t hdr, z, wnorm, tnorm, ids, alpha, blk_count, blk_mask, blk_off, counts, offsets,
+      mt_prefix, mt2_prefix, perm, row_of, xperm, amid, ash, ysh, total;
   int64_t cap_rows;
   int nblk;
 };
@@ -59,6 +61,7 @@ Layout make_layout(int32_t dtype, int32_t T, int32_t d, int32_t E,
   const int64_t zrows = dtype == REFLEX_DTYPE_F32 ? T : rx::screen_z_rows(T, E, d);
   L.z = take(static_cast<size_t>(zrows) * E * 4);
   L.wnorm = take(static_cast<size_t>(E) * 4);
+  L.tnorm = take(static_cast<size_t>(T) * 4);  // the batched screen's token sums of squares
   L.ids = take(cap * 4);
   L.alpha = take(cap * 4);
   L.blk_count = take(static_cast<size_t>(nblk) * E * 4);
@@ -427,7 +430,30 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
   const bool screen = dtype == REFLEX_DTYPE_BF16 && (flags & REFLEX_FLAG_RENORM_TOPK) &&
                       !(flags & REFLEX_FLAG_EXACT_SCORES) && d % 128 == 0 && E >= 128 &&
                       static_cast<int64_t>(T) * E >= 2048 * 256 && !rule;
-  if ((stages & REFLEX_STAGE_ROUTE) && screen) {
+  // the same screen for few experts and many tokens: the score GEMM also
+  // sums the squares of the token rows, and a batched recheck streams the
+  // CTA's token rows and the expert rows through shared memory, one chain
+  // per candidate pair (router.cu)
+  const bool batch_screen = dtype == REFLEX_DTYPE_BF16 && (flags & REFLEX_FLAG_RENORM_TOPK) &&
+                            !(flags & REFLEX_FLAG_EXACT_SCORES) && !rule && E <= 64 &&
+                            d % 64 == 0 && T >= kBatchScreenMinTokens;
+  if ((stages & REFLEX_STAGE_ROUTE) && batch_screen) {
+    CUtensorMap mh, mw, mhb, mwb;
+    if (!make_map(&mh, hidden, T, d, rx::kTileM) || !make_map(&mw, w_router, E, d, 64) ||
+        !make_map(&mhb, hidden, T, d, 64) || !make_map(&mwb, w_router, E, d, 64))
+      return REFLEX_ECUDA;
+    float* nw = reinterpret_cast<float*>(ws + L.wnorm);
+    float* hss = reinterpret_cast<float*>(ws + L.tnorm);
+    RX_CUDA(rx::launch_router_wnorm(static_cast<const __nv_bfloat16*>(w_router), E, d, nw,
+                                    reinterpret_cast<uint32_t*>(hdr),
+                                    static_cast<int>(sizeof(WsHeader) / 4), s));
+    rx::GroupRows rows{nullptr, nullptr, nullptr, nullptr, 1, T, T};
+    rx::TcGemmArgs sa{&mh, &mw, d, E, 0, 0, rows, nullptr, E, err, sms};
+    RX_CUDA(rx::launch_scores_tc(sa, 64, 1, z, static_cast<int64_t>(T) * E, E, true, s, hss));
+    if (ac != nullptr) RX_CUDA(launch_alloc(*ac, T, s, true));
+    RX_CUDA(rx::launch_router_screen_batch(&mhb, &mwb, z, hss, nw, k, T, E, d, k_max,
+                                           I32(L.ids), alpha, err, s));
+  } else if ((stages & REFLEX_STAGE_ROUTE) && screen) {
     const int bn = rx::screen_bn(E), ks = rx::screen_splits(T, E, d);
     CUtensorMap mh, mw;
     if (!make_map(&mh, hidden, T, d, rx::kTileM) || !make_map(&mw, w_router, E, d, bn))

@@ -1148,6 +1148,314 @@ __global__ void __launch_bounds__(kScreenWarps * 32)
   }
 }
 
+// ---- batched screen recheck (bf16, up to 64 experts) ------------------------
+// The screen of screen_select_kernel for many tokens and few experts, where
+// one warp per token leaves most lanes idle and streams expert rows from L2
+// one lane at a time.  A CTA owns 64 tokens:
+//   1. screening (8 warps, 8 tokens each): from the tensor-core estimates
+//      z~ and the row norms (the score GEMM's sums of squares, ||w_e|| from
+//      wnorm_kernel) the interval z~ -/+ del of every (token, expert), the
+//      k_t-th largest lower end L, and the candidates (upper end >= L) as a
+//      per-token bit mask; a prefix over the tokens lays the (token, expert)
+//      candidate pairs out in shared memory;
+//   2. chains: a producer warp streams 64-k chunks of the CTA's 64 token rows
+//      and of the 64 expert rows through a 4-stage TMA ring (128-byte
+//      swizzle); each compute thread advances the canonical fma chain of two
+//      candidate pairs over the chunk (more than 512 pairs: the rows are
+//      streamed again for the next 512);
+//   3. selection (a warp per token): TopK over the candidates' exact scores
+//      with the keys and tie rule of select_kernel, the weights with its
+//      arithmetic (the same bits), and the exact scores into z.
+constexpr int kBatchT = 64;                   // tokens per CTA
+constexpr int kBatchE = 64;                   // expert rows per stage (E <= 64)
+constexpr int kBatchStages = 4;
+constexpr int kBatchCompute = 256;            // 8 compute warps
+constexpr int kBatchThreads = kBatchCompute + 32;  // + the producer warp
+constexpr int kBatchSlots = 2 * kBatchCompute;     // candidate pairs per pass
+constexpr uint32_t kBatchTokBytes = kBatchT * 128;
+constexpr uint32_t kBatchStageBytes = kBatchTokBytes + kBatchE * 128;
+constexpr uint64_t kBatchWaitNs = 2000000000ull;
+constexpr uint64_t kBatchDrainNs = 1000000000ull;
+struct BatchSmem {
+  uint64_t full[kBatchStages];
+  uint64_t empty[kBatchStages];
+  uint32_t mask[kBatchT][2];
+  int32_t cnt[kBatchT];
+  int32_t kt[kBatchT];
+  int32_t off[kBatchT + 1];
+  float sel_z[8][32];
+  int32_t sel_e[8][32];
+  volatile int abort;
+  uint16_t pair[kBatchT * kBatchE];           // (token << 8) | expert
+  float zc[kBatchT * kBatchE];                // exact scores of the pairs
+};
+constexpr size_t kBatchSmemBytes =
+    1024 + kBatchStages * kBatchStageBytes + sizeof(BatchSmem);
+
+// the 16-byte chunk q of row r of a 128-byte-swizzled 64-column box
+__device__ __forceinline__ uint4 swz_ld16(const uint8_t* box, int r, int q) {
+  return *reinterpret_cast<const uint4*>(box + r * 128 + ((q ^ (r & 7)) << 4));
+}
+__device__ __forceinline__ void chain8(float& acc, const uint4& a, const uint4& b) {
+  fma_lo(acc, a.x, b.x);
+  fma_hi(acc, a.x, b.x);
+  fma_lo(acc, a.y, b.y);
+  fma_hi(acc, a.y, b.y);
+  fma_lo(acc, a.z, b.z);
+  fma_hi(acc, a.z, b.z);
+  fma_lo(acc, a.w, b.w);
+  fma_hi(acc, a.w, b.w);
+}
+
+__global__ void __launch_bounds__(kBatchThreads, 2)
+    screen_batch_kernel(const __grid_constant__ CUtensorMap map_h,
+                        const __grid_constant__ CUtensorMap map_w, float* __restrict__ z,
+                        const float* __restrict__ hss, const float* __restrict__ nw, float g,
+                        const int32_t* __restrict__ kin, int T, int E, int d, int k_max,
+                        int32_t* __restrict__ ids, float* __restrict__ alpha,
+                        uint32_t* __restrict__ err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* ring = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  BatchSmem& sm = *reinterpret_cast<BatchSmem*>(ring + kBatchStages * kBatchStageBytes);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t0 = blockIdx.x * kBatchT;
+  const int nt = min(kBatchT, T - t0);
+  const int kcap = k_max < E ? k_max : E;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kBatchStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], kBatchCompute / 32);
+    }
+    sm.abort = 0;
+    fence_mbar_init();
+  }
+  grid_dep_wait();
+  grid_dep_launch();
+  // ---- 1. screening: candidate masks ----
+  if (warp < 8) {
+    for (int i = 0; i < kBatchT / 8; ++i) {
+      const int tl = warp * (kBatchT / 8) + i;
+      const int t = t0 + tl;
+      if (tl >= nt) {
+        if (lane == 0) {
+          sm.mask[tl][0] = sm.mask[tl][1] = 0u;
+          sm.cnt[tl] = 0;
+          sm.kt[tl] = 0;
+        }
+        continue;
+      }
+      int kt = kin[t];
+      if (kt < 1 || kt > kcap) {
+        if (lane == 0) set_err(err, kErrKRange);
+        kt = kt < 1 ? 1 : kcap;
+      }
+      const float nh = sqrtf(hss[t] * (1.0f + 0x1p-10f)) * (1.0f + 0x1p-20f);
+      const float* zt = z + static_cast<int64_t>(t) * E;
+      float hi[2];
+      unsigned long long key[2];
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int e = lane + 32 * j;
+        hi[j] = -INFINITY;
+        key[j] = 0ull;
+        if (e < E) {
+          const float v = zt[e];
+          const float del = g * nh * nw[e] * (1.0f + 0x1p-16f) + fabsf(v) * 0x1p-22f;
+          hi[j] = v + del;
+          key[j] = score_key(v - del, e);
+        }
+      }
+      unsigned long long best = 0ull;
+      for (int j = 0; j < kt; ++j) {
+        best = key[0] > key[1] ? key[0] : key[1];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+          best = other > best ? other : best;
+        }
+        if (key[0] == best) key[0] = 0ull;
+        if (key[1] == best) key[1] = 0ull;
+      }
+      const float L = from_order_bits(static_cast<uint32_t>(best >> 32));
+      const uint32_t m0 = __ballot_sync(0xffffffffu, hi[0] >= L);
+      const uint32_t m1 = __ballot_sync(0xffffffffu, hi[1] >= L);
+      if (lane == 0) {
+        sm.mask[tl][0] = m0;
+        sm.mask[tl][1] = m1;
+        sm.cnt[tl] = __popc(m0) + __popc(m1);
+        sm.kt[tl] = kt;
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 0) {  // exclusive prefix of the candidate counts
+    int a = sm.cnt[lane], b = sm.cnt[lane + 32];
+    int ia = a, ib = b;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int va = __shfl_up_sync(0xffffffffu, ia, o);
+      const int vb = __shfl_up_sync(0xffffffffu, ib, o);
+      if (lane >= o) {
+        ia += va;
+        ib += vb;
+      }
+    }
+    const int tot_a = __shfl_sync(0xffffffffu, ia, 31);
+    sm.off[lane] = ia - a;
+    sm.off[lane + 32] = tot_a + ib - b;
+    if (lane == 31) sm.off[kBatchT] = tot_a + ib;
+  }
+  __syncthreads();
+  if (warp < 8) {  // the (token, expert) pairs in token order, experts ascending
+    for (int i = 0; i < kBatchT / 8; ++i) {
+      const int tl = warp * (kBatchT / 8) + i;
+      const uint32_t m0 = sm.mask[tl][0], m1 = sm.mask[tl][1];
+      const uint32_t below = (1u << lane) - 1u;
+      if ((m0 >> lane) & 1u)
+        sm.pair[sm.off[tl] + __popc(m0 & below)] = static_cast<uint16_t>((tl << 8) | lane);
+      if ((m1 >> lane) & 1u)
+        sm.pair[sm.off[tl] + __popc(m0) + __popc(m1 & below)] =
+            static_cast<uint16_t>((tl << 8) | (lane + 32));
+    }
+  }
+  __syncthreads();
+  const int npairs = sm.off[kBatchT];
+  const int passes = (npairs + kBatchSlots - 1) / kBatchSlots;
+  const int nch = d / 64;
+  // ---- 2. the chains ----
+  if (warp == 8) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0, issued = 0, issued_phase = 0;
+      bool ok = true;
+      for (int ps = 0; ps < passes && ok; ++ps) {
+        for (int c = 0; c < nch; ++c) {
+          if (!mbar_wait(&sm.empty[stage], phase ^ 1u, &sm.abort, kBatchWaitNs)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = smem_addr(&sm.full[stage]);
+          uint8_t* st = ring + stage * kBatchStageBytes;
+          mbar_arrive_tx(fb, kBatchStageBytes);
+          tma_tile_2d(smem_addr(st), &map_h, c * 64, t0, fb);
+          tma_tile_2d(smem_addr(st + kBatchTokBytes), &map_w, c * 64, 0, fb);
+          issued |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == kBatchStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        set_err(err, kErrTimeout);
+        sm.abort = 1;
+      }
+      if (sm.abort) {  // every issued copy lands before the CTA exits
+        for (int s = 0; s < kBatchStages; ++s)
+          if (issued & (1u << s))
+            mbar_wait(&sm.full[s], (issued_phase >> s) & 1u, nullptr, kBatchDrainNs);
+      }
+    }
+  } else {
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int ps = 0; ps < passes && ok; ++ps) {
+      const int p0 = ps * kBatchSlots + threadIdx.x, p1 = p0 + kBatchCompute;
+      const uint32_t q0 = p0 < npairs ? sm.pair[p0] : 0u, q1 = p1 < npairs ? sm.pair[p1] : 0u;
+      const int r0 = q0 >> 8, e0 = q0 & 255, r1 = q1 >> 8, e1 = q1 & 255;
+      float acc0 = 0.f, acc1 = 0.f;
+      for (int c = 0; c < nch; ++c) {
+        if (!__all_sync(0xffffffffu,
+                        mbar_wait(&sm.full[stage], phase, &sm.abort, kBatchWaitNs))) {
+          ok = false;
+          break;
+        }
+        const uint8_t* tok = ring + stage * kBatchStageBytes;
+        const uint8_t* ex = tok + kBatchTokBytes;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const uint4 a0 = swz_ld16(tok, r0, q), b0 = swz_ld16(ex, e0, q);
+          const uint4 a1 = swz_ld16(tok, r1, q), b1 = swz_ld16(ex, e1, q);
+          chain8(acc0, a0, b0);
+          chain8(acc1, a1, b1);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive_local(smem_addr(&sm.empty[stage]));
+        if (++stage == kBatchStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (ok) {
+        if (p0 < npairs) sm.zc[p0] = acc0;
+        if (p1 < npairs) sm.zc[p1] = acc1;
+      }
+    }
+    if (!ok && lane == 0) {
+      set_err(err, kErrTimeout);
+      sm.abort = 1;
+    }
+  }
+  __syncthreads();
+  if (sm.abort) return;
+  // ---- 3. selection over the candidates' exact scores ----
+  if (warp < 8) {
+    for (int i = 0; i < kBatchT / 8; ++i) {
+      const int tl = warp * (kBatchT / 8) + i;
+      if (tl >= nt) continue;
+      const int t = t0 + tl;
+      const int off = sm.off[tl], m = sm.cnt[tl], kt = sm.kt[tl];
+      float* zt = z + static_cast<int64_t>(t) * E;
+      unsigned long long ck[2];
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int idx = lane + 32 * j;
+        ck[j] = 0ull;
+        if (idx < m) {
+          const int e = sm.pair[off + idx] & 255;
+          const float v = sm.zc[off + idx];
+          zt[e] = v;
+          ck[j] = score_key(v, e);
+        }
+      }
+      for (int j = 0; j < kt; ++j) {
+        unsigned long long b = ck[0] > ck[1] ? ck[0] : ck[1];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const unsigned long long other = __shfl_xor_sync(0xffffffffu, b, o);
+          b = other > b ? other : b;
+        }
+        if (ck[0] == b) ck[0] = 0ull;
+        if (ck[1] == b) ck[1] = 0ull;
+        if (lane == 0) {
+          sm.sel_e[warp][j] = static_cast<int>(0xffffffffu - static_cast<uint32_t>(b & 0xffffffffull));
+          sm.sel_z[warp][j] = from_order_bits(static_cast<uint32_t>(b >> 32));
+        }
+      }
+      __syncwarp();
+      const float zmax = sm.sel_z[warp][0];
+      const float mine = lane < kt ? expf(sm.sel_z[warp][lane] - zmax) : 0.f;
+      float sel = mine;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) sel += __shfl_xor_sync(0xffffffffu, sel, o);
+      for (int j = lane; j < k_max; j += 32) {
+        const int64_t o = static_cast<int64_t>(t) * k_max + j;
+        if (j < kt) {
+          ids[o] = sm.sel_e[warp][j];
+          alpha[o] = mine / sel;
+        } else {
+          ids[o] = -1;
+          alpha[o] = 0.f;
+        }
+      }
+      __syncwarp();
+    }
+  }
+}
+
 template <int LY, int TM, int TN, int WT, int WE, int S, int KC = 32>
 cudaError_t launch_logits_mx(const __nv_bfloat16* h, const __nv_bfloat16* w, int T,
                              int d, int E, float* z, uint32_t* zw, int nz, cudaStream_t s) {
@@ -1263,6 +1571,25 @@ cudaError_t launch_router_screen_select(const __nv_bfloat16* h, const __nv_bfloa
   if (E <= 512) return RX_SCREEN(16);
   return RX_SCREEN(32);
 #undef RX_SCREEN
+}
+
+cudaError_t launch_router_screen_batch(const CUtensorMap* map_h, const CUtensorMap* map_w,
+                                       float* z, const float* hss, const float* nw,
+                                       const int32_t* k, int T, int E, int d, int k_max,
+                                       int32_t* ids, float* alpha, uint32_t* err,
+                                       cudaStream_t stream) {
+  if (T == 0) return cudaSuccess;
+  if (E > kBatchE || d % 64 != 0 || d < 64 || k_max > 32) return cudaErrorInvalidValue;
+  const double u = 1.0 / 16777216.0;
+  const double gamma = d * u / (1.0 - d * u);
+  // chain bound + tensor-core allowance + the score's own rounding (one K slice)
+  const float g = static_cast<float>((gamma + 1.0 / 4096.0 + 2 * u) * (1.0 + 1e-3));
+  const cudaError_t e = cudaFuncSetAttribute(
+      screen_batch_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kBatchSmemBytes);
+  if (e != cudaSuccess) return e;
+  const dim3 grid((T + kBatchT - 1) / kBatchT), block(kBatchThreads);
+  return launch_pdl(screen_batch_kernel, grid, block, kBatchSmemBytes, stream, *map_h, *map_w,
+                    z, hss, nw, g, k, T, E, d, k_max, ids, alpha, err);
 }
 
 cudaError_t launch_router_select_rule(const float* z, int T, int E, int k_hi, int k_lo,

@@ -180,12 +180,14 @@ def test_step_launch_counts_of_the_bench_layers():
     # LLaDA-MoE layer (count, scores, selection, count + scan, gather, two
     # GEMMs, combine), LLaDA2.0-mini layer (count, norms, score GEMM,
     # screened selection, count, scan, gather, four GEMMs, combine), 32 x 1024
-    # layer (count, scores, selection, count, scan, gather, two GEMMs, combine)
+    # layer (count, norms, score GEMM, batched recheck, count, scan, gather,
+    # two GEMMs, combine)
     from paper_2608_01784_gb300 import _binding as B
     from paper_2608_01784_gb300 import api
     assert api.step_launches("bf16", 1024, 2048, 64, 0) == 8
     assert api.step_launches("bf16", 8192, 2048, 256, 512) == 12
-    assert api.step_launches("bf16", 32768, 2048, 64, 0) == 9
+    assert api.step_launches("bf16", 32768, 2048, 64, 0) == 10   # batched screen
+    assert api.step_launches("bf16", 4096, 2048, 64, 0) == 8      # dense scores
     # exact scores: the screen's three kernels become scores + selection
     exact = B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_FLAG_EXACT_SCORES
     assert api.step_launches("bf16", 8192, 2048, 256, 512, flags=exact) == 11

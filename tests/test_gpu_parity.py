@@ -392,6 +392,83 @@ def test_screened_routing_router_rows_16_byte_aligned():
     np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
 
 
+# The batched screen for layers with at most 64 experts and many tokens
+# (bf16, renormalised weights, from 8192 tokens): tensor-core scores with
+# the token norms from the same GEMM, one exact chain per candidate pair in
+# a CTA of 64 tokens; ids, weights and selected scores bit for bit
+@pytest.mark.parametrize("T,E,d,kmax", [
+    (8192, 64, 2048, 12),    # whole token tiles
+    (9000, 64, 1024, 8),     # ragged last tile
+    (8256, 40, 512, 6),      # fewer experts than the 64-row expert box
+    (8192, 64, 256, 12),     # short rows (4 chunks)
+    (16384, 17, 2048, 4),    # odd expert count
+])
+def test_batch_screened_routing_bit_exact(T, E, d, kmax):
+    cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=5 * T + E + d)
+    k = np.random.default_rng(T + E).integers(1, min(kmax, E) + 1, T).astype(np.int32)
+    gl = G.GpuLayer(cfg, layer)
+    _, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE)
+    assert status == B.REFLEX_OK
+    z = oracle.router_logits(layer["hidden"], layer["w_router"])
+    ids, alpha = oracle.select(z, k, kmax)
+    assert np.array_equal(rec["ids"], ids)
+    valid = ids >= 0
+    np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
+    rows = np.repeat(np.arange(T), kmax).reshape(T, kmax)[valid]
+    assert np.array_equal(rec["scores"][rows, ids[valid]].view(np.uint32),
+                          z[rows, ids[valid]].view(np.uint32))
+    assert np.all(np.abs(rec["scores"].astype(np.float64) - z) <= _screen_bound(layer, d, 1))
+    # the weights are those of the dense path, bit for bit
+    _, rec_e, st_e = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE |
+                                B.REFLEX_FLAG_EXACT_SCORES)
+    assert st_e == B.REFLEX_OK
+    assert np.array_equal(rec["ids"], rec_e["ids"])
+    assert np.array_equal(rec["alpha"].view(np.uint32), rec_e["alpha"].view(np.uint32))
+
+
+@pytest.mark.parametrize("kind", ["ties", "all_candidates", "cancel", "wide"])
+def test_batch_screened_routing_hard_inputs(kind):
+    # ties: duplicated rows (the lower index wins), rows one bf16 step apart;
+    # all_candidates: every expert row equal for a third of the experts and
+    # tiny weights elsewhere, so many tokens keep more than 32 candidates and
+    # CTAs hold more pairs than one pass of the chain loop (rows streamed
+    # again); cancel / wide: the adversarial inputs of the 256-expert screen
+    T, E, d, kmax = 8192, 64, 1024, 8
+    cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=77)
+    hb, wb = layer["hidden"], layer["w_router"].copy()
+    if kind == "ties":
+        wb[5] = wb[3]
+        wb[9] = wb[3]
+        wb[12] = wb[11]
+        wb[12, 7] ^= np.uint16(1)
+    elif kind == "all_candidates":
+        wb[:] = W.to_bf16_bits(W.bf16_bits_to_f32(wb) * np.float32(1e-3))
+        wb[10:40] = wb[10]
+    elif kind == "cancel":
+        hb, wb = _cancelling_case(T, d, E, 78)
+    else:
+        hb, wb = _wide_exponent_case(T, d, E, 79)
+    layer = dict(layer, hidden=hb, w_router=wb)
+    k = np.random.default_rng(80).integers(1, kmax + 1, T).astype(np.int32)
+    gl = G.GpuLayer(cfg, layer)
+    _, rec, status = gl.forward(k, flags=B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_STAGE_ROUTE)
+    assert status == B.REFLEX_OK
+    z = oracle.router_logits(hb, wb)
+    ids, alpha = oracle.select(z, k, kmax)
+    assert np.array_equal(rec["ids"], ids)
+    valid = ids >= 0
+    np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
+    est = rec["scores"].view(np.uint32) != z.view(np.uint32)
+    if est.any():
+        hf = _bf16_floats(hb).astype(np.float64)
+        wf = _bf16_floats(wb).astype(np.float64)
+        ratio = np.abs(rec["scores"].astype(np.float64) - hf @ wf.T)[est] / \
+            (np.abs(hf) @ np.abs(wf).T)[est]
+        print(f"TC_ERROR_RATIO batch kind={kind} max={float(ratio.max()):.3e} "
+              f"estimates={int(est.sum())}")
+        assert float(ratio.max()) <= 2.0 ** -12
+
+
 @pytest.mark.parametrize("T,d,E,inter,shared,kmax,kmode", [
     (96, 256, 8, 128, 0, 4, "random"),     # one partial m-tile per expert
     (1000, 256, 4, 128, 0, 4, "max"),      # 8 m-tiles per expert, ragged tail
