@@ -201,6 +201,12 @@ __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
                "r"(bytes)
                : "memory");
 }
+// Orders this thread's earlier generic-proxy accesses of shared memory with
+// later async-proxy (TMA) accesses: a consumer that read a ring stage with
+// ordinary loads issues it before releasing the stage to the next TMA fill.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
 __device__ __forceinline__ void mbar_arrive_local(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }

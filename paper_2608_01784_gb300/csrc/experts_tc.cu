@@ -464,6 +464,7 @@ __global__ void __launch_bounds__(MODE == kModeScores ? kThreadsScores : kThread
               ss = fmaf(hi, hi, ss);
             }
           }
+          fence_proxy_async_smem();  // the reads above, before the next TMA fill
           __syncwarp();
           if (lane == 0) mbar_arrive1(smem_addr(&empty[stage]));
           if (++stage == kStages) {

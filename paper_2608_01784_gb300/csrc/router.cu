@@ -1152,26 +1152,29 @@ __global__ void __launch_bounds__(kScreenWarps * 32)
 // The screen of screen_select_kernel for many tokens and few experts, where
 // one warp per token leaves most lanes idle and streams expert rows from L2
 // one lane at a time.  A CTA owns 64 tokens:
-//   1. screening (8 warps, 8 tokens each): from the tensor-core estimates
-//      z~ and the row norms (the score GEMM's sums of squares, ||w_e|| from
-//      wnorm_kernel) the interval z~ -/+ del of every (token, expert), the
-//      k_t-th largest lower end L, and the candidates (upper end >= L) as a
-//      per-token bit mask; a prefix over the tokens lays the (token, expert)
-//      candidate pairs out in shared memory;
+//   1. screening (8 warps, 8 tokens each, four tokens' rounds interleaved):
+//      from the tensor-core estimates z~ and the row norms (the score GEMM's
+//      sums of squares, ||w_e|| from wnorm_kernel) the interval z~ -/+ del
+//      of every (token, expert), the k_t-th largest lower end L, and the
+//      candidates (upper end >= L) as a per-token bit mask; a prefix over
+//      the tokens lays the (token, expert) candidate pairs out in shared
+//      memory;
 //   2. chains: a producer warp streams 64-k chunks of the CTA's 64 token rows
 //      and of the 64 expert rows through a 4-stage TMA ring (128-byte
 //      swizzle); each compute thread advances the canonical fma chain of two
 //      candidate pairs over the chunk (more than 512 pairs: the rows are
 //      streamed again for the next 512);
-//   3. selection (a warp per token): TopK over the candidates' exact scores
-//      with the keys and tie rule of select_kernel, the weights with its
-//      arithmetic (the same bits), and the exact scores into z.
+//   3. selection (four tokens of a warp at a time): TopK over the
+//      candidates' exact scores with the keys and tie rule of select_kernel,
+//      the weights with its arithmetic (the same bits), and the exact scores
+//      into z.
 constexpr int kBatchT = 64;                   // tokens per CTA
 constexpr int kBatchE = 64;                   // expert rows per stage (E <= 64)
 constexpr int kBatchStages = 4;
 constexpr int kBatchCompute = 256;            // 8 compute warps
 constexpr int kBatchThreads = kBatchCompute + 32;  // + the producer warp
 constexpr int kBatchSlots = 2 * kBatchCompute;     // candidate pairs per pass
+constexpr int kBatchGroup = 4;                // tokens whose rounds interleave
 constexpr uint32_t kBatchTokBytes = kBatchT * 128;
 constexpr uint32_t kBatchStageBytes = kBatchTokBytes + kBatchE * 128;
 constexpr uint64_t kBatchWaitNs = 2000000000ull;
@@ -1183,8 +1186,8 @@ struct BatchSmem {
   int32_t cnt[kBatchT];
   int32_t kt[kBatchT];
   int32_t off[kBatchT + 1];
-  float sel_z[8][32];
-  int32_t sel_e[8][32];
+  float sel_z[8][kBatchGroup][32];
+  int32_t sel_e[8][kBatchGroup][32];
   volatile int abort;
   uint16_t pair[kBatchT * kBatchE];           // (token << 8) | expert
   float zc[kBatchT * kBatchE];                // exact scores of the pairs
@@ -1192,9 +1195,24 @@ struct BatchSmem {
 constexpr size_t kBatchSmemBytes =
     1024 + kBatchStages * kBatchStageBytes + sizeof(BatchSmem);
 
-// the 16-byte chunk q of row r of a 128-byte-swizzled 64-column box
-__device__ __forceinline__ uint4 swz_ld16(const uint8_t* box, int r, int q) {
-  return *reinterpret_cast<const uint4*>(box + r * 128 + ((q ^ (r & 7)) << 4));
+// 16 bytes of shared memory.  The "memory" clobber keeps every such read
+// between the stage's mbarrier wait and its release (both asm statements
+// with the same clobber): without it the compiler may move a read of a ring
+// stage above the wait that makes the TMA data visible.
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+// Row r of a 128-byte-swizzled box of 128-byte rows at a 1024-aligned
+// address: the 16-byte chunk q sits at r * 128 + ((q ^ (r & 7)) << 4), i.e.
+// at (base + r * 128 + ((r & 7) << 4)) ^ (q << 4) (bits 4-6 of the row base
+// hold r & 7); swz_row gives the part before the XOR.
+__device__ __forceinline__ uint32_t swz_row(int r) {
+  return static_cast<uint32_t>(r * 128 + ((r & 7) << 4));
 }
 __device__ __forceinline__ void chain8(float& acc, const uint4& a, const uint4& b) {
   fma_lo(acc, a.x, b.x);
@@ -1205,6 +1223,10 @@ __device__ __forceinline__ void chain8(float& acc, const uint4& a, const uint4& 
   fma_hi(acc, a.z, b.z);
   fma_lo(acc, a.w, b.w);
   fma_hi(acc, a.w, b.w);
+}
+__device__ __forceinline__ unsigned long long umax64(unsigned long long a,
+                                                     unsigned long long b) {
+  return a > b ? a : b;
 }
 
 __global__ void __launch_bounds__(kBatchThreads, 2)
@@ -1232,59 +1254,80 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
   }
   grid_dep_wait();
   grid_dep_launch();
-  // ---- 1. screening: candidate masks ----
+  // ---- 1. screening: candidate masks, four tokens' rounds interleaved ----
   if (warp < 8) {
-    for (int i = 0; i < kBatchT / 8; ++i) {
-      const int tl = warp * (kBatchT / 8) + i;
-      const int t = t0 + tl;
-      if (tl >= nt) {
+    const float nw0 = lane < E ? nw[lane] : 0.f;
+    const float nw1 = lane + 32 < E ? nw[lane + 32] : 0.f;
+    for (int g0 = 0; g0 < kBatchT / 8; g0 += kBatchGroup) {
+      float zv[kBatchGroup][2], hs[kBatchGroup];
+      int kt[kBatchGroup];
+#pragma unroll
+      for (int i = 0; i < kBatchGroup; ++i) {  // every load of the group first
+        const int tl = warp * (kBatchT / 8) + g0 + i;
+        const int t = t0 + tl;
+        const bool ok = tl < nt;
+        kt[i] = ok ? kin[t] : 1;
+        hs[i] = ok ? hss[t] : 0.f;
+        const float* zt = z + static_cast<int64_t>(ok ? t : 0) * E;
+        zv[i][0] = ok && lane < E ? zt[lane] : 0.f;
+        zv[i][1] = ok && lane + 32 < E ? zt[lane + 32] : 0.f;
+      }
+      unsigned long long key[kBatchGroup][2], best[kBatchGroup];
+      float hi[kBatchGroup][2];
+      int rounds = 0;
+#pragma unroll
+      for (int i = 0; i < kBatchGroup; ++i) {
+        if (kt[i] < 1 || kt[i] > kcap) {
+          const int tl = warp * (kBatchT / 8) + g0 + i;
+          if (lane == 0 && tl < nt) set_err(err, kErrKRange);
+          kt[i] = kt[i] < 1 ? 1 : kcap;
+        }
+        rounds = max(rounds, kt[i]);
+        const float nh = sqrtf(hs[i] * (1.0f + 0x1p-10f)) * (1.0f + 0x1p-20f);
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          const int e = lane + 32 * j;
+          hi[i][j] = -INFINITY;
+          key[i][j] = 0ull;
+          if (e < E) {
+            const float v = zv[i][j];
+            const float del = g * nh * (j ? nw1 : nw0) * (1.0f + 0x1p-16f) + fabsf(v) * 0x1p-22f;
+            hi[i][j] = v + del;
+            key[i][j] = score_key(v - del, e);
+          }
+        }
+        best[i] = 0ull;
+      }
+      for (int r = 0; r < rounds; ++r) {
+        unsigned long long b[kBatchGroup];
+#pragma unroll
+        for (int i = 0; i < kBatchGroup; ++i) b[i] = umax64(key[i][0], key[i][1]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+          for (int i = 0; i < kBatchGroup; ++i)
+            b[i] = umax64(b[i], __shfl_xor_sync(0xffffffffu, b[i], o));
+#pragma unroll
+        for (int i = 0; i < kBatchGroup; ++i) {
+          if (r < kt[i]) {
+            best[i] = b[i];
+            if (key[i][0] == b[i]) key[i][0] = 0ull;
+            if (key[i][1] == b[i]) key[i][1] = 0ull;
+          }
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < kBatchGroup; ++i) {
+        const int tl = warp * (kBatchT / 8) + g0 + i;
+        const float L = from_order_bits(static_cast<uint32_t>(best[i] >> 32));
+        const uint32_t m0 = __ballot_sync(0xffffffffu, tl < nt && hi[i][0] >= L);
+        const uint32_t m1 = __ballot_sync(0xffffffffu, tl < nt && hi[i][1] >= L);
         if (lane == 0) {
-          sm.mask[tl][0] = sm.mask[tl][1] = 0u;
-          sm.cnt[tl] = 0;
-          sm.kt[tl] = 0;
+          sm.mask[tl][0] = m0;
+          sm.mask[tl][1] = m1;
+          sm.cnt[tl] = __popc(m0) + __popc(m1);
+          sm.kt[tl] = tl < nt ? kt[i] : 0;
         }
-        continue;
-      }
-      int kt = kin[t];
-      if (kt < 1 || kt > kcap) {
-        if (lane == 0) set_err(err, kErrKRange);
-        kt = kt < 1 ? 1 : kcap;
-      }
-      const float nh = sqrtf(hss[t] * (1.0f + 0x1p-10f)) * (1.0f + 0x1p-20f);
-      const float* zt = z + static_cast<int64_t>(t) * E;
-      float hi[2];
-      unsigned long long key[2];
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int e = lane + 32 * j;
-        hi[j] = -INFINITY;
-        key[j] = 0ull;
-        if (e < E) {
-          const float v = zt[e];
-          const float del = g * nh * nw[e] * (1.0f + 0x1p-16f) + fabsf(v) * 0x1p-22f;
-          hi[j] = v + del;
-          key[j] = score_key(v - del, e);
-        }
-      }
-      unsigned long long best = 0ull;
-      for (int j = 0; j < kt; ++j) {
-        best = key[0] > key[1] ? key[0] : key[1];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
-          best = other > best ? other : best;
-        }
-        if (key[0] == best) key[0] = 0ull;
-        if (key[1] == best) key[1] = 0ull;
-      }
-      const float L = from_order_bits(static_cast<uint32_t>(best >> 32));
-      const uint32_t m0 = __ballot_sync(0xffffffffu, hi[0] >= L);
-      const uint32_t m1 = __ballot_sync(0xffffffffu, hi[1] >= L);
-      if (lane == 0) {
-        sm.mask[tl][0] = m0;
-        sm.mask[tl][1] = m1;
-        sm.cnt[tl] = __popc(m0) + __popc(m1);
-        sm.kt[tl] = kt;
       }
     }
   }
@@ -1359,13 +1402,16 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
       }
     }
   } else {
+    const uint32_t ring_s = smem_addr(ring);
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
     for (int ps = 0; ps < passes && ok; ++ps) {
       const int p0 = ps * kBatchSlots + threadIdx.x, p1 = p0 + kBatchCompute;
       const uint32_t q0 = p0 < npairs ? sm.pair[p0] : 0u, q1 = p1 < npairs ? sm.pair[p1] : 0u;
-      const int r0 = q0 >> 8, e0 = q0 & 255, r1 = q1 >> 8, e1 = q1 & 255;
+      // row bases inside a stage (the swizzle is an XOR on bits 4-6)
+      const uint32_t ta0 = swz_row(q0 >> 8), ea0 = kBatchTokBytes + swz_row(q0 & 255);
+      const uint32_t ta1 = swz_row(q1 >> 8), ea1 = kBatchTokBytes + swz_row(q1 & 255);
       float acc0 = 0.f, acc1 = 0.f;
       for (int c = 0; c < nch; ++c) {
         if (!__all_sync(0xffffffffu,
@@ -1373,15 +1419,29 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
           ok = false;
           break;
         }
-        const uint8_t* tok = ring + stage * kBatchStageBytes;
-        const uint8_t* ex = tok + kBatchTokBytes;
+        const uint32_t sb = ring_s + stage * kBatchStageBytes;
+        const uint32_t h0 = sb + ta0, w0 = sb + ea0, h1 = sb + ta1, w1 = sb + ea1;
+        uint4 a0 = lds128(h0), b0 = lds128(w0), a1 = lds128(h1), b1 = lds128(w1);
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
-          const uint4 a0 = swz_ld16(tok, r0, q), b0 = swz_ld16(ex, e0, q);
-          const uint4 a1 = swz_ld16(tok, r1, q), b1 = swz_ld16(ex, e1, q);
+          uint4 na0, nb0, na1, nb1;
+          if (q + 1 < 8) {
+            const uint32_t x = static_cast<uint32_t>((q + 1) << 4);
+            na0 = lds128(h0 ^ x);
+            nb0 = lds128(w0 ^ x);
+            na1 = lds128(h1 ^ x);
+            nb1 = lds128(w1 ^ x);
+          }
           chain8(acc0, a0, b0);
           chain8(acc1, a1, b1);
+          if (q + 1 < 8) {
+            a0 = na0;
+            b0 = nb0;
+            a1 = na1;
+            b1 = nb1;
+          }
         }
+        fence_proxy_async_smem();  // the reads above, before the next TMA fill
         __syncwarp();
         if (lane == 0) mbar_arrive_local(smem_addr(&sm.empty[stage]));
         if (++stage == kBatchStages) {
@@ -1403,52 +1463,77 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
   if (sm.abort) return;
   // ---- 3. selection over the candidates' exact scores ----
   if (warp < 8) {
-    for (int i = 0; i < kBatchT / 8; ++i) {
-      const int tl = warp * (kBatchT / 8) + i;
-      if (tl >= nt) continue;
-      const int t = t0 + tl;
-      const int off = sm.off[tl], m = sm.cnt[tl], kt = sm.kt[tl];
-      float* zt = z + static_cast<int64_t>(t) * E;
-      unsigned long long ck[2];
+    for (int g0 = 0; g0 < kBatchT / 8; g0 += kBatchGroup) {
+      unsigned long long ck[kBatchGroup][2];
+      int kt[kBatchGroup];
+      int rounds = 0;
 #pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int idx = lane + 32 * j;
-        ck[j] = 0ull;
-        if (idx < m) {
-          const int e = sm.pair[off + idx] & 255;
-          const float v = sm.zc[off + idx];
-          zt[e] = v;
-          ck[j] = score_key(v, e);
+      for (int i = 0; i < kBatchGroup; ++i) {
+        const int tl = warp * (kBatchT / 8) + g0 + i;
+        const int off = sm.off[tl], m = sm.cnt[tl];
+        kt[i] = sm.kt[tl];  // 0 past the batch
+        rounds = max(rounds, kt[i]);
+        float* zt = z + static_cast<int64_t>(t0 + tl) * E;
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          const int idx = lane + 32 * j;
+          ck[i][j] = 0ull;
+          if (idx < m) {
+            const int e = sm.pair[off + idx] & 255;
+            const float v = sm.zc[off + idx];
+            zt[e] = v;
+            ck[i][j] = score_key(v, e);
+          }
         }
       }
-      for (int j = 0; j < kt; ++j) {
-        unsigned long long b = ck[0] > ck[1] ? ck[0] : ck[1];
+      for (int r = 0; r < rounds; ++r) {
+        unsigned long long b[kBatchGroup];
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          const unsigned long long other = __shfl_xor_sync(0xffffffffu, b, o);
-          b = other > b ? other : b;
-        }
-        if (ck[0] == b) ck[0] = 0ull;
-        if (ck[1] == b) ck[1] = 0ull;
-        if (lane == 0) {
-          sm.sel_e[warp][j] = static_cast<int>(0xffffffffu - static_cast<uint32_t>(b & 0xffffffffull));
-          sm.sel_z[warp][j] = from_order_bits(static_cast<uint32_t>(b >> 32));
+        for (int i = 0; i < kBatchGroup; ++i) b[i] = umax64(ck[i][0], ck[i][1]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+          for (int i = 0; i < kBatchGroup; ++i)
+            b[i] = umax64(b[i], __shfl_xor_sync(0xffffffffu, b[i], o));
+#pragma unroll
+        for (int i = 0; i < kBatchGroup; ++i) {
+          if (r < kt[i]) {
+            if (ck[i][0] == b[i]) ck[i][0] = 0ull;
+            if (ck[i][1] == b[i]) ck[i][1] = 0ull;
+            if (lane == 0) {
+              sm.sel_e[warp][i][r] =
+                  static_cast<int>(0xffffffffu - static_cast<uint32_t>(b[i] & 0xffffffffull));
+              sm.sel_z[warp][i][r] = from_order_bits(static_cast<uint32_t>(b[i] >> 32));
+            }
+          }
         }
       }
       __syncwarp();
-      const float zmax = sm.sel_z[warp][0];
-      const float mine = lane < kt ? expf(sm.sel_z[warp][lane] - zmax) : 0.f;
-      float sel = mine;
+      float mine[kBatchGroup], sel[kBatchGroup];
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) sel += __shfl_xor_sync(0xffffffffu, sel, o);
-      for (int j = lane; j < k_max; j += 32) {
-        const int64_t o = static_cast<int64_t>(t) * k_max + j;
-        if (j < kt) {
-          ids[o] = sm.sel_e[warp][j];
-          alpha[o] = mine / sel;
-        } else {
-          ids[o] = -1;
-          alpha[o] = 0.f;
+      for (int i = 0; i < kBatchGroup; ++i) {
+        const float zmax = sm.sel_z[warp][i][0];
+        mine[i] = lane < kt[i] ? expf(sm.sel_z[warp][i][lane] - zmax) : 0.f;
+        sel[i] = mine[i];
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+        for (int i = 0; i < kBatchGroup; ++i) sel[i] += __shfl_xor_sync(0xffffffffu, sel[i], o);
+#pragma unroll
+      for (int i = 0; i < kBatchGroup; ++i) {
+        const int tl = warp * (kBatchT / 8) + g0 + i;
+        if (tl >= nt) continue;
+        const int64_t t = t0 + tl;
+        for (int j = lane; j < k_max; j += 32) {
+          const int64_t o = t * k_max + j;
+          if (j < kt[i]) {
+            ids[o] = sm.sel_e[warp][i][j];
+            alpha[o] = mine[i] / sel[i];
+          } else {
+            ids[o] = -1;
+            alpha[o] = 0.f;
+          }
         }
       }
       __syncwarp();
