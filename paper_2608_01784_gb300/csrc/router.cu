@@ -1162,10 +1162,11 @@ __global__ void __launch_bounds__(kScreenWarps * 32)
 //   2. chains: a producer warp streams 64-k chunks of the CTA's 64 token rows
 //      and of the 64 expert rows through a 4-stage TMA ring (128-byte
 //      swizzle); each compute thread advances the canonical fma chain of two
-//      candidate pairs over the chunk (more than 512 pairs: the rows are
-//      streamed again for the next 512);
-//   3. selection (four tokens of a warp at a time): TopK over the
-//      candidates' exact scores with the keys and tie rule of select_kernel,
+//      candidate pairs over the chunk, the pairs laid out so that a quarter
+//      warp's expert rows fall in distinct bank groups (more than 512 pairs:
+//      the rows are streamed again for the next 512);
+//   3. selection (a warp per token): TopK over the candidates' exact
+//      scores by rank counting, with the keys and tie rule of select_kernel,
 //      the weights with its arithmetic (the same bits), and the exact scores
 //      into z.
 constexpr int kBatchT = 64;                   // tokens per CTA
@@ -1190,6 +1191,7 @@ struct BatchSmem {
   int32_t sel_e[8][kBatchGroup][32];
   volatile int abort;
   uint16_t pair[kBatchT * kBatchE];           // (token << 8) | expert
+  uint16_t slot[kBatchT * kBatchE];           // chain slot -> pair (0xffff: none)
   float zc[kBatchT * kBatchE];                // exact scores of the pairs
 };
 constexpr size_t kBatchSmemBytes =
@@ -1364,7 +1366,30 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
   }
   __syncthreads();
   const int npairs = sm.off[kBatchT];
-  const int passes = (npairs + kBatchSlots - 1) / kBatchSlots;
+  // Chain slots: each run of 32 pairs is reordered so that the 8 lanes of a
+  // quarter warp read expert rows of distinct swizzle classes (e & 7): a
+  // 16-byte shared load is served a quarter warp per wavefront, and rows of
+  // one class share a bank group.  The pairs are sorted by class within the
+  // run and dealt to the quarters in turn (sorted position i -> lane
+  // 8 (i % 4) + i / 4).
+  if (warp < 8) {
+    for (int base = warp * 32; base < npairs; base += 8 * 32) {
+      const int idx = base + lane;
+      const bool valid = idx < npairs;
+      const int cls = valid ? (sm.pair[idx] & 7) : 8;
+      int pos = 0;
+#pragma unroll
+      for (int c = 0; c <= 8; ++c) {
+        const uint32_t mc = __ballot_sync(0xffffffffu, cls == c);
+        if (c < cls) pos += __popc(mc);
+        if (c == cls) pos += __popc(mc & ((1u << lane) - 1u));
+      }
+      sm.slot[base + 8 * (pos & 3) + (pos >> 2)] = valid ? static_cast<uint16_t>(idx) : 0xffff;
+    }
+  }
+  __syncthreads();
+  const int nslots = (npairs + 31) & ~31;
+  const int passes = (nslots + kBatchSlots - 1) / kBatchSlots;
   const int nch = d / 64;
   // ---- 2. the chains ----
   if (warp == 8) {
@@ -1407,11 +1432,16 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
     uint32_t phase = 0;
     bool ok = true;
     for (int ps = 0; ps < passes && ok; ++ps) {
-      const int p0 = ps * kBatchSlots + threadIdx.x, p1 = p0 + kBatchCompute;
-      const uint32_t q0 = p0 < npairs ? sm.pair[p0] : 0u, q1 = p1 < npairs ? sm.pair[p1] : 0u;
+      const int s0 = ps * kBatchSlots + threadIdx.x, s1 = s0 + kBatchCompute;
+      const int p0 = s0 < nslots ? sm.slot[s0] : 0xffff;
+      const int p1 = s1 < nslots ? sm.slot[s1] : 0xffff;
+      const uint32_t q0 = p0 != 0xffff ? sm.pair[p0] : 0u;
+      const uint32_t q1 = p1 != 0xffff ? sm.pair[p1] : 0u;
       // row bases inside a stage (the swizzle is an XOR on bits 4-6)
       const uint32_t ta0 = swz_row(q0 >> 8), ea0 = kBatchTokBytes + swz_row(q0 & 255);
       const uint32_t ta1 = swz_row(q1 >> 8), ea1 = kBatchTokBytes + swz_row(q1 & 255);
+      // the second slot only where a lane of the warp has a pair for it
+      const bool two = __any_sync(0xffffffffu, p1 != 0xffff);
       float acc0 = 0.f, acc1 = 0.f;
       for (int c = 0; c < nch; ++c) {
         if (!__all_sync(0xffffffffu,
@@ -1421,24 +1451,42 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
         }
         const uint32_t sb = ring_s + stage * kBatchStageBytes;
         const uint32_t h0 = sb + ta0, w0 = sb + ea0, h1 = sb + ta1, w1 = sb + ea1;
-        uint4 a0 = lds128(h0), b0 = lds128(w0), a1 = lds128(h1), b1 = lds128(w1);
+        if (two) {
+          uint4 a0 = lds128(h0), b0 = lds128(w0), a1 = lds128(h1), b1 = lds128(w1);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          uint4 na0, nb0, na1, nb1;
-          if (q + 1 < 8) {
-            const uint32_t x = static_cast<uint32_t>((q + 1) << 4);
-            na0 = lds128(h0 ^ x);
-            nb0 = lds128(w0 ^ x);
-            na1 = lds128(h1 ^ x);
-            nb1 = lds128(w1 ^ x);
+          for (int q = 0; q < 8; ++q) {
+            uint4 na0, nb0, na1, nb1;
+            if (q + 1 < 8) {
+              const uint32_t x = static_cast<uint32_t>((q + 1) << 4);
+              na0 = lds128(h0 ^ x);
+              nb0 = lds128(w0 ^ x);
+              na1 = lds128(h1 ^ x);
+              nb1 = lds128(w1 ^ x);
+            }
+            chain8(acc0, a0, b0);
+            chain8(acc1, a1, b1);
+            if (q + 1 < 8) {
+              a0 = na0;
+              b0 = nb0;
+              a1 = na1;
+              b1 = nb1;
+            }
           }
-          chain8(acc0, a0, b0);
-          chain8(acc1, a1, b1);
-          if (q + 1 < 8) {
-            a0 = na0;
-            b0 = nb0;
-            a1 = na1;
-            b1 = nb1;
+        } else {
+          uint4 a0 = lds128(h0), b0 = lds128(w0);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            uint4 na0, nb0;
+            if (q + 1 < 8) {
+              const uint32_t x = static_cast<uint32_t>((q + 1) << 4);
+              na0 = lds128(h0 ^ x);
+              nb0 = lds128(w0 ^ x);
+            }
+            chain8(acc0, a0, b0);
+            if (q + 1 < 8) {
+              a0 = na0;
+              b0 = nb0;
+            }
           }
         }
         fence_proxy_async_smem();  // the reads above, before the next TMA fill
@@ -1450,8 +1498,8 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
         }
       }
       if (ok) {
-        if (p0 < npairs) sm.zc[p0] = acc0;
-        if (p1 < npairs) sm.zc[p1] = acc1;
+        if (p0 != 0xffff) sm.zc[p0] = acc0;
+        if (p1 != 0xffff) sm.zc[p1] = acc1;
       }
     }
     if (!ok && lane == 0) {
@@ -1462,78 +1510,61 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
   __syncthreads();
   if (sm.abort) return;
   // ---- 3. selection over the candidates' exact scores ----
+  // A warp per token: lane l takes candidates l and l + 32, keys as in
+  // select_kernel (score, then the lower expert index); a candidate's rank is
+  // the number of the token's candidates with a larger key, and the k_t
+  // candidates of rank < k_t go to slot rank (the TopK in rank order).
   if (warp < 8) {
-    for (int g0 = 0; g0 < kBatchT / 8; g0 += kBatchGroup) {
-      unsigned long long ck[kBatchGroup][2];
-      int kt[kBatchGroup];
-      int rounds = 0;
+    for (int i = 0; i < kBatchT / 8; ++i) {
+      const int tl = warp * (kBatchT / 8) + i;
+      if (tl >= nt) continue;
+      const int t = t0 + tl;
+      const int off = sm.off[tl], m = sm.cnt[tl], kt = sm.kt[tl];
+      float* zt = z + static_cast<int64_t>(t) * E;
+      unsigned long long key[2];
+      int ex[2];
 #pragma unroll
-      for (int i = 0; i < kBatchGroup; ++i) {
-        const int tl = warp * (kBatchT / 8) + g0 + i;
-        const int off = sm.off[tl], m = sm.cnt[tl];
-        kt[i] = sm.kt[tl];  // 0 past the batch
-        rounds = max(rounds, kt[i]);
-        float* zt = z + static_cast<int64_t>(t0 + tl) * E;
-#pragma unroll
-        for (int j = 0; j < 2; ++j) {
-          const int idx = lane + 32 * j;
-          ck[i][j] = 0ull;
-          if (idx < m) {
-            const int e = sm.pair[off + idx] & 255;
-            const float v = sm.zc[off + idx];
-            zt[e] = v;
-            ck[i][j] = score_key(v, e);
-          }
+      for (int j = 0; j < 2; ++j) {
+        const int idx = lane + 32 * j;
+        key[j] = 0ull;
+        ex[j] = 0;
+        if (idx < m) {
+          ex[j] = sm.pair[off + idx] & 255;
+          const float v = sm.zc[off + idx];
+          zt[ex[j]] = v;
+          key[j] = score_key(v, ex[j]);
         }
       }
-      for (int r = 0; r < rounds; ++r) {
-        unsigned long long b[kBatchGroup];
+      // every candidate's key in shared memory (the token's zc slots hold
+      // the scores; the keys are rebuilt from them), then the ranks
+      int rank[2] = {0, 0};
+      for (int o = 0; o < m; ++o) {
+        const unsigned long long ko =
+            score_key(sm.zc[off + o], sm.pair[off + o] & 255);  // broadcast reads
+        rank[0] += ko > key[0];
+        rank[1] += ko > key[1];
+      }
 #pragma unroll
-        for (int i = 0; i < kBatchGroup; ++i) b[i] = umax64(ck[i][0], ck[i][1]);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-          for (int i = 0; i < kBatchGroup; ++i)
-            b[i] = umax64(b[i], __shfl_xor_sync(0xffffffffu, b[i], o));
-#pragma unroll
-        for (int i = 0; i < kBatchGroup; ++i) {
-          if (r < kt[i]) {
-            if (ck[i][0] == b[i]) ck[i][0] = 0ull;
-            if (ck[i][1] == b[i]) ck[i][1] = 0ull;
-            if (lane == 0) {
-              sm.sel_e[warp][i][r] =
-                  static_cast<int>(0xffffffffu - static_cast<uint32_t>(b[i] & 0xffffffffull));
-              sm.sel_z[warp][i][r] = from_order_bits(static_cast<uint32_t>(b[i] >> 32));
-            }
-          }
+      for (int j = 0; j < 2; ++j) {
+        if (lane + 32 * j < m && rank[j] < kt) {
+          sm.sel_e[warp][0][rank[j]] = ex[j];
+          sm.sel_z[warp][0][rank[j]] = from_order_bits(static_cast<uint32_t>(key[j] >> 32));
         }
       }
       __syncwarp();
-      float mine[kBatchGroup], sel[kBatchGroup];
+      const float zmax = sm.sel_z[warp][0][0];
+      const float mine = lane < kt ? expf(sm.sel_z[warp][0][lane] - zmax) : 0.f;
+      float sel = mine;
 #pragma unroll
-      for (int i = 0; i < kBatchGroup; ++i) {
-        const float zmax = sm.sel_z[warp][i][0];
-        mine[i] = lane < kt[i] ? expf(sm.sel_z[warp][i][lane] - zmax) : 0.f;
-        sel[i] = mine[i];
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-        for (int i = 0; i < kBatchGroup; ++i) sel[i] += __shfl_xor_sync(0xffffffffu, sel[i], o);
-#pragma unroll
-      for (int i = 0; i < kBatchGroup; ++i) {
-        const int tl = warp * (kBatchT / 8) + g0 + i;
-        if (tl >= nt) continue;
-        const int64_t t = t0 + tl;
-        for (int j = lane; j < k_max; j += 32) {
-          const int64_t o = t * k_max + j;
-          if (j < kt[i]) {
-            ids[o] = sm.sel_e[warp][i][j];
-            alpha[o] = mine[i] / sel[i];
-          } else {
-            ids[o] = -1;
-            alpha[o] = 0.f;
-          }
+      for (int o = 16; o > 0; o >>= 1) sel += __shfl_xor_sync(0xffffffffu, sel, o);
+      for (int j = lane; j < k_max; j += 32) {
+        const int64_t o = static_cast<int64_t>(t) * k_max + j;
+        if (j < kt) {
+          ids[o] = sm.sel_e[warp][0][j];
+          alpha[o] = mine / sel;
+        } else {
+          ids[o] = -1;
+          alpha[o] = 0.f;
         }
       }
       __syncwarp();
