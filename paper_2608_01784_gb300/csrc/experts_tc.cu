@@ -718,10 +718,12 @@ __device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols
 
 struct Cfg2 {
   static constexpr int BN = 256;                 // output tile width of the pair
-  static constexpr int kABytes = BM * BK * 2;    // 16 KB: this CTA's 128 rows
-  static constexpr int kBBytes = (BN / 2) * BK * 2;  // 16 KB: this CTA's half
+  static constexpr int KS = 2;                   // 64-k blocks per stage
+  static constexpr int kSubBytes = BM * BK * 2;  // 16 KB: one 128-row x 64-k box
+  static constexpr int kABytes = KS * kSubBytes; // this CTA's 128 rows
+  static constexpr int kBBytes = KS * kSubBytes; // this CTA's half of the weight tile
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStages = kRingBytes / kStageBytes;  // 6
+  static constexpr int kStages = kRingBytes / kStageBytes;  // 3
   static constexpr int kTmemCols = 2 * BN;       // two accumulators
   static constexpr int kStagingBytes = 32 * 128; // per epilogue warp: 32 rows x 128 B
   static constexpr int kSmemBytes =
@@ -808,7 +810,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
   grid_dep_launch();
   // tiles are 256 rows (both CTAs) x 256 columns; mt_prefix counts 256-row tiles
   const int ntiles = total_tiles(p);
-  const int nk = p.K / BK;
+  const int nk = p.K / (BK * C::KS);  // stages per tile
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer (each CTA: its A rows, its B half) -------
@@ -833,15 +835,20 @@ __global__ void __launch_bounds__(kThreads2, 1)
           mbar_expect_tx(smem_addr(&full[stage]), C::kStageBytes);
         else
           mbar_expect_tx_cluster(fb, C::kStageBytes);
-        const int k0 = kb * BK;
-        tma_load_2d_pair(smem_addr(sa + stage * C::kABytes), &map_a, k0,
-                         tl.row0 + static_cast<int>(rank) * BM, fb);
         int brow;
         if (MODE == kModeSwiGLU)
           brow = tl.e * p.b_rows_per_group + (rank ? p.b_up_offset : 0) + tl.n * (BN / 2);
         else
           brow = tl.e * p.b_rows_per_group + tl.n * BN + static_cast<int>(rank) * (BN / 2);
-        tma_load_2d_pair(smem_addr(sb + stage * C::kBBytes), &map_b, k0, brow, fb);
+        // consecutive k blocks of the same rows back to back
+#pragma unroll
+        for (int u = 0; u < C::KS; ++u) {
+          const int k0 = (kb * C::KS + u) * BK;
+          tma_load_2d_pair(smem_addr(sa + stage * C::kABytes + u * C::kSubBytes), &map_a, k0,
+                           tl.row0 + static_cast<int>(rank) * BM, fb);
+          tma_load_2d_pair(smem_addr(sb + stage * C::kBBytes + u * C::kSubBytes), &map_b, k0,
+                           brow, fb);
+        }
         issued_mask |= 1u << stage;
         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
         if (++stage == kStages) {
@@ -886,9 +893,12 @@ __global__ void __launch_bounds__(kThreads2, 1)
         const uint32_t a0 = smem_addr(sa + stage * C::kABytes);
         const uint32_t b0 = smem_addr(sb + stage * C::kBBytes);
 #pragma unroll
-        for (int k = 0; k < BK / UMMA_K; ++k)
-          mma_bf16_pair(d_tmem, desc_sw128(a0 + k * UMMA_K * 2), desc_sw128(b0 + k * UMMA_K * 2),
-                        idesc, (kb > 0 || k > 0) ? 1u : 0u);
+        for (int u = 0; u < C::KS; ++u)
+#pragma unroll
+          for (int k = 0; k < BK / UMMA_K; ++k)
+            mma_bf16_pair(d_tmem, desc_sw128(a0 + u * C::kSubBytes + k * UMMA_K * 2),
+                          desc_sw128(b0 + u * C::kSubBytes + k * UMMA_K * 2), idesc,
+                          (kb > 0 || u > 0 || k > 0) ? 1u : 0u);
         issued_any = true;
         mma_commit_pair(smem_addr(&empty[stage]));
         if (++stage == kStages) {
@@ -1025,6 +1035,7 @@ cudaError_t launch_pair_impl(const TcGemmArgs& a, cudaStream_t stream) {
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        C::kSmemBytes);
   if (e != cudaSuccess) return e;
+  if (a.K % (BK * C::KS) != 0) return cudaErrorInvalidValue;  // whole stages
   KParams p;
   p.K = a.K;
   p.n_tiles = MODE == kModeSwiGLU ? a.n_total / (C::BN / 2) : a.n_total / C::BN;
