@@ -1,0 +1,59 @@
+"""Host logic of bench.py that needs no GPU: the two arms report the same
+config, the DRAM-traffic figure is dropped once the kernel source it was
+captured on has changed, and the count-rule ablations carry the paper's
+thresholds."""
+import importlib
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def bench():
+    if ROOT not in sys.path:
+        sys.path.insert(0, ROOT)
+    return importlib.import_module("bench")
+
+
+def test_both_arms_share_the_config(bench):
+    from paper_2608_01784_gb300 import workloads as W
+    # the stack: the GPU arm adds only its timing note to the shared dict
+    c = bench.stack_config(1)
+    assert c["workload"] == "llada_moe_stack16" and c["layers"] == 16
+    assert c["tokens_per_step"] == 32 * 1024
+    # single layers: one dict for both arms
+    for name in ("llada_moe", "llada2_mini", "llada_moe_b32", "tiny_fp32"):
+        lc = bench.layer_config(W.CONFIGS[name], 2)
+        assert lc["workload"] == name and lc["tokens_per_step"] == W.CONFIGS[name].T
+        assert lc["parallelism"] == "replicas2"
+
+
+def test_traffic_follows_the_kernel_source(bench, monkeypatch):
+    sha = bench.kernel_source_sha16()
+    assert len(sha) == 16
+    monkeypatch.setitem(bench.NCU_TRAFFIC, "x", (123, sha))
+    assert bench.ncu_traffic("x") == 123
+    monkeypatch.setitem(bench.NCU_TRAFFIC, "x", (123, "0" * 16))
+    assert bench.ncu_traffic("x") is None          # captured on another source
+    monkeypatch.setitem(bench.NCU_TRAFFIC, "x", (None, sha))
+    assert bench.ncu_traffic("x") is None
+    assert bench.ncu_traffic("no such workload") is None
+
+
+def test_rule_ablations_use_the_paper_thresholds(bench):
+    # App. B: Top-p 0.15 / 0.20 (LLaDA-MoE), 0.25 / 0.325 (LLaDA2.0-mini);
+    # Expert-Threshold 0.0215 / 0.0190 and 0.0270 / 0.0220; counts in [1, 12]
+    got = {n: o for n, o in bench.rule_ablations("llada_moe")}
+    assert got["top_p_low"]["rule_threshold"] == 0.15
+    assert got["top_p_high"]["rule_threshold"] == 0.20
+    assert got["expert_threshold_low"]["rule_threshold"] == 0.0215
+    assert got["expert_threshold_high"]["rule_threshold"] == 0.0190
+    got = {n: o for n, o in bench.rule_ablations("llada2_mini")}
+    assert got["top_p_high"]["rule_threshold"] == 0.325
+    assert got["expert_threshold_low"]["rule_threshold"] == 0.0270
+    for o in got.values():
+        assert (o["k_min"], o["k_max"]) == (1, 12)
+    assert bench.rule_ablations("tiny_fp32") == []
