@@ -57,7 +57,7 @@ METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
 NCU_TRAFFIC = {
     "llada_moe": (561284352, "7507f281c153b35d"),
     "llada2_mini": (1407363048, None),
-    "llada_moe_stack16": (1655431424, "e46c7ba9e7a711fe"),
+    "llada_moe_stack16": (1634441472, "8628c28aa125c661"),
 }
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2608_01784_gb300", "csrc", "experts_tc.cu")
 
