@@ -482,6 +482,9 @@ def test_batch_screened_routing_hard_inputs(kind):
     (2048, 512, 8, 256, 0, 4, "max"),      # CTA-pair GEMMs, several n-tiles
     (4096, 256, 512, 64, 0, 8, "random"),  # block masks past one CTA: 32-token count + scan
     (5000, 256, 16, 128, 0, 4, "random"),  # 256-token dispatch blocks, ragged last block
+    (1030, 256, 4, 128, 0, 1, "one"),      # CTA-pair tiles, ~257 rows per group: the last
+                                           # tile holds a row or two (peer CTA's half empty)
+    (4099, 256, 4, 128, 0, 4, "max"),      # CTA-pair tiles, T % 4 != 0, every token at k_max
 ])
 @pytest.mark.parametrize("simt", [False, True])
 def test_forward_bf16_small(T, d, E, inter, shared, kmax, kmode, simt):
