@@ -571,45 +571,73 @@ def oracle_stack_rate(cfg, stack, state, target_s, seed, threads=None):
 
 
 def run_stack_reference(args, rank, world):
-    """The oracle as it stands on the host cores, on the stack workload: each
-    step is the whole forward (counts once, 16 layers with the residual) on a
-    seeded token sample of the 32 x 1024 batch."""
+    """The oracle as it stands on the host cores, on the stack workload.  One
+    token through the 16 layers costs about 0.5 core-seconds in the oracle,
+    so a step samples (token, layer) units instead of whole tokens: an
+    untimed oracle pass over a seeded pool of tokens records every layer's
+    input, and each step computes the counts of the whole batch (Eq. 5 /
+    Eq. 9 + clip) and then takes one seeded layer through n seeded pooled
+    tokens (scores, TopK / alpha, pair order, Eq. 2, residual) on their
+    inputs at that layer, in one call so that the host threads share it.
+    Every layer has the same shapes, so n units are n / 16 whole forwards; n
+    is sized so that the W + K steps take about two minutes."""
     import torch  # noqa: F401  (keeps the launch environment identical)
     if rank != 0:
         return
     import oracle
     oracle.build()
     cfg = W.CONFIGS[STACK_LAYER_CFG]
-    stack = W.make_stack(cfg, args.seed, STACK_LAYERS)
+    L = STACK_LAYERS
+    stack = W.make_stack(cfg, args.seed, L)
     state = W.make_state(cfg, args.seed)
     T = cfg.T
     rng = np.random.default_rng(args.seed)
-    per_step_s = max(0.5, min(5.0, 150.0 / max(1, args.steps + args.warmup)))
-    n = min(T, 2 * oracle.num_threads())
-    t0 = time.perf_counter()
-    oracle_stack(cfg, stack, state, np.arange(n, dtype=np.int32))
-    dt = time.perf_counter() - t0
-    n = int(min(T, max(1, n * per_step_s / max(dt, 1e-6))))
+    threads = oracle.num_threads()
+    pool = np.sort(rng.choice(T, min(T, max(64, 16 * threads)), replace=False)).astype(np.int32)
+    P = pool.size
 
-    def one():
-        oracle_stack(cfg, stack, state,
-                     np.sort(rng.choice(T, n, replace=False)).astype(np.int32))
+    def counts():
+        return oracle.allocate(state["conf1"], state["conf2"], state["hist_len"],
+                               state["masked"], state["block_id"], state["seq_offsets"],
+                               state["active_block"], **cfg.alloc_params())
+    k_pool = counts()[pool]
+    trace = oracle.moe_stack(stack["hidden"][pool], stack["layers"], k_pool, cfg.k_max)
+    h_in = [trace[l]["h_in"] for l in range(L)]
+    del trace
+
+    def one(n):
+        k_all = counts()
+        l = int(rng.integers(L))
+        ps = np.sort(rng.choice(P, n, replace=False))
+        w = stack["layers"][l]
+        res = oracle.moe_layer(h_in[l][ps], w["w_router"], w["w_gate_up"], w["w_down"],
+                               k_all[pool[ps]], cfg.k_max)
+        oracle.residual_bf16(h_in[l][ps], res["out"])
+
+    per_step_s = min(5.0, 120.0 / max(1, args.steps + args.warmup))
+    n0 = min(P, 4 * threads)
+    t0 = time.perf_counter()
+    one(n0)
+    dt0 = time.perf_counter() - t0
+    n = int(min(P, max(1, n0 * per_step_s / max(dt0, 1e-6))))
     for _ in range(args.warmup):
-        one()
+        one(n)
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        one()
+        one(n)
     dt = time.perf_counter() - t0
-    value = n * args.steps / dt
-    sample = (f"{n} seeded tokens of the {T}-token batch per step through all "
-              f"{STACK_LAYERS} layers (counts on the whole batch)")
+    value = n / L * args.steps / dt
+    sample = (f"per step one seeded layer of {L} through {n} seeded tokens of a pool "
+              f"of {P} from the {T}-token batch, on their inputs at that layer (from "
+              f"an untimed oracle pass), plus the whole batch's counts: {n} / {L} "
+              f"whole forwards per step")
     line = dict(metric=METRIC, value=value, unit="tokens/s", impl="reference",
                 n_gpus=args.gpus, steps=args.steps, warmup=args.warmup,
                 ms_per_step=1e3 * dt / args.steps, higher_is_better=True,
                 scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
                 config=stack_config(world),
                 cpu_baseline=dict(value=value, unit="tokens/s", kind="oracle",
-                                  cores=oracle.num_threads(), sample=sample),
+                                  cores=threads, sample=sample),
                 e2e=dict(value=value, unit="tokens/s", h2d_bytes_per_step=0,
                          d2h_bytes_per_step=0))
     print(json.dumps(line), flush=True)
