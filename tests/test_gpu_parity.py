@@ -402,6 +402,8 @@ def test_screened_routing_router_rows_16_byte_aligned():
     (8256, 40, 512, 6),      # fewer experts than the 64-row expert box
     (8192, 64, 256, 12),     # short rows (4 chunks)
     (16384, 17, 2048, 4),    # odd expert count
+    (12289, 64, 1024, 8),    # one token in the last CTA
+    (30000, 48, 512, 12),    # ragged last CTA, 48 experts
 ])
 def test_batch_screened_routing_bit_exact(T, E, d, kmax):
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=5 * T + E + d)
