@@ -91,6 +91,9 @@ def parse():
     ap.add_argument("--ablation", action="store_true",
                     help="REFLEX and its App. C allocation ablations on one layer")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--gather-in-gemm", action="store_true",
+                    help="fused dispatch: the CTA-pair gate/up GEMM gathers its "
+                         "rows (REFLEX_FLAG_GATHER_IN_GEMM; slower, off by default)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target seconds of oracle work for cpu_baseline")
@@ -289,7 +292,7 @@ def run_gpu(args, cfg, rank, world, local_rank):
     k_sum = torch.zeros(1, dtype=torch.int64, device=dev)
     st = torch.zeros(1, dtype=torch.int32, device=dev)
     out = torch.empty((T, d), dtype=moe.tdtype, device=dev)
-    F = B.REFLEX_FLAG_RENORM_TOPK
+    F = B.REFLEX_FLAG_RENORM_TOPK | (B.REFLEX_FLAG_GATHER_IN_GEMM if args.gather_in_gemm else 0)
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
 
     # every call takes the current stream, so the steps can be captured into
@@ -504,6 +507,8 @@ def run_gpu(args, cfg, rank, world, local_rank):
                                sample=f"{n1} seeded tokens, {dt1:.1f} s"))
     elif world > 1:
         line["cpu_baseline"] = None
+    if args.gather_in_gemm:
+        line["dispatch"] = "rows gathered inside the gate/up GEMM (REFLEX_FLAG_GATHER_IN_GEMM)"
     print(json.dumps(line), flush=True)
 
 
@@ -669,7 +674,7 @@ def run_stack(args, rank, world, local_rank):
     k_sum = torch.zeros(1, dtype=torch.int64, device=dev)
     st = torch.zeros(1, dtype=torch.int32, device=dev)
     out = torch.empty_like(h0)
-    F = B.REFLEX_FLAG_RENORM_TOPK
+    F = B.REFLEX_FLAG_RENORM_TOPK | (B.REFLEX_FLAG_GATHER_IN_GEMM if args.gather_in_gemm else 0)
     p_reflex = B.make_params(**cfg.alloc_params())
     p_fixed = B.make_params(**cfg.alloc_params(delta_role=0, delta_cur=0))
 
@@ -854,6 +859,8 @@ def run_stack(args, rank, world, local_rank):
                                sample=f"{n1} seeded tokens, {dt1:.1f} s"))
     elif world > 1:
         line["cpu_baseline"] = None
+    if args.gather_in_gemm:
+        line["dispatch"] = "rows gathered inside the gate/up GEMM (REFLEX_FLAG_GATHER_IN_GEMM)"
     print(json.dumps(line), flush=True)
 
 

@@ -71,11 +71,25 @@ extern "C" {
  * bits either way (the screen's bound is stated with reflex_moe_forward);
  * only the record's other scores differ (tensor-core estimates). */
 #define REFLEX_FLAG_EXACT_SCORES 0x8u
+/* bf16 tcgen05 path, routed gate/up GEMM on CTA pairs (at least 128 rows
+ * per expert expected: T * k_max / (2 E) >= 128, inter % 128 == 0, d % 256
+ * == 0): the GEMM fetches its input rows from hidden itself with four-row
+ * TMA gathers through the pair permutation, and DISPATCH only places the
+ * pairs (no copy of the rows in pair order is written).  The outputs are the
+ * same bits as without the flag.  Elsewhere the flag changes nothing.  The
+ * fused dispatch is slower on GB300 (a four-row gather costs about four
+ * times what a row of a tiled box does: the 32 x 1024-token LLaDA-MoE layer's
+ * gate/up GEMM 0.84 -> 3.08 ms), so it is off by default.  With stage
+ * selection the DISPATCH and EXPERT_UP calls must agree on the flag. */
+#define REFLEX_FLAG_GATHER_IN_GEMM 0x10u
 /* Stage selection.  No stage bit = all five stages in order.  Stages read
  * what the previous stages left in the same workspace; running a stage whose
  * predecessors did not run on that workspace gives unspecified values (every
  * index read from the workspace is range-checked on the device, so no
- * out-of-bounds access results). */
+ * out-of-bounds access results).  hidden must hold the same values at the
+ * DISPATCH and EXPERT_UP stages of one forward (the shared expert reads it
+ * at EXPERT_UP, and so do the routed experts with REFLEX_FLAG_GATHER_IN_GEMM)
+ * and, with REFLEX_FLAG_RESIDUAL, at COMBINE. */
 #define REFLEX_STAGE_ROUTE 0x100u       /* router scores, TopK, alpha        */
 #define REFLEX_STAGE_DISPATCH 0x200u    /* pair counts, offsets, permutation */
 #define REFLEX_STAGE_EXPERT_UP 0x400u   /* gate/up GEMM + SwiGLU (+ shared)  */

@@ -28,6 +28,7 @@ REFLEX_FLAG_RENORM_TOPK = 0x1
 REFLEX_FLAG_SIMT_EXPERTS = 0x2
 REFLEX_FLAG_RESIDUAL = 0x4
 REFLEX_FLAG_EXACT_SCORES = 0x8
+REFLEX_FLAG_GATHER_IN_GEMM = 0x10
 REFLEX_SIGNAL_FPS = 0
 REFLEX_SIGNAL_FRONTIER = 1
 REFLEX_SIGNAL_PROGRESS = 2
@@ -37,7 +38,7 @@ REFLEX_RULE_REFLEX = 0
 REFLEX_RULE_TOP_P = 1
 REFLEX_RULE_EXPERT_THRESHOLD = 2
 # the reflex_alloc_params layout above matches this ABI version
-ABI_VERSION = 113
+ABI_VERSION = 114
 REFLEX_STAGE_ROUTE = 0x100
 REFLEX_STAGE_DISPATCH = 0x200
 REFLEX_STAGE_EXPERT_UP = 0x400

@@ -12,7 +12,8 @@
 //           256-row tile counts = tile prefixes for the grouped GEMMs;
 //   gather  the row of pair (t, j) is offsets[e] + block prefix + popcount
 //           of the lower tokens' bits in the block's masks (kept in global
-//           memory by count); X rows are copied into pair order on the way.
+//           memory by count); X rows are copied into pair order on the way
+//           (with REFLEX_FLAG_GATHER_IN_GEMM the CTA-pair GEMM fetches them).
 // Short batches whose masks fit in one CTA's shared memory take two: count
 // and scan in one CTA, then the gather.
 #include "common.cuh"
@@ -232,7 +233,8 @@ __global__ void __launch_bounds__(1024)
   }
 }
 
-// Token-order gather with the scatter step.  W warps per token (W = 1 for
+// Token-order gather with the scatter step (xp == nullptr: the pairs are
+// placed and no row is copied; the grouped GEMM gathers the rows itself).  W warps per token (W = 1 for
 // long batches), each reading one 1/W segment of the token's hidden row
 // once (up to 8 16-byte vectors per lane in flight) and writing it to each
 // of the token's k_t pair rows, so every hidden row crosses HBM once however
@@ -269,10 +271,12 @@ __global__ void __launch_bounds__(256)
     // loads overlap the position lookups
     const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(t) * d) + v0;
     uint4 v[kMaxVec];
+    if (xp != nullptr) {
 #pragma unroll
-    for (int i = 0; i < kMaxVec; ++i) {
-      const int q = lane + 32 * i;
-      if (q < seg_vecs) v[i] = __ldg(src + q);
+      for (int i = 0; i < kMaxVec; ++i) {
+        const int q = lane + 32 * i;
+        if (q < seg_vecs) v[i] = __ldg(src + q);
+      }
     }
     int my_row = -1;
     if (lane < k_max) {
@@ -309,6 +313,7 @@ __global__ void __launch_bounds__(256)
         if (my_row >= 0) perm[my_row] = static_cast<int32_t>(o);
       }
     }
+    if (xp == nullptr) continue;  // placement only
     for (int base = 0; base < seg_vecs; base += 32 * kMaxVec) {
       if (base > 0) {
 #pragma unroll
@@ -333,10 +338,11 @@ __global__ void __launch_bounds__(256)
 
 // warps per token for the gather (enough warps for 16 per SM, each segment
 // whole 16-byte vectors) and the grid
-void gather_shape(int dtype, int T, int d, int num_sms, int* wpt_out, int* grid_out) {
+void gather_shape(int dtype, int T, int d, int num_sms, bool copy, int* wpt_out,
+                  int* grid_out) {
   const int row_vecs = d * (dtype == 0 ? 4 : 2) / 16;
   int wpt = 1;
-  while (wpt < 8 && static_cast<int64_t>(T) * wpt < 16LL * num_sms &&
+  while (copy && wpt < 8 && static_cast<int64_t>(T) * wpt < 16LL * num_sms &&
          row_vecs % (2 * wpt) == 0)
     wpt *= 2;
   const int64_t warps = static_cast<int64_t>(T) * wpt;
@@ -390,7 +396,7 @@ static cudaError_t launch_gather_scatter(const Te* hidden, const int32_t* ids, c
                                          const DispatchBufs& b, Te* x_perm, int num_sms,
                                          cudaStream_t stream) {
   int wpt, grid;
-  gather_shape(sizeof(Te) == 4 ? 0 : 1, T, d, num_sms, &wpt, &grid);
+  gather_shape(sizeof(Te) == 4 ? 0 : 1, T, d, num_sms, x_perm != nullptr, &wpt, &grid);
   return launch_pdl(gather_scatter_kernel<Te, KW>, dim3(grid), dim3(256), 0, stream, hidden,
                     ids, k, static_cast<const uint32_t*>(b.blk_mask),
                     static_cast<const int32_t*>(b.blk_off), static_cast<const int32_t*>(b.offsets),

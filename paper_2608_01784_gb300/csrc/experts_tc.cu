@@ -89,6 +89,10 @@ struct KParams {
   int b3d;
   // scores mode, k_splits == 1: sum of squares of every A row (fp32), nullable
   float* norm_out;
+  // SwiGLU on CTA pairs: A rows gathered from the token rows (TcGemmArgs)
+  const int32_t* gather_perm;
+  int gather_kmax;
+  int gather_tokens;
 };
 
 // ---- PTX wrappers ---------------------------------------------------------
@@ -619,6 +623,9 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.defer_wait = 0;
   p.b3d = MODE == kModeSwiGLU && a.b_gate_up_3d ? 1 : 0;
   p.norm_out = nullptr;
+  p.gather_perm = nullptr;
+  p.gather_kmax = 1;
+  p.gather_tokens = 0;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   const int grid = static_cast<int>(max_tiles < a.num_sms ? max_tiles : a.num_sms);
@@ -632,8 +639,13 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
 // A cluster of two CTAs on one TPC computes a 256 x 256 tile: CTA rank r
 // holds rows [row0 + 128 r, +128) of A and one half of the weight tile
 // (SwiGLU: rank 0 the 128 gate rows, rank 1 the 128 matching up rows; down:
-// rows n*256 + 128 r of W_down), so each SM streams 32 KB per 64-k stage
-// instead of 48 KB, and the 192 KB ring holds 6 stages.  One thread of the
+// rows n*256 + 128 r of W_down), so each SM streams 32 KB per 64-k block
+// instead of 48 KB; the 192 KB ring holds 3 stages of two consecutive 64-k
+// blocks.  With gathered rows (SwiGLU, TcGemmArgs::gather_perm) the A rows
+// come straight from the token rows: every lane of the producer warp issues
+// one four-row TMA gather per 64-k block, the tokens looked up through the
+// pair permutation once per tile; the rows, tiles and MMA order are those of
+// the copied rows, so the outputs are the same bits.  One thread of the
 // leader CTA (rank 0) issues tcgen05.mma.cta_group::2 (M = 256, N = 256);
 // each CTA's TMEM receives its 128 rows x 256 fp32 columns (two buffers of
 // 256 columns, allocated collectively by one warp per CTA).
@@ -685,6 +697,19 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(cl_bar)
+      : "memory");
+}
+// Four rows r0..r3 of a map whose box is {64, 1}, copied to four consecutive
+// 128-byte rows at dst (the same 128-byte swizzle as a tiled box: it follows
+// the shared-memory address, and dst is 512-byte aligned, half of an 8-row
+// swizzle atom), completion counted on a barrier in either CTA of the pair.
+__device__ __forceinline__ void tma_gather4_pair(uint32_t dst, const CUtensorMap* map, int c0,
+                                                 const int (&r)[4], uint32_t cl_bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
+      ".cta_group::2 [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]),
+      "r"(cl_bar)
       : "memory");
 }
 __device__ __forceinline__ void mma_bf16_pair(uint32_t tmem_d, uint64_t da, uint64_t db,
@@ -812,7 +837,11 @@ __global__ void __launch_bounds__(kThreads2, 1)
   const int ntiles = total_tiles(p);
   const int nk = p.K / (BK * C::KS);  // stages per tile
 
-  if (warp == 0 && lane == 0) {
+  // SwiGLU with gathered A rows: the whole producer warp issues the A
+  // copies, one four-row gather per lane and 64-k block (lane l: rows 4 l ..
+  // 4 l + 3 of this CTA's 128); otherwise lane 0 issues everything
+  const bool gather = MODE == kModeSwiGLU && p.gather_perm != nullptr;
+  if (warp == 0 && (gather || lane == 0)) {
     // ---------------- TMA producer (each CTA: its A rows, its B half) -------
     int stage = 0;
     uint32_t phase = 0;
@@ -820,34 +849,64 @@ __global__ void __launch_bounds__(kThreads2, 1)
     bool ok = true;
     for (int t = pair; t < ntiles && ok; t += npairs) {
       Tile tl;
-      if (!decode_tile(p, t, tl)) {
-        set_err(p.err, kErrIndex);
-        *abort_flag = 1;
+      if (!decode_tile(p, t, tl)) {  // the same outcome in every lane
+        if (lane == 0) {
+          set_err(p.err, kErrIndex);
+          *abort_flag = 1;
+        }
         break;
       }
+      // token of each of this lane's four rows; rows past the tile's end
+      // repeat its last row (computed, never stored)
+      int tok[4] = {0, 0, 0, 0};
+      if (gather) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int r = min(static_cast<int>(rank) * BM + 4 * lane + i, tl.rows - 1);
+          const int o = p.gather_perm[tl.row0 + r];
+          const int tk = o >= 0 ? o / p.gather_kmax : -1;
+          if (tk < 0 || tk >= p.gather_tokens)
+            set_err(p.err, kErrIndex);
+          else
+            tok[i] = tk;
+        }
+      }
       for (int kb = 0; kb < nk; ++kb) {
-        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitNs)) {
+        // every issuing lane observes the stage's release itself
+        const bool w = mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitNs);
+        if (!(gather ? __all_sync(0xffffffffu, w) : w)) {
           ok = false;
           break;
         }
         const uint32_t fb = map_to_rank(smem_addr(&full[stage]), 0);
-        if (leader)
-          mbar_expect_tx(smem_addr(&full[stage]), C::kStageBytes);
-        else
-          mbar_expect_tx_cluster(fb, C::kStageBytes);
         int brow;
         if (MODE == kModeSwiGLU)
           brow = tl.e * p.b_rows_per_group + (rank ? p.b_up_offset : 0) + tl.n * (BN / 2);
         else
           brow = tl.e * p.b_rows_per_group + tl.n * BN + static_cast<int>(rank) * (BN / 2);
-        // consecutive k blocks of the same rows back to back
+        if (lane == 0) {
+          if (leader)
+            mbar_expect_tx(smem_addr(&full[stage]), C::kStageBytes);
+          else
+            mbar_expect_tx_cluster(fb, C::kStageBytes);
+          // consecutive k blocks of the same rows back to back
 #pragma unroll
-        for (int u = 0; u < C::KS; ++u) {
-          const int k0 = (kb * C::KS + u) * BK;
-          tma_load_2d_pair(smem_addr(sa + stage * C::kABytes + u * C::kSubBytes), &map_a, k0,
-                           tl.row0 + static_cast<int>(rank) * BM, fb);
-          tma_load_2d_pair(smem_addr(sb + stage * C::kBBytes + u * C::kSubBytes), &map_b, k0,
-                           brow, fb);
+          for (int u = 0; u < C::KS; ++u) {
+            const int k0 = (kb * C::KS + u) * BK;
+            if (!gather)
+              tma_load_2d_pair(smem_addr(sa + stage * C::kABytes + u * C::kSubBytes), &map_a,
+                               k0, tl.row0 + static_cast<int>(rank) * BM, fb);
+            tma_load_2d_pair(smem_addr(sb + stage * C::kBBytes + u * C::kSubBytes), &map_b, k0,
+                             brow, fb);
+          }
+        }
+        if (gather) {
+          __syncwarp();
+#pragma unroll
+          for (int u = 0; u < C::KS; ++u)
+            tma_gather4_pair(
+                smem_addr(sa + stage * C::kABytes + u * C::kSubBytes + lane * 4 * 128), &map_a,
+                (kb * C::KS + u) * BK, tok, fb);
         }
         issued_mask |= 1u << stage;
         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -857,14 +916,16 @@ __global__ void __launch_bounds__(kThreads2, 1)
         }
       }
     }
-    if (!ok) {
-      set_err(p.err, kErrTimeout);
-      *abort_flag = 1;
-    }
-    if (*abort_flag && leader) {
-      for (int s = 0; s < kStages; ++s)
-        if (issued_mask & (1u << s))
-          mbar_wait(&full[s], (issued_phase >> s) & 1u, nullptr, kDrainNs);
+    if (lane == 0) {
+      if (!ok) {
+        set_err(p.err, kErrTimeout);
+        *abort_flag = 1;
+      }
+      if (*abort_flag && leader) {
+        for (int s = 0; s < kStages; ++s)
+          if (issued_mask & (1u << s))
+            mbar_wait(&full[s], (issued_phase >> s) & 1u, nullptr, kDrainNs);
+      }
     }
   } else if (warp == 1 && lane == 0 && leader) {
     // ---------------- MMA issuer (leader CTA only) ----------------
@@ -1056,6 +1117,11 @@ cudaError_t launch_pair_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.defer_wait = 0;
   p.b3d = 0;
   p.norm_out = nullptr;
+  p.gather_perm = MODE == kModeSwiGLU ? a.gather_perm : nullptr;
+  p.gather_kmax = a.gather_kmax;
+  p.gather_tokens = a.gather_tokens;
+  if (p.gather_perm != nullptr && (p.gather_kmax < 1 || p.gather_tokens < 1))
+    return cudaErrorInvalidValue;
   const int64_t max_tiles = static_cast<int64_t>(p.n_tiles) * p.max_mtiles;
   if (max_tiles == 0) return cudaSuccess;
   int pairs = a.num_sms / 2;

@@ -145,7 +145,8 @@ inline int64_t dispatch_blocks_alloc(int T) {
          (T + kDispatchBlock - 1) / kDispatchBlock;
 }
 // The pair layout (counts, offsets, tile prefixes, perm, row_of) and the
-// gathered rows X_perm[row_of[t, j]] = X[t] for j < k_t.
+// gathered rows X_perm[row_of[t, j]] = X[t] for j < k_t (x_perm nullptr:
+// the layout only, for a consumer that gathers the rows itself).
 // mask words for either block size (monotonic in T, like the block counts)
 inline int64_t dispatch_mask_words_alloc(int T) {
   const int ts = T < kDispatchSmallT ? T : kDispatchSmallT;
@@ -192,6 +193,13 @@ struct TcGemmArgs {
   // SwiGLU, 1-SM kernel: map_b is the 3D map of tc_gate_up_3d (box {64,
   // bn / 2, 2}: a tile's gate and up rows in one copy) instead of a 2D map
   bool b_gate_up_3d = false;
+  // SwiGLU, CTA-pair kernel: when set, map_a is a {64, 1}-box map of the
+  // token rows X [gather_tokens, K], and A row r is token gather_perm[r] /
+  // gather_kmax (row r's pair index over k_max), fetched by four-row TMA
+  // gathers; nullptr: map_a holds the rows in pair order
+  const int32_t* gather_perm = nullptr;
+  int gather_kmax = 0;
+  int gather_tokens = 0;
 };
 // SwiGLU: out = silu(A Wg^T) * (A Wu^T).  Down: out = A Wd^T.  bn = tile
 // width (128 or 256, from tc_pick_bn); the B tensor map's box must have

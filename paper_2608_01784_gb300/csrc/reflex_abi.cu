@@ -238,7 +238,7 @@ cudaError_t launch_alloc(const AllocCall& c, int32_t T, cudaStream_t s, bool alo
 
 extern "C" {
 
-int reflex_abi_version(void) { return 113; }
+int reflex_abi_version(void) { return 114; }
 
 const char* reflex_status_string(int s) {
   switch (s) {
@@ -397,6 +397,9 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
   // (LLaDA2.0-mini layer, about 160 rows per expert: 0.820 -> 0.749 ms)
   const int64_t rows_per_group_est = static_cast<int64_t>(T) * k_max / 2 / E;
   const bool pair_routed = rows_per_group_est >= 128 && inter % 128 == 0 && d % 256 == 0;
+  // fused dispatch (opt-in): the CTA-pair gate/up GEMM gathers its rows from
+  // hidden through perm, and the dispatch only places the pairs
+  const bool gemm_gathers = !simt && pair_routed && (flags & REFLEX_FLAG_GATHER_IN_GEMM);
   if (!simt) {
     if (bn_up == 0 || bn_dn == 0 || bn_sup == 0 || bn_sdn == 0) return REFLEX_EUNSUPPORTED;
     if (encode_fn() == nullptr) return REFLEX_ECUDA;
@@ -511,7 +514,7 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
                        I32(L.perm),      I32(L.row_of),    totals,
                        err,              reinterpret_cast<uint32_t*>(ws + L.blk_mask)};
     RX_CUDA(rx::launch_dispatch_gather(dtype, hidden, I32(L.ids), k, T, E, k_max, cap, d, b,
-                                       xperm, sms, s));
+                                       gemm_gathers ? nullptr : xperm, sms, s));
   }
   const bool up = (stages & REFLEX_STAGE_EXPERT_UP) != 0;
   const bool down = (stages & REFLEX_STAGE_EXPERT_DOWN) != 0;
@@ -532,7 +535,8 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
       }
     } else {
       CUtensorMap ma1, mb1, ma2, mb2;
-      if (!make_map(&ma1, xperm, cap, d, rx::kTileM) ||
+      if (!(gemm_gathers ? make_map(&ma1, hidden, T, d, 1)
+                         : make_map(&ma1, xperm, cap, d, rx::kTileM)) ||
           !(pair_routed ? make_map(&mb1, w_gate_up, static_cast<int64_t>(E) * 2 * inter, d, 128)
                         : make_map_gate_up(&mb1, w_gate_up, E, inter, d,
                                            rx::tc_b_box_rows(true, bn_up))) ||
@@ -542,6 +546,11 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
         return REFLEX_ECUDA;
       rx::TcGemmArgs g1{&ma1, &mb1, d, inter, 2 * inter, inter, grouped, amid, inter, err, sms,
                         !pair_routed};
+      if (gemm_gathers) {
+        g1.gather_perm = I32(L.perm);
+        g1.gather_kmax = k_max;
+        g1.gather_tokens = T;
+      }
       rx::TcGemmArgs g2{&ma2, &mb2, inter, d, d, 0, grouped, xperm, d, err, sms};
       // the dense shared expert on CTA pairs once it has enough rows: a 256 x
       // 256 pair tile moves a quarter of the operand bytes per output that a

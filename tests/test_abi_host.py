@@ -48,7 +48,7 @@ def test_status_strings_and_version(lib):
     assert B.reflex_status_string(B.REFLEX_OK) == "ok"
     assert "workspace" in B.reflex_status_string(B.REFLEX_EWORKSPACE)
     assert B.reflex_status_string(999) == "unknown status"
-    assert B.reflex_abi_version() == B.ABI_VERSION == 113
+    assert B.reflex_abi_version() == B.ABI_VERSION == 114
 
 
 def test_default_params_are_the_paper_settings(lib):

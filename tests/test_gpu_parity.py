@@ -626,6 +626,7 @@ def test_forward_count_out_of_range_flagged():
     ("llada_moe", 0),
     ("llada2_mini", 0),
     ("llada_moe", B.REFLEX_FLAG_RESIDUAL),
+    ("llada2_mini", B.REFLEX_FLAG_GATHER_IN_GEMM),  # DISPATCH places, EXPERT_UP gathers
 ])
 def test_forward_stages_compose(name, extra):
     cfg = CFG[name]
@@ -642,6 +643,54 @@ def test_forward_stages_compose(name, extra):
                        flags=B.REFLEX_FLAG_RENORM_TOPK | extra | st)
     torch.cuda.synchronize()
     assert np.array_equal(G.to_f32(out), full)
+
+
+# ---------------------------------------------------------------------------
+# fused dispatch (REFLEX_FLAG_GATHER_IN_GEMM): the CTA-pair gate/up GEMM
+# fetches its rows from the token rows with four-row TMA gathers; same rows,
+# tiles and MMA order as the copied rows, so the same output bits
+# ---------------------------------------------------------------------------
+_GATHER = B.REFLEX_FLAG_RENORM_TOPK | B.REFLEX_FLAG_GATHER_IN_GEMM
+
+
+@pytest.mark.parametrize("T,d,E,inter,kmax,kmode", [
+    (1500, 256, 8, 256, 4, "random"),   # a few hundred rows per group
+    (4096, 256, 4, 128, 4, "random"),   # ragged groups
+    (2048, 512, 8, 256, 4, "max"),      # several n-tiles
+    (1030, 256, 4, 128, 1, "one"),      # last tile a row or two: clamped gathers
+    (4099, 256, 4, 128, 4, "max"),      # the last token gathered, T % 4 != 0
+    (300, 256, 64, 128, 2, "one"),      # 1-SM tiles: the flag changes nothing
+])
+def test_gather_in_gemm_gives_the_default_bits(T, d, E, inter, kmax, kmode):
+    cfg, layer = _bf16_case(T, d, E, inter, 0, kmax, seed=T + E + 1)
+    rng = np.random.default_rng(T + 1)
+    if kmode == "random":
+        k = rng.integers(1, kmax + 1, T).astype(np.int32)
+    elif kmode == "max":
+        k = np.full(T, kmax, np.int32)
+    else:
+        k = np.ones(T, np.int32)
+    gl = G.GpuLayer(cfg, layer)
+    out_d, _, st_d = gl.forward(k)
+    out_g, rec_g, st_g = gl.forward(k, flags=_GATHER)
+    assert st_d == B.REFLEX_OK and st_g == B.REFLEX_OK
+    assert np.array_equal(out_g.view(np.uint32), out_d.view(np.uint32))
+    ref = G.oracle_layer(cfg, layer, k)
+    G.check_routing(rec_g, ref, k, cfg.E)
+    rel, mx = G.out_errors(out_g, ref["out"])
+    assert rel <= G.BF16_REL_L2 and mx <= G.BF16_MAX_ABS, (rel, mx)
+
+
+@pytest.mark.parametrize("name", ["llada2_mini", "llada_moe_b32"])
+def test_gather_in_gemm_full_layers_give_the_default_bits(name):
+    cfg = CFG[name]
+    layer = W.make_layer(cfg, 3)
+    k = _k_for(cfg, 3)
+    gl = G.GpuLayer(cfg, layer)
+    out_d, _, st_d = gl.forward(k)
+    out_g, _, st_g = gl.forward(k, flags=_GATHER)
+    assert st_d == B.REFLEX_OK and st_g == B.REFLEX_OK
+    assert np.array_equal(out_g.view(np.uint32), out_d.view(np.uint32))
 
 
 # ---------------------------------------------------------------------------
