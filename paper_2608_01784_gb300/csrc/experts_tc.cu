@@ -60,7 +60,8 @@ struct Cfg {
   static constexpr int kStages = kRingBytes / kStageBytes;  // 4 (BN 256), 6 (BN 128)
   static constexpr int kTmemCols = 2 * BN;
   static constexpr int kBarBytes = 256;
-  static constexpr int kSmemBytes = kStages * kStageBytes + kBarBytes + 1024;
+  static constexpr int kIndexInts = 2 * 1025;  // both prefix arrays, E <= 1024
+  static constexpr int kSmemBytes = kStages * kStageBytes + kBarBytes + kIndexInts * 4 + 1024;
   static_assert(kStages >= 2 && kStages <= 8, "ring depth");
 };
 
@@ -230,12 +231,41 @@ struct Tile {
   int ks;      // K slice (scores mode; 0 otherwise)
 };
 
-__device__ __forceinline__ int total_tiles(const KParams& p) {
+// The group prefix arrays a tile lookup reads: copies in shared memory where
+// they fit, else the global arrays.  Looking a tile up takes a binary search
+// over the experts; from global memory that is a chain of about log2(E) + 2
+// dependent L2 loads (about 3 us), longer than the ring's lead over the MMAs
+// at each tile start, so the copies are made once per CTA.
+struct TileIndex {
+  const int32_t* pref;  // [E+1] tile-count prefix (p.mt_prefix)
+  const int32_t* offs;  // [E+1] row offsets (p.g.offsets)
+};
+// Every thread of the CTA calls this (it synchronises the CTA) after the
+// kernel's dependency wait; cache holds cap ints.
+__device__ __forceinline__ TileIndex load_tile_index(const KParams& p, int32_t* cache,
+                                                     int cap) {
+  TileIndex ix{p.mt_prefix, p.g.offsets};
+  if (p.g.offsets == nullptr) return ix;
+  const int n = p.g.E + 1;
+  const bool both = 2 * n <= cap, pref_only = !both && n <= cap;
+  if (both || pref_only) {
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+      cache[i] = p.mt_prefix[i];
+      if (both) cache[n + i] = p.g.offsets[i];
+    }
+    __syncthreads();
+    ix.pref = cache;
+    if (both) ix.offs = cache + n;
+  }
+  return ix;
+}
+
+__device__ __forceinline__ int total_tiles(const KParams& p, const TileIndex& ix) {
   int mt;
   if (p.g.offsets == nullptr) {
     mt = (p.g.dense_rows + p.tile_rows - 1) / p.tile_rows * p.k_splits;
   } else {
-    mt = p.mt_prefix[p.g.E];
+    mt = ix.pref[p.g.E];
     if (mt < 0) mt = 0;
     if (mt > p.max_mtiles) mt = p.max_mtiles;
   }
@@ -243,7 +273,8 @@ __device__ __forceinline__ int total_tiles(const KParams& p) {
 }
 
 // Tile t -> (expert, n-tile, rows); false when the workspace is inconsistent.
-__device__ __forceinline__ bool decode_tile(const KParams& p, int t, Tile& o) {
+__device__ __forceinline__ bool decode_tile(const KParams& p, const TileIndex& ix, int t,
+                                            Tile& o) {
   if (p.g.offsets == nullptr) {
     const int mt = (p.g.dense_rows + p.tile_rows - 1) / p.tile_rows;
     const int per = mt * p.n_tiles;
@@ -260,16 +291,16 @@ __device__ __forceinline__ bool decode_tile(const KParams& p, int t, Tile& o) {
   int lo = 0, hi = p.g.E;  // n_tiles*prefix[lo] <= t < n_tiles*prefix[hi]
   while (hi - lo > 1) {
     const int mid = (lo + hi) >> 1;
-    if (p.n_tiles * p.mt_prefix[mid] <= t) lo = mid; else hi = mid;
+    if (p.n_tiles * ix.pref[mid] <= t) lo = mid; else hi = mid;
   }
-  const int mt_e = p.mt_prefix[lo + 1] - p.mt_prefix[lo];
+  const int mt_e = ix.pref[lo + 1] - ix.pref[lo];
   if (mt_e <= 0) return false;
-  const int l = t - p.n_tiles * p.mt_prefix[lo];
+  const int l = t - p.n_tiles * ix.pref[lo];
   o.e = lo;
   o.mtiles = mt_e;
   o.n = l / mt_e;
-  o.row0 = p.g.offsets[lo] + (l % mt_e) * p.tile_rows;
-  o.rows = min(p.tile_rows, p.g.offsets[lo + 1] - o.row0);
+  o.row0 = ix.offs[lo] + (l % mt_e) * p.tile_rows;
+  o.rows = min(p.tile_rows, ix.offs[lo + 1] - o.row0);
   return o.n < p.n_tiles && o.row0 >= 0 && o.rows > 0 &&
          o.row0 + o.rows <= p.g.cap_rows;
 }
@@ -322,7 +353,10 @@ __global__ void __launch_bounds__(MODE == kModeScores ? kThreadsScores : kThread
   // the tile count and every operand come from earlier kernels
   if (!p.defer_wait) grid_dep_wait();
   grid_dep_launch();
-  const int ntiles = total_tiles(p);
+  const TileIndex ix = load_tile_index(
+      p, reinterpret_cast<int32_t*>(smem + kStages * C::kStageBytes + C::kBarBytes),
+      C::kIndexInts);
+  const int ntiles = total_tiles(p, ix);
   const int nk = p.K / BK / p.k_splits;  // k-blocks per tile
 
   if (warp == 0 && lane == 0) {
@@ -335,7 +369,7 @@ __global__ void __launch_bounds__(MODE == kModeScores ? kThreadsScores : kThread
     const uint64_t pol_once = l2_policy(kPolFirst);
     for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
       Tile tl;
-      if (!decode_tile(p, t, tl)) {
+      if (!decode_tile(p, ix, t, tl)) {
         set_err(p.err, kErrIndex);
         *abort_flag = 1;
         break;
@@ -443,7 +477,7 @@ __global__ void __launch_bounds__(MODE == kModeScores ? kThreadsScores : kThread
       bool ok = true;
       for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
         Tile tl;
-        const bool tile_ok = decode_tile(p, t, tl);
+        const bool tile_ok = decode_tile(p, ix, t, tl);
         float ss = 0.f;
         for (int kb = 0; kb < nk; ++kb) {
           // every lane observes the stage's completion before reading it
@@ -490,7 +524,7 @@ __global__ void __launch_bounds__(MODE == kModeScores ? kThreadsScores : kThread
     int lt = 0;
     for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++lt) {
       Tile tl;
-      const bool tile_ok = decode_tile(p, t, tl);
+      const bool tile_ok = decode_tile(p, ix, t, tl);
       const int ab = lt & 1;
       const uint32_t acc_phase = (lt >> 1) & 1;
       int ok = 1;
@@ -751,8 +785,9 @@ struct Cfg2 {
   static constexpr int kStages = kRingBytes / kStageBytes;  // 3
   static constexpr int kTmemCols = 2 * BN;       // two accumulators
   static constexpr int kStagingBytes = 32 * 128; // per epilogue warp: 32 rows x 128 B
+  static constexpr int kIndexInts = 384;         // both prefix arrays to E = 191, the first to 383
   static constexpr int kSmemBytes =
-      kStages * kStageBytes + 256 + kEpiWarps2 * kStagingBytes + 1024;
+      kStages * kStageBytes + 256 + kEpiWarps2 * kStagingBytes + kIndexInts * 4 + 1024;
   static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
 };
 
@@ -833,8 +868,13 @@ __global__ void __launch_bounds__(kThreads2, 1)
   const uint32_t tmem_base = *tmem_slot;
   grid_dep_wait();
   grid_dep_launch();
+  const TileIndex ix = load_tile_index(
+      p,
+      reinterpret_cast<int32_t*>(smem + kStages * C::kStageBytes + 256 +
+                                 kEpiWarps2 * C::kStagingBytes),
+      C::kIndexInts);
   // tiles are 256 rows (both CTAs) x 256 columns; mt_prefix counts 256-row tiles
-  const int ntiles = total_tiles(p);
+  const int ntiles = total_tiles(p, ix);
   const int nk = p.K / (BK * C::KS);  // stages per tile
 
   // SwiGLU with gathered A rows: the whole producer warp issues the A
@@ -849,7 +889,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
     bool ok = true;
     for (int t = pair; t < ntiles && ok; t += npairs) {
       Tile tl;
-      if (!decode_tile(p, t, tl)) {  // the same outcome in every lane
+      if (!decode_tile(p, ix, t, tl)) {  // the same outcome in every lane
         if (lane == 0) {
           set_err(p.err, kErrIndex);
           *abort_flag = 1;
@@ -995,7 +1035,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
     int lt = 0;
     for (int t = pair; t < ntiles; t += npairs, ++lt) {
       Tile tl;
-      const bool tile_ok = decode_tile(p, t, tl);
+      const bool tile_ok = decode_tile(p, ix, t, tl);
       const int ab = lt & 1;
       const uint32_t acc_phase = (lt >> 1) & 1;
       int ok = 1;
