@@ -90,6 +90,8 @@ struct KParams {
   int b3d;
   // scores mode, k_splits == 1: sum of squares of every A row (fp32), nullable
   float* norm_out;
+  // CTA pairs: whole 32-row output chunks leave by TMA store (map_out)
+  int tma_out;
   // SwiGLU on CTA pairs: A rows gathered from the token rows (TcGemmArgs)
   const int32_t* gather_perm;
   int gather_kmax;
@@ -657,6 +659,7 @@ cudaError_t launch_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.defer_wait = 0;
   p.b3d = MODE == kModeSwiGLU && a.b_gate_up_3d ? 1 : 0;
   p.norm_out = nullptr;
+  p.tma_out = 0;
   p.gather_perm = nullptr;
   p.gather_kmax = 1;
   p.gather_tokens = 0;
@@ -791,6 +794,25 @@ struct Cfg2 {
   static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
 };
 
+// TMA tile store of a shared-memory box (bulk-group completion) and its waits.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int c0,
+                                             int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];"
+               ::"l"(reinterpret_cast<uint64_t>(map)), "r"(src), "r"(c0), "r"(c1)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// the stores issued so far have read their shared-memory source
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+// ... and completed
+__device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
 // The epilogue's bf16 rows reach global memory through a per-warp staging
 // tile: each thread writes its row's 128 bytes (16-byte chunk j at position
 // j ^ (row & 7), so the 32 rows' writes spread over the banks), then each
@@ -820,7 +842,8 @@ __device__ __forceinline__ void flush_staging(const uint8_t* stg, int lane,
 template <int MODE>
 __global__ void __launch_bounds__(kThreads2, 1)
     grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap map_a,
-                             const __grid_constant__ CUtensorMap map_b, const KParams p) {
+                             const __grid_constant__ CUtensorMap map_b,
+                             const __grid_constant__ CUtensorMap map_out, const KParams p) {
   using C = Cfg2;
   constexpr int kStages = C::kStages;
   constexpr int BN = C::BN;
@@ -829,7 +852,10 @@ __global__ void __launch_bounds__(kThreads2, 1)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* sa = smem;
   uint8_t* sb = smem + kStages * C::kABytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * C::kStageBytes);
+  // after the ring: the epilogue warps' staging tiles (1024-byte aligned,
+  // the 128-byte swizzle of the output map), the barriers, the tile index
+  uint8_t* staging = smem + kStages * C::kStageBytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(staging + kEpiWarps2 * C::kStagingBytes);
   uint64_t* full = bars;                        // leader's is the one used
   uint64_t* empty = bars + kStages;             // per CTA
   uint64_t* acc_full = bars + 2 * kStages;      // per CTA
@@ -859,6 +885,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
     fence_mbar_init();
     prefetch_map(&map_a);
     prefetch_map(&map_b);
+    if (p.tma_out) prefetch_map(&map_out);
   }
   cluster_sync_all();  // barriers of both CTAs initialised; the peer is running
   if (warp == 1) tmem_alloc_pair(smem_addr(tmem_slot), C::kTmemCols);
@@ -868,11 +895,9 @@ __global__ void __launch_bounds__(kThreads2, 1)
   const uint32_t tmem_base = *tmem_slot;
   grid_dep_wait();
   grid_dep_launch();
-  const TileIndex ix = load_tile_index(
-      p,
-      reinterpret_cast<int32_t*>(smem + kStages * C::kStageBytes + 256 +
-                                 kEpiWarps2 * C::kStagingBytes),
-      C::kIndexInts);
+  const TileIndex ix =
+      load_tile_index(p, reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(bars) + 256),
+                      C::kIndexInts);
   // tiles are 256 rows (both CTAs) x 256 columns; mt_prefix counts 256-row tiles
   const int ntiles = total_tiles(p, ix);
   const int nk = p.K / (BK * C::KS);  // stages per tile
@@ -1029,7 +1054,32 @@ __global__ void __launch_bounds__(kThreads2, 1)
     const int quarter = warp & 3;
     const int half = (warp - 2) >> 2;
     const int wrow0 = static_cast<int>(rank) * BM + quarter * 32;  // warp's first row in the 256
-    uint8_t* stg = smem + kStages * C::kStageBytes + 256 + (warp - 2) * C::kStagingBytes;
+    uint8_t* stg = staging + (warp - 2) * C::kStagingBytes;
+    // Whole 32-row chunks leave by one TMA store of the staging tile (the
+    // store engine writes the lines; per-lane stores of the same lines cost
+    // the down GEMM of the 32 x 1024 layer about 57 us of its 455); a chunk
+    // that ends inside the tile's group keeps the per-lane stores, which
+    // stop at its last row.  The tile is rewritten only after the previous
+    // store has read it.
+    const bool tma_out = p.tma_out != 0;
+    auto staging_free = [&]() {
+      if (tma_out) {
+        if (lane == 0) bulk_wait_read();
+        __syncwarp();
+      }
+    };
+    auto emit = [&](int64_t rbase, int col0, int nrows) {
+      if (tma_out && nrows == 32) {
+        fence_proxy_async_smem();  // this lane's staging writes, before the store reads them
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(&map_out, smem_addr(stg), col0, static_cast<int>(rbase));
+          bulk_commit();
+        }
+      } else {
+        flush_staging(stg, lane, p.out, rbase, p.ldo, col0, nrows);
+      }
+    };
     const uint32_t acc_empty_leader0 = map_to_rank(smem_addr(&acc_empty[0]), 0);
     const uint32_t acc_empty_leader1 = map_to_rank(smem_addr(&acc_empty[1]), 0);
     int lt = 0;
@@ -1063,6 +1113,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
       if (MODE == kModeSwiGLU) {
         // output columns [64 half, +64): gate at c, up at BN/2 + c; both
         // 32-column rounds fill one 128-byte staging row
+        staging_free();
 #pragma unroll
         for (int r = 0; r < 2; ++r) {
           const int c = half * 64 + 32 * r;
@@ -1087,7 +1138,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
                         make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
                                    packed[4 * v + 3]));
         }
-        flush_staging(stg, lane, p.out, row_base, p.ldo, tl.n * (BN / 2) + half * 64, nrows);
+        emit(row_base, tl.n * (BN / 2) + half * 64, nrows);
       } else {
         // columns [128 half, +128) in two rounds of 64 (one staging row each)
 #pragma unroll
@@ -1108,15 +1159,17 @@ __global__ void __launch_bounds__(kThreads2, 1)
             packed[i] = *reinterpret_cast<uint32_t*>(&h0);
             packed[16 + i] = *reinterpret_cast<uint32_t*>(&h1);
           }
+          staging_free();
 #pragma unroll
           for (int v = 0; v < 8; ++v)
             stage_chunk(stg, lane, v,
                         make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
                                    packed[4 * v + 3]));
-          flush_staging(stg, lane, p.out, row_base, p.ldo, tl.n * BN + c, nrows);
+          emit(row_base, tl.n * BN + c, nrows);
         }
       }
     }
+    if (tma_out && lane == 0) bulk_wait_all();  // every store written before exit
   }
 
   tc_fence_before();
@@ -1157,6 +1210,7 @@ cudaError_t launch_pair_impl(const TcGemmArgs& a, cudaStream_t stream) {
   p.defer_wait = 0;
   p.b3d = 0;
   p.norm_out = nullptr;
+  p.tma_out = a.map_out != nullptr ? 1 : 0;
   p.gather_perm = MODE == kModeSwiGLU ? a.gather_perm : nullptr;
   p.gather_kmax = a.gather_kmax;
   p.gather_tokens = a.gather_tokens;
@@ -1181,7 +1235,9 @@ cudaError_t launch_pair_impl(const TcGemmArgs& a, cudaStream_t stream) {
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, kernel, *a.map_a, *a.map_b, p);
+  // without an output map the per-lane stores run and map_a stands in
+  return cudaLaunchKernelEx(&cfg, kernel, *a.map_a, *a.map_b,
+                            a.map_out != nullptr ? *a.map_out : *a.map_a, p);
 }
 
 }  // namespace

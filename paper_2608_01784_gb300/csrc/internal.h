@@ -200,6 +200,10 @@ struct TcGemmArgs {
   const int32_t* gather_perm = nullptr;
   int gather_kmax = 0;
   int gather_tokens = 0;
+  // CTA-pair kernels: 2D map of out [rows, ldo] with a {64, 32} box, 128-byte
+  // swizzle; whole 32-row output chunks are written by TMA stores through it
+  // (nullptr: per-lane stores)
+  const CUtensorMap* map_out = nullptr;
 };
 // SwiGLU: out = silu(A Wg^T) * (A Wu^T).  Down: out = A Wd^T.  bn = tile
 // width (128 or 256, from tc_pick_bn); the B tensor map's box must have

@@ -552,6 +552,14 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
         g1.gather_tokens = T;
       }
       rx::TcGemmArgs g2{&ma2, &mb2, inter, d, d, 0, grouped, xperm, d, err, sms};
+      // output maps of the CTA-pair GEMMs (whole 32-row chunks by TMA store)
+      CUtensorMap mo1, mo2;
+      if (pair_routed) {
+        if (!make_map(&mo1, amid, cap, inter, 32) || !make_map(&mo2, xperm, cap, d, 32))
+          return REFLEX_ECUDA;
+        g1.map_out = &mo1;
+        g2.map_out = &mo2;
+      }
       // the dense shared expert on CTA pairs once it has enough rows: a 256 x
       // 256 pair tile moves a quarter of the operand bytes per output that a
       // 128 x 128 tile of the 1-SM kernel moves from L2 (LLaDA2.0-mini layer
@@ -572,6 +580,13 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
       rx::TcGemmArgs h1{&sa1, &sb1, d, shared_inter, 2 * shared_inter, shared_inter,
                         dense, ash, shared_inter, err, sms, !pair_shared};
       rx::TcGemmArgs h2{&sa2, &sb2, shared_inter, d, d, 0, dense, ysh, d, err, sms};
+      CUtensorMap so1, so2;
+      if (pair_shared) {
+        if (!make_map(&so1, ash, T, shared_inter, 32) || !make_map(&so2, ysh, T, d, 32))
+          return REFLEX_ECUDA;
+        h1.map_out = &so1;
+        h2.map_out = &so2;
+      }
       if (up) {
         if (pair_routed)
           RX_CUDA(rx::launch_swiglu_tc_pair(g1, s));
