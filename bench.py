@@ -55,9 +55,9 @@ METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
 # kernel source it was taken on; once the source differs the line reports
 # null (the counters no longer describe the kernel that ran).
 NCU_TRAFFIC = {
-    "llada_moe": (561004032, "ff14544b3b786cba"),
-    "llada2_mini": (1282214912, "ff14544b3b786cba"),
-    "llada_moe_stack16": (1634241280, "ff14544b3b786cba"),
+    "llada_moe": (561207296, "051461413b65ddc6"),
+    "llada2_mini": (1280278784, "051461413b65ddc6"),
+    "llada_moe_stack16": (1634616064, "051461413b65ddc6"),
 }
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2608_01784_gb300", "csrc", "experts_tc.cu")
 
