@@ -404,6 +404,8 @@ def test_screened_routing_router_rows_16_byte_aligned():
     (16384, 17, 2048, 4),    # odd expert count
     (12289, 64, 1024, 8),    # one token in the last CTA
     (30000, 48, 512, 12),    # ragged last CTA, 48 experts
+    (8192, 1, 256, 1),       # a single expert: every token's one candidate
+    (8200, 8, 512, 8),       # counts up to k = E
 ])
 def test_batch_screened_routing_bit_exact(T, E, d, kmax):
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=5 * T + E + d)
@@ -487,6 +489,8 @@ def test_batch_screened_routing_hard_inputs(kind):
     (1030, 256, 4, 128, 0, 1, "one"),      # CTA-pair tiles, ~257 rows per group: the last
                                            # tile holds a row or two (peer CTA's half empty)
     (4099, 256, 4, 128, 0, 4, "max"),      # CTA-pair tiles, T % 4 != 0, every token at k_max
+    (300, 256, 1, 128, 0, 1, "one"),       # a single expert: one dense group (CTA pairs)
+    (257, 256, 8, 128, 0, 8, "max"),       # every token selects every expert (k = E)
 ])
 @pytest.mark.parametrize("simt", [False, True])
 def test_forward_bf16_small(T, d, E, inter, shared, kmax, kmode, simt):
