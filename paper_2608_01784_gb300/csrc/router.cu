@@ -1226,6 +1226,18 @@ __device__ __forceinline__ void chain8(float& acc, const uint4& a, const uint4& 
   fma_lo(acc, a.w, b.w);
   fma_hi(acc, a.w, b.w);
 }
+// 32-bit screening key for at most 64 experts: the order bits of an
+// interval's lower end with the low 6 bits replaced by 63 - e (so no two
+// experts tie, and the lower index wins among equal truncated values).
+// Truncation is monotone, so the k-th largest key's value part is the
+// truncated k-th largest lower end: the threshold it gives is never above
+// the exact one and the candidates are a superset of the exact candidates.
+// 0 stays free for "removed" (only a negative NaN could map there).
+__device__ __forceinline__ uint32_t screen_key64(float v, int e) {
+  v = (v == 0.0f) ? 0.0f : v;
+  const uint32_t k = (order_bits(v) & ~63u) | static_cast<uint32_t>(63 - e);
+  return k != 0u ? k : 1u;
+}
 __device__ __forceinline__ unsigned long long umax64(unsigned long long a,
                                                      unsigned long long b) {
   return a > b ? a : b;
@@ -1274,7 +1286,8 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
         zv[i][0] = ok && lane < E ? zt[lane] : 0.f;
         zv[i][1] = ok && lane + 32 < E ? zt[lane + 32] : 0.f;
       }
-      unsigned long long key[kBatchGroup][2], best[kBatchGroup];
+      // 32-bit keys: one shuffle per step of the rounds' warp maximum
+      uint32_t key[kBatchGroup][2], best[kBatchGroup];
       float hi[kBatchGroup][2];
       int rounds = 0;
 #pragma unroll
@@ -1290,38 +1303,38 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
         for (int j = 0; j < 2; ++j) {
           const int e = lane + 32 * j;
           hi[i][j] = -INFINITY;
-          key[i][j] = 0ull;
+          key[i][j] = 0u;
           if (e < E) {
             const float v = zv[i][j];
             const float del = g * nh * (j ? nw1 : nw0) * (1.0f + 0x1p-16f) + fabsf(v) * 0x1p-22f;
             hi[i][j] = v + del;
-            key[i][j] = score_key(v - del, e);
+            key[i][j] = screen_key64(v - del, e);
           }
         }
-        best[i] = 0ull;
+        best[i] = 0u;
       }
       for (int r = 0; r < rounds; ++r) {
-        unsigned long long b[kBatchGroup];
+        uint32_t b[kBatchGroup];
 #pragma unroll
-        for (int i = 0; i < kBatchGroup; ++i) b[i] = umax64(key[i][0], key[i][1]);
+        for (int i = 0; i < kBatchGroup; ++i) b[i] = max(key[i][0], key[i][1]);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
           for (int i = 0; i < kBatchGroup; ++i)
-            b[i] = umax64(b[i], __shfl_xor_sync(0xffffffffu, b[i], o));
+            b[i] = max(b[i], __shfl_xor_sync(0xffffffffu, b[i], o));
 #pragma unroll
         for (int i = 0; i < kBatchGroup; ++i) {
           if (r < kt[i]) {
             best[i] = b[i];
-            if (key[i][0] == b[i]) key[i][0] = 0ull;
-            if (key[i][1] == b[i]) key[i][1] = 0ull;
+            if (key[i][0] == b[i]) key[i][0] = 0u;
+            if (key[i][1] == b[i]) key[i][1] = 0u;
           }
         }
       }
 #pragma unroll
       for (int i = 0; i < kBatchGroup; ++i) {
         const int tl = warp * (kBatchT / 8) + g0 + i;
-        const float L = from_order_bits(static_cast<uint32_t>(best[i] >> 32));
+        const float L = from_order_bits(best[i] & ~63u);
         const uint32_t m0 = __ballot_sync(0xffffffffu, tl < nt && hi[i][0] >= L);
         const uint32_t m1 = __ballot_sync(0xffffffffu, tl < nt && hi[i][1] >= L);
         if (lane == 0) {
