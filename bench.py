@@ -33,6 +33,7 @@ from __future__ import annotations
 import argparse
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -55,17 +56,27 @@ METRIC = ("MoE-layer tokens/s and expert TFLOP/s (frac of roofline) REFLEX vs "
 # kernel source it was taken on; once the source differs the line reports
 # null (the counters no longer describe the kernel that ran).
 NCU_TRAFFIC = {
-    "llada_moe": (561207296, "051461413b65ddc6"),
-    "llada2_mini": (1280278784, "051461413b65ddc6"),
-    "llada_moe_stack16": (1634616064, "051461413b65ddc6"),
+    "llada_moe": (561207296, "f1ace3cfdb36717b"),
+    "llada2_mini": (1280278784, "f1ace3cfdb36717b"),
+    "llada_moe_stack16": (1634616064, "f1ace3cfdb36717b"),
 }
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2608_01784_gb300", "csrc", "experts_tc.cu")
 
 
+def code_of(text: str) -> str:
+    """C++ source without comments and with whitespace runs collapsed: what
+    the compiler sees of it (string literals hold no comment markers here)."""
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
 def kernel_source_sha16() -> str:
+    """SHA-256 prefix of the GEMM source's code (comments and layout
+    ignored), the key the DRAM-traffic captures are kept under."""
     import hashlib
-    with open(KERNEL_SOURCE, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    with open(KERNEL_SOURCE, encoding="utf-8") as f:
+        return hashlib.sha256(code_of(f.read()).encode()).hexdigest()[:16]
 
 
 def ncu_traffic(workload: str):

@@ -20,8 +20,9 @@
 // in L2.
 //
 // Kernel.  Persistent: one CTA per SM walks tiles blockIdx.x, +gridDim.x, ...
-//   warp 0     TMA producer: 4-stage ring of (A 128x64, B BNx64) bf16 tiles,
-//              128-byte swizzle, completion on a per-stage mbarrier;
+//   warp 0     TMA producer: 192 KB ring of (A 128x64, B BNx64) bf16 stages
+//              (4 for BN 256, 6 for 128, 8 for 64), 128-byte swizzle,
+//              completion on a per-stage mbarrier;
 //   warp 1     allocates 2*BN TMEM columns (two accumulators) and issues
 //              tcgen05.mma (M=128, N=BN, K=16) from one thread; each stage
 //              is released with tcgen05.commit when its MMAs have read it;
@@ -29,9 +30,11 @@
 //              SwiGLU or conversion, 16-byte stores; the accumulator is
 //              handed back through an mbarrier, so the epilogue of tile i
 //              overlaps the main loop of tile i+1.
-// Every wait is bounded (2 s); on expiry the CTA records the timeout in the
-// error word, drains its outstanding TMA loads and MMAs, frees TMEM and
-// exits.
+// A tile number maps to (expert, n-tile, rows) through the per-expert tile
+// prefix, copied into shared memory once per CTA (TileIndex).  Every wait is
+// bounded (2 s); on expiry the CTA records the timeout in the error word,
+// drains its outstanding TMA loads and MMAs, frees TMEM and exits.  The
+// 2-SM (CTA pair) variant further down has its own description.
 #include "common.cuh"
 #include "internal.h"
 

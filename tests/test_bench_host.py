@@ -57,3 +57,11 @@ def test_rule_ablations_use_the_paper_thresholds(bench):
     for o in got.values():
         assert (o["k_min"], o["k_max"]) == (1, 12)
     assert bench.rule_ablations("tiny_fp32") == []
+
+
+def test_traffic_key_ignores_comments_only(bench):
+    a = "int f(int x) {  // twice\n  return 2 * x; /* no overflow\n here */ }\n"
+    b = "// a header\nint f(int x) {\n    return 2 * x;\n}\n"
+    c = "int f(int x) { return 3 * x; }"
+    assert bench.code_of(a) == bench.code_of(b)
+    assert bench.code_of(a) != bench.code_of(c)
