@@ -99,6 +99,8 @@ inline int64_t screen_z_rows(int T, int E, int d) {
 // the hidden states [T, d] and the router weights [E, d] with 64 x 64 boxes
 // (128-byte swizzle).  Writes ids / alpha and the candidates' exact scores
 // into z.
+// tokens per CTA of the batched screen: the row count of map_h's box
+constexpr int kBatchScreenTokens = 32;
 cudaError_t launch_router_screen_batch(const CUtensorMap* map_h, const CUtensorMap* map_w,
                                        float* z, const float* hss, const float* nw,
                                        const int32_t* k, int T, int E, int d, int k_max,

@@ -443,7 +443,8 @@ static int forward_impl(int32_t dtype, const void* hidden, const void* w_router,
   if ((stages & REFLEX_STAGE_ROUTE) && batch_screen) {
     CUtensorMap mh, mw, mhb, mwb;
     if (!make_map(&mh, hidden, T, d, rx::kTileM) || !make_map(&mw, w_router, E, d, 64) ||
-        !make_map(&mhb, hidden, T, d, 64) || !make_map(&mwb, w_router, E, d, 64))
+        !make_map(&mhb, hidden, T, d, rx::kBatchScreenTokens) ||
+        !make_map(&mwb, w_router, E, d, 64))
       return REFLEX_ECUDA;
     float* nw = reinterpret_cast<float*>(ws + L.wnorm);
     float* hss = reinterpret_cast<float*>(ws + L.tnorm);

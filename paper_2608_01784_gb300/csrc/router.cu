@@ -1151,15 +1151,18 @@ __global__ void __launch_bounds__(kScreenWarps * 32)
 // ---- batched screen recheck (bf16, up to 64 experts) ------------------------
 // The screen of screen_select_kernel for many tokens and few experts, where
 // one warp per token leaves most lanes idle and streams expert rows from L2
-// one lane at a time.  A CTA owns 64 tokens:
-//   1. screening (8 warps, 8 tokens each, four tokens' rounds interleaved):
+// one lane at a time.  A CTA owns 32 tokens, three CTAs per SM (32 x 1024
+// tokens: 1024 CTAs, so the CTAs spread evenly over the SMs; 64-token CTAs,
+// two per SM, left some SMs idle for half of the kernel; 16-token CTAs
+// stream the expert rows too often):
+//   1. screening (8 warps, 4 tokens each, four tokens' rounds interleaved):
 //      from the tensor-core estimates z~ and the row norms (the score GEMM's
 //      sums of squares, ||w_e|| from wnorm_kernel) the interval z~ -/+ del
 //      of every (token, expert), the k_t-th largest lower end L, and the
 //      candidates (upper end >= L) as a per-token bit mask; a prefix over
 //      the tokens lays the (token, expert) candidate pairs out in shared
 //      memory;
-//   2. chains: a producer warp streams 64-k chunks of the CTA's 64 token rows
+//   2. chains: a producer warp streams 64-k chunks of the CTA's 32 token rows
 //      and of the 64 expert rows through a 4-stage TMA ring (128-byte
 //      swizzle); each compute thread advances the canonical fma chain of two
 //      candidate pairs over the chunk, the pairs laid out so that a quarter
@@ -1169,9 +1172,10 @@ __global__ void __launch_bounds__(kScreenWarps * 32)
 //      scores by rank counting, with the keys and tie rule of select_kernel,
 //      the weights with its arithmetic (the same bits), and the exact scores
 //      into z.
-constexpr int kBatchT = 64;                   // tokens per CTA
+constexpr int kBatchT = kBatchScreenTokens;   // tokens per CTA
 constexpr int kBatchE = 64;                   // expert rows per stage (E <= 64)
 constexpr int kBatchStages = 4;
+constexpr int kBatchMinCtas = 3;              // co-resident CTAs per SM (72 registers)
 constexpr int kBatchCompute = 256;            // 8 compute warps
 constexpr int kBatchThreads = kBatchCompute + 32;  // + the producer warp
 constexpr int kBatchSlots = 2 * kBatchCompute;     // candidate pairs per pass
@@ -1187,8 +1191,8 @@ struct BatchSmem {
   int32_t cnt[kBatchT];
   int32_t kt[kBatchT];
   int32_t off[kBatchT + 1];
-  float sel_z[8][kBatchGroup][32];
-  int32_t sel_e[8][kBatchGroup][32];
+  float sel_z[8][32];
+  int32_t sel_e[8][32];
   volatile int abort;
   uint16_t pair[kBatchT * kBatchE];           // (token << 8) | expert
   uint16_t slot[kBatchT * kBatchE];           // chain slot -> pair (0xffff: none)
@@ -1243,7 +1247,7 @@ __device__ __forceinline__ unsigned long long umax64(unsigned long long a,
   return a > b ? a : b;
 }
 
-__global__ void __launch_bounds__(kBatchThreads, 2)
+__global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
     screen_batch_kernel(const __grid_constant__ CUtensorMap map_h,
                         const __grid_constant__ CUtensorMap map_w, float* __restrict__ z,
                         const float* __restrict__ hss, const float* __restrict__ nw, float g,
@@ -1277,9 +1281,11 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
       int kt[kBatchGroup];
 #pragma unroll
       for (int i = 0; i < kBatchGroup; ++i) {  // every load of the group first
+        // a warp's last group of four is partial when kBatchT / 8 is not a
+        // multiple of four
         const int tl = warp * (kBatchT / 8) + g0 + i;
         const int t = t0 + tl;
-        const bool ok = tl < nt;
+        const bool ok = g0 + i < kBatchT / 8 && tl < nt;
         kt[i] = ok ? kin[t] : 1;
         hs[i] = ok ? hss[t] : 0.f;
         const float* zt = z + static_cast<int64_t>(ok ? t : 0) * E;
@@ -1294,7 +1300,7 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
       for (int i = 0; i < kBatchGroup; ++i) {
         if (kt[i] < 1 || kt[i] > kcap) {
           const int tl = warp * (kBatchT / 8) + g0 + i;
-          if (lane == 0 && tl < nt) set_err(err, kErrKRange);
+          if (lane == 0 && g0 + i < kBatchT / 8 && tl < nt) set_err(err, kErrKRange);
           kt[i] = kt[i] < 1 ? 1 : kcap;
         }
         rounds = max(rounds, kt[i]);
@@ -1333,6 +1339,7 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
       }
 #pragma unroll
       for (int i = 0; i < kBatchGroup; ++i) {
+        if (g0 + i >= kBatchT / 8) break;  // the next warp's token
         const int tl = warp * (kBatchT / 8) + g0 + i;
         const float L = from_order_bits(best[i] & ~63u);
         const uint32_t m0 = __ballot_sync(0xffffffffu, tl < nt && hi[i][0] >= L);
@@ -1348,7 +1355,8 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
   }
   __syncthreads();
   if (warp == 0) {  // exclusive prefix of the candidate counts
-    int a = sm.cnt[lane], b = sm.cnt[lane + 32];
+    int a = lane < kBatchT ? sm.cnt[lane] : 0;
+    int b = lane + 32 < kBatchT ? sm.cnt[lane + 32] : 0;
     int ia = a, ib = b;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -1360,9 +1368,9 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
       }
     }
     const int tot_a = __shfl_sync(0xffffffffu, ia, 31);
-    sm.off[lane] = ia - a;
-    sm.off[lane + 32] = tot_a + ib - b;
-    if (lane == 31) sm.off[kBatchT] = tot_a + ib;
+    if (lane < kBatchT) sm.off[lane] = ia - a;
+    if (lane + 32 < kBatchT) sm.off[lane + 32] = tot_a + ib - b;
+    if (lane == 31) sm.off[kBatchT] = tot_a + ib;  // the total
   }
   __syncthreads();
   if (warp < 8) {  // the (token, expert) pairs in token order, experts ascending
@@ -1560,20 +1568,20 @@ __global__ void __launch_bounds__(kBatchThreads, 2)
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
         if (lane + 32 * j < m && rank[j] < kt) {
-          sm.sel_e[warp][0][rank[j]] = ex[j];
-          sm.sel_z[warp][0][rank[j]] = from_order_bits(static_cast<uint32_t>(key[j] >> 32));
+          sm.sel_e[warp][rank[j]] = ex[j];
+          sm.sel_z[warp][rank[j]] = from_order_bits(static_cast<uint32_t>(key[j] >> 32));
         }
       }
       __syncwarp();
-      const float zmax = sm.sel_z[warp][0][0];
-      const float mine = lane < kt ? expf(sm.sel_z[warp][0][lane] - zmax) : 0.f;
+      const float zmax = sm.sel_z[warp][0];
+      const float mine = lane < kt ? expf(sm.sel_z[warp][lane] - zmax) : 0.f;
       float sel = mine;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) sel += __shfl_xor_sync(0xffffffffu, sel, o);
       for (int j = lane; j < k_max; j += 32) {
         const int64_t o = static_cast<int64_t>(t) * k_max + j;
         if (j < kt) {
-          ids[o] = sm.sel_e[warp][0][j];
+          ids[o] = sm.sel_e[warp][j];
           alpha[o] = mine / sel;
         } else {
           ids[o] = -1;
