@@ -84,8 +84,9 @@ def step_launches(dtype: str, T: int, d: int, E: int, shared_inter: int,
     library's choices: the count kernel; the score kernel and the selection,
     or (bf16, renormalised weights, >= 128 experts, T E >= 2048 x 256,
     d % 128 == 0) the norm kernel, the score GEMM and the screened selection,
-    or (bf16, renormalised weights, at most 64 experts, >= 8192 tokens) the
-    norm kernel, the score GEMM and the batched recheck; count + scan in one
+    or (bf16, renormalised weights, at most 64 experts and >= 8192 tokens, or
+    65-256 experts and >= 2048 tokens) the norm kernel, the score GEMM and
+    the batched recheck; count + scan in one
     CTA (short batches whose block masks fit in shared memory) or count and
     scan, then the gather, which also places the pairs; the gate/up and down
     GEMMs (and the shared expert's two); the combine.
@@ -95,7 +96,8 @@ def step_launches(dtype: str, T: int, d: int, E: int, shared_inter: int,
     screened = (dtype == "bf16" and flags & B.REFLEX_FLAG_RENORM_TOPK and
                 not flags & B.REFLEX_FLAG_EXACT_SCORES and not count_rule)
     screen = screened and d % 128 == 0 and E >= 128 and T * E >= 2048 * 256
-    batch_screen = screened and E <= 64 and d % 64 == 0 and T >= 8192
+    batch_screen = screened and d % 64 == 0 and (
+        (E <= 64 and T >= 8192) or (64 < E <= 256 and T >= 2048))
     n += 3 if (screen or batch_screen) else 2
     n += 1 if T <= 4096 and (T + 31) // 32 * E * 4 <= 160 * 1024 else 2
     n += 1 + 2 + (2 if shared_inter else 0) + 1

@@ -93,14 +93,15 @@ inline int64_t screen_z_rows(int T, int E, int d) {
   }
   return rows;
 }
-// Batched screen for E <= 64 (bf16, renormalised weights): z holds the
+// Batched screen for E <= 256 (bf16, renormalised weights): z holds the
 // tensor-core estimates [T, E] (one K slice), hss the tokens' sums of
 // squares, nw the experts' norms (wnorm_kernel); map_h / map_w are 2D maps of
-// the hidden states [T, d] and the router weights [E, d] with 64 x 64 boxes
-// (128-byte swizzle).  Writes ids / alpha and the candidates' exact scores
-// into z.
-// tokens per CTA of the batched screen: the row count of map_h's box
-constexpr int kBatchScreenTokens = 32;
+// the hidden states [T, d] and the router weights [E, d] with boxes of 64
+// columns and screen_batch_token_rows(E) / screen_batch_expert_rows(E) rows (128-byte
+// swizzle).  Writes ids / alpha and the candidates' exact scores into z.
+// the box heights of map_h (tokens per CTA) and map_w for E experts
+int screen_batch_token_rows(int E);
+int screen_batch_expert_rows(int E);
 cudaError_t launch_router_screen_batch(const CUtensorMap* map_h, const CUtensorMap* map_w,
                                        float* z, const float* hss, const float* nw,
                                        const int32_t* k, int T, int E, int d, int k_max,

@@ -1148,22 +1148,23 @@ __global__ void __launch_bounds__(kScreenWarps * 32)
   }
 }
 
-// ---- batched screen recheck (bf16, up to 64 experts) ------------------------
-// The screen of screen_select_kernel for many tokens and few experts, where
-// one warp per token leaves most lanes idle and streams expert rows from L2
-// one lane at a time.  A CTA owns 32 tokens, three CTAs per SM (32 x 1024
-// tokens: 1024 CTAs, so the CTAs spread evenly over the SMs; 64-token CTAs,
-// two per SM, left some SMs idle for half of the kernel; 16-token CTAs
-// stream the expert rows too often):
-//   1. screening (8 warps, 4 tokens each, four tokens' rounds interleaved):
+// ---- batched screen recheck (bf16, up to 256 experts) -----------------------
+// The screen of screen_select_kernel for many tokens, where one warp per
+// token streams each candidate's expert row from L2 one lane at a time.  A
+// CTA owns a block of tokens (BatchCfg: 32 tokens and three CTAs per SM up
+// to 64 experts; at 32 x 1024 tokens 1024 CTAs spread evenly over the SMs,
+// where 64-token CTAs, two per SM, left some SMs idle for half of the
+// kernel and 16-token CTAs stream the expert rows too often):
+//   1. screening (8 warps, the CTA's tokens in turn, up to four tokens'
+//      rounds interleaved):
 //      from the tensor-core estimates z~ and the row norms (the score GEMM's
 //      sums of squares, ||w_e|| from wnorm_kernel) the interval z~ -/+ del
 //      of every (token, expert), the k_t-th largest lower end L, and the
 //      candidates (upper end >= L) as a per-token bit mask; a prefix over
 //      the tokens lays the (token, expert) candidate pairs out in shared
 //      memory;
-//   2. chains: a producer warp streams 64-k chunks of the CTA's 32 token rows
-//      and of the 64 expert rows through a 4-stage TMA ring (128-byte
+//   2. chains: a producer warp streams 64-k chunks of the CTA's token rows
+//      and of the 32 NPL expert rows through a TMA ring (128-byte
 //      swizzle); each compute thread advances the canonical fma chain of two
 //      candidate pairs over the chunk, the pairs laid out so that a quarter
 //      warp's expert rows fall in distinct bank groups (more than 512 pairs:
@@ -1172,34 +1173,51 @@ __global__ void __launch_bounds__(kScreenWarps * 32)
 //      scores by rank counting, with the keys and tie rule of select_kernel,
 //      the weights with its arithmetic (the same bits), and the exact scores
 //      into z.
-constexpr int kBatchT = kBatchScreenTokens;   // tokens per CTA
-constexpr int kBatchE = 64;                   // expert rows per stage (E <= 64)
-constexpr int kBatchStages = 4;
-constexpr int kBatchMinCtas = 3;              // co-resident CTAs per SM (72 registers)
 constexpr int kBatchCompute = 256;            // 8 compute warps
 constexpr int kBatchThreads = kBatchCompute + 32;  // + the producer warp
 constexpr int kBatchSlots = 2 * kBatchCompute;     // candidate pairs per pass
-constexpr int kBatchGroup = 4;                // tokens whose rounds interleave
-constexpr uint32_t kBatchTokBytes = kBatchT * 128;
-constexpr uint32_t kBatchStageBytes = kBatchTokBytes + kBatchE * 128;
 constexpr uint64_t kBatchWaitNs = 2000000000ull;
 constexpr uint64_t kBatchDrainNs = 1000000000ull;
+// NPL groups of 32 experts: every lane of a screening warp holds NPL of a
+// token's experts, and every stage holds the 32 NPL expert rows.  Up to 64
+// experts (NPL 2): 32 tokens per CTA, three CTAs per SM, four tokens'
+// rounds interleaved per warp; up to 256 (NPL 8): 16 tokens per CTA, a
+// 2-stage ring, two CTAs per SM, one token at a time (LLaDA2.0-mini layer
+// 0.553 ms with 32 tokens and one CTA per SM, 0.558 with 16 and one, 0.546
+// with 16 and two).
+template <int NPL>
+struct BatchCfg {
+  static constexpr int kT = NPL <= 2 ? 32 : 16;       // tokens per CTA
+  static constexpr int kE = 32 * NPL;                 // expert rows per stage
+  static constexpr int kStages = NPL <= 2 ? 4 : 2;
+  static constexpr int kMinCtas = NPL <= 2 ? 3 : 2;   // co-resident CTAs per SM
+  static constexpr int kGroup = NPL <= 2 ? 4 : 1;     // tokens whose rounds interleave
+  static constexpr int kIdBits = NPL <= 2 ? 6 : 8;    // expert index bits of a key
+  static constexpr uint32_t kTokBytes = kT * 128;
+  static constexpr uint32_t kStageBytes = kTokBytes + kE * 128;
+  static_assert(kT % 8 == 0 && kT <= 64, "whole swizzle atoms; the prefix's 64 lanes");
+};
+template <int NPL>
 struct BatchSmem {
-  uint64_t full[kBatchStages];
-  uint64_t empty[kBatchStages];
-  uint32_t mask[kBatchT][2];
-  int32_t cnt[kBatchT];
-  int32_t kt[kBatchT];
-  int32_t off[kBatchT + 1];
+  static constexpr int kT = BatchCfg<NPL>::kT;
+  uint64_t full[BatchCfg<NPL>::kStages];
+  uint64_t empty[BatchCfg<NPL>::kStages];
+  uint32_t mask[kT][NPL];
+  int32_t cnt[kT];
+  int32_t kt[kT];
+  int32_t off[kT + 1];
   float sel_z[8][32];
   int32_t sel_e[8][32];
   volatile int abort;
-  uint16_t pair[kBatchT * kBatchE];           // (token << 8) | expert
-  uint16_t slot[kBatchT * kBatchE];           // chain slot -> pair (0xffff: none)
-  float zc[kBatchT * kBatchE];                // exact scores of the pairs
+  uint16_t pair[kT * 32 * NPL];                 // (token << 8) | expert
+  uint16_t slot[kT * 32 * NPL];                 // chain slot -> pair (0xffff: none)
+  float zc[kT * 32 * NPL];                      // exact scores of the pairs
 };
-constexpr size_t kBatchSmemBytes =
-    1024 + kBatchStages * kBatchStageBytes + sizeof(BatchSmem);
+template <int NPL>
+constexpr size_t batch_smem_bytes() {
+  return 1024 + BatchCfg<NPL>::kStages * BatchCfg<NPL>::kStageBytes + sizeof(BatchSmem<NPL>);
+}
+static_assert(batch_smem_bytes<8>() <= 227 * 1024, "one CTA per SM at 256 experts");
 
 // 16 bytes of shared memory.  The "memory" clobber keeps every such read
 // between the stage's mbarrier wait and its release (both asm statements
@@ -1230,24 +1248,23 @@ __device__ __forceinline__ void chain8(float& acc, const uint4& a, const uint4& 
   fma_lo(acc, a.w, b.w);
   fma_hi(acc, a.w, b.w);
 }
-// 32-bit screening key for at most 64 experts: the order bits of an
-// interval's lower end with the low 6 bits replaced by 63 - e (so no two
-// experts tie, and the lower index wins among equal truncated values).
+// 32-bit screening key for at most 2^B experts: the order bits of an
+// interval's lower end with the low B bits replaced by 2^B - 1 - e (so no
+// two experts tie, and the lower index wins among equal truncated values).
 // Truncation is monotone, so the k-th largest key's value part is the
 // truncated k-th largest lower end: the threshold it gives is never above
 // the exact one and the candidates are a superset of the exact candidates.
 // 0 stays free for "removed" (only a negative NaN could map there).
-__device__ __forceinline__ uint32_t screen_key64(float v, int e) {
+template <int B>
+__device__ __forceinline__ uint32_t screen_key(float v, int e) {
+  constexpr uint32_t m = (1u << B) - 1u;
   v = (v == 0.0f) ? 0.0f : v;
-  const uint32_t k = (order_bits(v) & ~63u) | static_cast<uint32_t>(63 - e);
+  const uint32_t k = (order_bits(v) & ~m) | (m - static_cast<uint32_t>(e));
   return k != 0u ? k : 1u;
 }
-__device__ __forceinline__ unsigned long long umax64(unsigned long long a,
-                                                     unsigned long long b) {
-  return a > b ? a : b;
-}
 
-__global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
+template <int NPL>
+__global__ void __launch_bounds__(kBatchThreads, BatchCfg<NPL>::kMinCtas)
     screen_batch_kernel(const __grid_constant__ CUtensorMap map_h,
                         const __grid_constant__ CUtensorMap map_w, float* __restrict__ z,
                         const float* __restrict__ hss, const float* __restrict__ nw, float g,
@@ -1257,7 +1274,15 @@ __global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  BatchSmem& sm = *reinterpret_cast<BatchSmem*>(ring + kBatchStages * kBatchStageBytes);
+  using Cf = BatchCfg<NPL>;
+  constexpr int kBatchT = Cf::kT;
+  constexpr int kBatchStages = Cf::kStages;
+  constexpr uint32_t kBatchTokBytes = Cf::kTokBytes;
+  constexpr int kGroup = Cf::kGroup;
+  constexpr uint32_t kStageBytes = Cf::kStageBytes;
+  constexpr uint32_t kIdMask = (1u << Cf::kIdBits) - 1u;
+  BatchSmem<NPL>& sm =
+      *reinterpret_cast<BatchSmem<NPL>*>(ring + kBatchStages * kStageBytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t0 = blockIdx.x * kBatchT;
   const int nt = min(kBatchT, T - t0);
@@ -1272,32 +1297,34 @@ __global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
   }
   grid_dep_wait();
   grid_dep_launch();
-  // ---- 1. screening: candidate masks, four tokens' rounds interleaved ----
+  // ---- 1. screening: candidate masks, kGroup tokens' rounds interleaved ----
   if (warp < 8) {
-    const float nw0 = lane < E ? nw[lane] : 0.f;
-    const float nw1 = lane + 32 < E ? nw[lane + 32] : 0.f;
-    for (int g0 = 0; g0 < kBatchT / 8; g0 += kBatchGroup) {
-      float zv[kBatchGroup][2], hs[kBatchGroup];
-      int kt[kBatchGroup];
+    float nwj[NPL];  // the norms of this lane's experts lane + 32 j
 #pragma unroll
-      for (int i = 0; i < kBatchGroup; ++i) {  // every load of the group first
-        // a warp's last group of four is partial when kBatchT / 8 is not a
-        // multiple of four
+    for (int j = 0; j < NPL; ++j) nwj[j] = lane + 32 * j < E ? nw[lane + 32 * j] : 0.f;
+    for (int g0 = 0; g0 < kBatchT / 8; g0 += kGroup) {
+      float zv[kGroup][NPL], hs[kGroup];
+      int kt[kGroup];
+#pragma unroll
+      for (int i = 0; i < kGroup; ++i) {  // every load of the group first
+        // a warp's last group is partial when kBatchT / 8 is not a multiple
+        // of kGroup
         const int tl = warp * (kBatchT / 8) + g0 + i;
         const int t = t0 + tl;
         const bool ok = g0 + i < kBatchT / 8 && tl < nt;
         kt[i] = ok ? kin[t] : 1;
         hs[i] = ok ? hss[t] : 0.f;
         const float* zt = z + static_cast<int64_t>(ok ? t : 0) * E;
-        zv[i][0] = ok && lane < E ? zt[lane] : 0.f;
-        zv[i][1] = ok && lane + 32 < E ? zt[lane + 32] : 0.f;
+#pragma unroll
+        for (int j = 0; j < NPL; ++j)
+          zv[i][j] = ok && lane + 32 * j < E ? zt[lane + 32 * j] : 0.f;
       }
       // 32-bit keys: one shuffle per step of the rounds' warp maximum
-      uint32_t key[kBatchGroup][2], best[kBatchGroup];
-      float hi[kBatchGroup][2];
+      uint32_t key[kGroup][NPL], best[kGroup];
+      float hi[kGroup][NPL];
       int rounds = 0;
 #pragma unroll
-      for (int i = 0; i < kBatchGroup; ++i) {
+      for (int i = 0; i < kGroup; ++i) {
         if (kt[i] < 1 || kt[i] > kcap) {
           const int tl = warp * (kBatchT / 8) + g0 + i;
           if (lane == 0 && g0 + i < kBatchT / 8 && tl < nt) set_err(err, kErrKRange);
@@ -1306,48 +1333,56 @@ __global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
         rounds = max(rounds, kt[i]);
         const float nh = sqrtf(hs[i] * (1.0f + 0x1p-10f)) * (1.0f + 0x1p-20f);
 #pragma unroll
-        for (int j = 0; j < 2; ++j) {
+        for (int j = 0; j < NPL; ++j) {
           const int e = lane + 32 * j;
           hi[i][j] = -INFINITY;
           key[i][j] = 0u;
           if (e < E) {
             const float v = zv[i][j];
-            const float del = g * nh * (j ? nw1 : nw0) * (1.0f + 0x1p-16f) + fabsf(v) * 0x1p-22f;
+            const float del = g * nh * nwj[j] * (1.0f + 0x1p-16f) + fabsf(v) * 0x1p-22f;
             hi[i][j] = v + del;
-            key[i][j] = screen_key64(v - del, e);
+            key[i][j] = screen_key<Cf::kIdBits>(v - del, e);
           }
         }
         best[i] = 0u;
       }
       for (int r = 0; r < rounds; ++r) {
-        uint32_t b[kBatchGroup];
+        uint32_t b[kGroup];
 #pragma unroll
-        for (int i = 0; i < kBatchGroup; ++i) b[i] = max(key[i][0], key[i][1]);
+        for (int i = 0; i < kGroup; ++i) {
+          b[i] = key[i][0];
+#pragma unroll
+          for (int j = 1; j < NPL; ++j) b[i] = max(b[i], key[i][j]);
+        }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
-          for (int i = 0; i < kBatchGroup; ++i)
+          for (int i = 0; i < kGroup; ++i)
             b[i] = max(b[i], __shfl_xor_sync(0xffffffffu, b[i], o));
 #pragma unroll
-        for (int i = 0; i < kBatchGroup; ++i) {
+        for (int i = 0; i < kGroup; ++i) {
           if (r < kt[i]) {
             best[i] = b[i];
-            if (key[i][0] == b[i]) key[i][0] = 0u;
-            if (key[i][1] == b[i]) key[i][1] = 0u;
+#pragma unroll
+            for (int j = 0; j < NPL; ++j)
+              if (key[i][j] == b[i]) key[i][j] = 0u;
           }
         }
       }
 #pragma unroll
-      for (int i = 0; i < kBatchGroup; ++i) {
+      for (int i = 0; i < kGroup; ++i) {
         if (g0 + i >= kBatchT / 8) break;  // the next warp's token
         const int tl = warp * (kBatchT / 8) + g0 + i;
-        const float L = from_order_bits(best[i] & ~63u);
-        const uint32_t m0 = __ballot_sync(0xffffffffu, tl < nt && hi[i][0] >= L);
-        const uint32_t m1 = __ballot_sync(0xffffffffu, tl < nt && hi[i][1] >= L);
+        const float L = from_order_bits(best[i] & ~kIdMask);
+        int c = 0;
+#pragma unroll
+        for (int j = 0; j < NPL; ++j) {
+          const uint32_t m = __ballot_sync(0xffffffffu, tl < nt && hi[i][j] >= L);
+          if (lane == 0) sm.mask[tl][j] = m;
+          c += __popc(m);
+        }
         if (lane == 0) {
-          sm.mask[tl][0] = m0;
-          sm.mask[tl][1] = m1;
-          sm.cnt[tl] = __popc(m0) + __popc(m1);
+          sm.cnt[tl] = c;
           sm.kt[tl] = tl < nt ? kt[i] : 0;
         }
       }
@@ -1376,13 +1411,15 @@ __global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
   if (warp < 8) {  // the (token, expert) pairs in token order, experts ascending
     for (int i = 0; i < kBatchT / 8; ++i) {
       const int tl = warp * (kBatchT / 8) + i;
-      const uint32_t m0 = sm.mask[tl][0], m1 = sm.mask[tl][1];
       const uint32_t below = (1u << lane) - 1u;
-      if ((m0 >> lane) & 1u)
-        sm.pair[sm.off[tl] + __popc(m0 & below)] = static_cast<uint16_t>((tl << 8) | lane);
-      if ((m1 >> lane) & 1u)
-        sm.pair[sm.off[tl] + __popc(m0) + __popc(m1 & below)] =
-            static_cast<uint16_t>((tl << 8) | (lane + 32));
+      int pos = sm.off[tl];
+#pragma unroll
+      for (int j = 0; j < NPL; ++j) {
+        const uint32_t m = sm.mask[tl][j];
+        if ((m >> lane) & 1u)
+          sm.pair[pos + __popc(m & below)] = static_cast<uint16_t>((tl << 8) | (lane + 32 * j));
+        pos += __popc(m);
+      }
     }
   }
   __syncthreads();
@@ -1425,8 +1462,8 @@ __global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
             break;
           }
           const uint32_t fb = smem_addr(&sm.full[stage]);
-          uint8_t* st = ring + stage * kBatchStageBytes;
-          mbar_arrive_tx(fb, kBatchStageBytes);
+          uint8_t* st = ring + stage * kStageBytes;
+          mbar_arrive_tx(fb, kStageBytes);
           tma_tile_2d(smem_addr(st), &map_h, c * 64, t0, fb);
           tma_tile_2d(smem_addr(st + kBatchTokBytes), &map_w, c * 64, 0, fb);
           issued |= 1u << stage;
@@ -1470,7 +1507,7 @@ __global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
           ok = false;
           break;
         }
-        const uint32_t sb = ring_s + stage * kBatchStageBytes;
+        const uint32_t sb = ring_s + stage * kStageBytes;
         const uint32_t h0 = sb + ta0, w0 = sb + ea0, h1 = sb + ta1, w1 = sb + ea1;
         if (two) {
           uint4 a0 = lds128(h0), b0 = lds128(w0), a1 = lds128(h1), b1 = lds128(w1);
@@ -1531,7 +1568,7 @@ __global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
   __syncthreads();
   if (sm.abort) return;
   // ---- 3. selection over the candidates' exact scores ----
-  // A warp per token: lane l takes candidates l and l + 32, keys as in
+  // A warp per token: lane l takes candidates l + 32 j, keys as in
   // select_kernel (score, then the lower expert index); a candidate's rank is
   // the number of the token's candidates with a larger key, and the k_t
   // candidates of rank < k_t go to slot rank (the TopK in rank order).
@@ -1541,11 +1578,12 @@ __global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
       if (tl >= nt) continue;
       const int t = t0 + tl;
       const int off = sm.off[tl], m = sm.cnt[tl], kt = sm.kt[tl];
+      const int nj = (m + 31) / 32;  // candidate groups of 32 in use
       float* zt = z + static_cast<int64_t>(t) * E;
-      unsigned long long key[2];
-      int ex[2];
+      unsigned long long key[NPL];
+      int ex[NPL];
 #pragma unroll
-      for (int j = 0; j < 2; ++j) {
+      for (int j = 0; j < NPL; ++j) {
         const int idx = lane + 32 * j;
         key[j] = 0ull;
         ex[j] = 0;
@@ -1558,15 +1596,18 @@ __global__ void __launch_bounds__(kBatchThreads, kBatchMinCtas)
       }
       // every candidate's key in shared memory (the token's zc slots hold
       // the scores; the keys are rebuilt from them), then the ranks
-      int rank[2] = {0, 0};
+      int rank[NPL];
+#pragma unroll
+      for (int j = 0; j < NPL; ++j) rank[j] = 0;
       for (int o = 0; o < m; ++o) {
         const unsigned long long ko =
             score_key(sm.zc[off + o], sm.pair[off + o] & 255);  // broadcast reads
-        rank[0] += ko > key[0];
-        rank[1] += ko > key[1];
+#pragma unroll
+        for (int j = 0; j < NPL; ++j)
+          if (j < nj) rank[j] += ko > key[j];
       }
 #pragma unroll
-      for (int j = 0; j < 2; ++j) {
+      for (int j = 0; j < NPL; ++j) {
         if (lane + 32 * j < m && rank[j] < kt) {
           sm.sel_e[warp][rank[j]] = ex[j];
           sm.sel_z[warp][rank[j]] = from_order_bits(static_cast<uint32_t>(key[j] >> 32));
@@ -1716,18 +1757,27 @@ cudaError_t launch_router_screen_batch(const CUtensorMap* map_h, const CUtensorM
                                        int32_t* ids, float* alpha, uint32_t* err,
                                        cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
-  if (E > kBatchE || d % 64 != 0 || d < 64 || k_max > 32) return cudaErrorInvalidValue;
+  if (E > 256 || d % 64 != 0 || d < 64 || k_max > 32) return cudaErrorInvalidValue;
   const double u = 1.0 / 16777216.0;
   const double gamma = d * u / (1.0 - d * u);
   // chain bound + tensor-core allowance + the score's own rounding (one K slice)
   const float g = static_cast<float>((gamma + 1.0 / 4096.0 + 2 * u) * (1.0 + 1e-3));
-  const cudaError_t e = cudaFuncSetAttribute(
-      screen_batch_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kBatchSmemBytes);
-  if (e != cudaSuccess) return e;
-  const dim3 grid((T + kBatchT - 1) / kBatchT), block(kBatchThreads);
-  return launch_pdl(screen_batch_kernel, grid, block, kBatchSmemBytes, stream, *map_h, *map_w,
-                    z, hss, nw, g, k, T, E, d, k_max, ids, alpha, err);
+  auto go = [&](auto kernel, size_t smem, int rows) -> cudaError_t {
+    const cudaError_t e =
+        cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const dim3 grid((T + rows - 1) / rows), block(kBatchThreads);
+    return launch_pdl(kernel, grid, block, smem, stream, *map_h, *map_w, z, hss, nw, g, k, T,
+                      E, d, k_max, ids, alpha, err);
+  };
+  // map_h's box is screen_batch_token_rows(E) rows high, map_w's
+  // screen_batch_expert_rows(E)
+  if (E <= 64) return go(screen_batch_kernel<2>, batch_smem_bytes<2>(), BatchCfg<2>::kT);
+  return go(screen_batch_kernel<8>, batch_smem_bytes<8>(), BatchCfg<8>::kT);
 }
+
+int screen_batch_token_rows(int E) { return E <= 64 ? BatchCfg<2>::kT : BatchCfg<8>::kT; }
+int screen_batch_expert_rows(int E) { return E <= 64 ? BatchCfg<2>::kE : BatchCfg<8>::kE; }
 
 cudaError_t launch_router_select_rule(const float* z, int T, int E, int k_hi, int k_lo,
                                       int rule, float thr, int k_max, bool renorm,

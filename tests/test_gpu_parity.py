@@ -406,6 +406,9 @@ def test_screened_routing_router_rows_16_byte_aligned():
     (30000, 48, 512, 12),    # ragged last CTA, 48 experts
     (8192, 1, 256, 1),       # a single expert: every token's one candidate
     (8200, 8, 512, 8),       # counts up to k = E
+    (8192, 256, 2048, 12),   # 256 experts: eight 32-expert groups per lane
+    (9000, 200, 1024, 8),    # 200 experts (a partial group), ragged last CTA
+    (8192, 96, 512, 32),     # 96 experts, counts up to 32
 ])
 def test_batch_screened_routing_bit_exact(T, E, d, kmax):
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=5 * T + E + d)
