@@ -229,13 +229,16 @@ def _screen_bound(layer, d, k_splits_max=16):
 
 # screened routing (tensor-core scores, exact recomputation of the experts
 # that could be selected): ids, alpha and the selected scores bit for bit
-# (the screen runs from 128 experts and 2048 x 256 scores on)
+# (the screen runs from 128 experts and 2048 x 256 scores on; up to 256
+# experts the batched recheck, above it the per-token recheck)
 @pytest.mark.parametrize("T,E,d,kmax", [
-    (4096, 128, 2048, 12),   # 128-wide score tiles, one slice
+    (4096, 128, 2048, 12),   # 128-wide score tiles
     (2100, 256, 1024, 12),   # ragged token tiles, two score tiles per row
     (4096, 256, 2048, 8),    # LLaDA2.0-mini expert count
     (3300, 160, 512, 6),     # ragged expert tile
     (2048, 256, 256, 4),     # short rows
+    (2048, 512, 1024, 12),   # per-token recheck, split-K score slices
+    (1024, 1024, 512, 8),    # per-token recheck, 1024 experts
 ])
 def test_screened_routing_bit_exact(T, E, d, kmax):
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=3 * T + E)
@@ -255,12 +258,13 @@ def test_screened_routing_bit_exact(T, E, d, kmax):
     assert np.all(np.abs(rec["scores"].astype(np.float64) - z) <= _screen_bound(layer, d))
 
 
-@pytest.mark.parametrize("T,E", [(4096, 128), (1000, 64)])
+@pytest.mark.parametrize("T,E", [(4096, 128), (1000, 64), (1024, 512)])
 def test_screened_routing_ties_and_many_candidates(T, E):
     # exact ties (duplicated router rows: the lower index wins), near ties
     # (rows one bf16 step apart) and 40 identical rows, more candidates than
-    # one warp recomputes (every expert of such a token is recomputed); at
-    # 1000 x 64 the dense score kernels and the plain selection
+    # one warp recomputes (every expert of such a token is recomputed); 4096
+    # x 128 runs the batched recheck, 1024 x 512 the per-token recheck, 1000
+    # x 64 the dense score kernels and the plain selection
     d, kmax = 1024, 8
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=99)
     w = layer["w_router"].copy()
@@ -332,6 +336,8 @@ def _wide_exponent_case(T, d, E, seed):
     ("wide", 2048, 256, 2048),       # 2 K slices
     ("wide", 4096, 256, 4096),       # 1 slice, d = 4096
     ("gauss", 2048, 256, 4096),      # 2 K slices, d = 4096
+    ("cancel", 1024, 512, 2048),     # the per-token recheck (more than 256 experts)
+    ("wide", 1024, 512, 4096),       # the per-token recheck, d = 4096
 ])
 def test_screened_routing_adversarial_inputs(kind, T, E, d):
     kmax = 8
@@ -371,10 +377,12 @@ def test_screened_routing_adversarial_inputs(kind, T, E, d):
     assert worst <= 2.0 ** -12
 
 
-def test_screened_routing_router_rows_16_byte_aligned():
+@pytest.mark.parametrize("T,E", [(4096, 256), (1024, 512)])
+def test_screened_routing_router_rows_16_byte_aligned(T, E):
     # a router matrix that starts 16 bytes past a 32-byte boundary: the
-    # recheck reads expert rows with 16-byte loads instead of 32-byte ones
-    T, E, d, kmax = 4096, 256, 2048, 8
+    # per-token recheck (E = 512) reads expert rows with 16-byte loads
+    # instead of 32-byte ones; the batched one (E = 256) stages them by TMA
+    d, kmax = 2048, 8
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=51)
     gl = G.GpuLayer(cfg, layer)
     flat = torch.empty(E * d + 8, dtype=torch.bfloat16, device="cuda")
