@@ -495,6 +495,10 @@ def run_gpu(args, cfg, rank, world, local_rank):
                            "and read-back from pinned host memory on a copy stream, "
                            "double-buffered so they overlap the neighbouring steps"),
         expert_tflops=flops_step * world / (ms_step * 1e-3) / 1e12,
+        # Eq. 10 counts the routed experts only; the shared expert's dense
+        # SwiGLU (6 d s T) is added here
+        expert_tflops_with_shared=(layer_flops * world / (ms_step * 1e-3) / 1e12
+                                   if S else None),
         layer_roofline_frac=t_roof / (ms_step * 1e-3),
         avg_k=pairs / T, pairs=pairs,
         fixed_topk=dict(k=cfg.k_base, pairs=pairs_fixed, ms_per_step=ms_fixed,
@@ -927,6 +931,7 @@ def run_sweep(args, rank, world, local_rank):
             line = dict(sweep="llada2_mini", tokens=T, skew=skew, avg_k=pairs / T,
                         pairs=pairs, ms=ms, tokens_per_s=T / (ms * 1e-3),
                         expert_tflops=6.0 * d * I * pairs / (ms * 1e-3) / 1e12,
+                        expert_tflops_with_shared=flops / (ms * 1e-3) / 1e12,
                         roofline_frac=t_roof / (ms * 1e-3),
                         bound="hbm" if bytes_ / (peaks["hbm"] * 1e9) >= flops / (peaks["bf16"] * 1e12) else "tensor",
                         load_imbalance=float(counts.max() / max(counts.mean(), 1e-9)),
