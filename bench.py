@@ -19,12 +19,13 @@ forward from pinned host buffers through the public API with the copies
 inside the timed region; `cpu_baseline` times the oracle on the host cores.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reflex|reference]
-                  [--config NAME] [--no-cpu-baseline] [--sweep] [--ablation]
-                  [--trajectory]
+                  [--config NAME] [--no-cpu-baseline] [--sweep [--sweep-tokens
+                  T1,T2..] [--sweep-skews S1,S2..]] [--ablation] [--trajectory]
 --config llada_moe | llada2_mini | llada_moe_b32 | tiny_fp32: one layer, one
 reflex_step call (counts + layer) per step.
 --sweep: LLaDA2.0-mini layer shapes, 256 .. 65536 tokens x count skew
-0 .. 1 (0 = uniform K_base, 1 = 70% K_min / 30% K_max), forward only.
+0 .. 1 (0 = uniform K_base, 1 = 70% K_min / 30% K_max), forward only; the
+token counts and skews can be listed instead.
 Under torchrun each rank runs its own batch on its own GPU (weak scaling, no
 data-path collective; a barrier and a max-reduce of the times only).
 """
@@ -97,6 +98,12 @@ def parse():
     ap.add_argument("--sweep", action="store_true",
                     help="token-count x count-skew sweep on the LLaDA2.0-mini "
                          "layer (one JSON line per point)")
+    ap.add_argument("--sweep-tokens", default=None,
+                    help="comma-separated token counts of --sweep (default 256 .. "
+                         "65536, doubling)")
+    ap.add_argument("--sweep-skews", default=None,
+                    help="comma-separated count skews of --sweep (default 0, 0.25, "
+                         "0.5, 0.75, 1)")
     ap.add_argument("--trajectory", action="store_true",
                     help="whole denoising trajectories: NFE and pairs per sample")
     ap.add_argument("--ablation", action="store_true",
@@ -889,7 +896,15 @@ def run_sweep(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     cfg = W.CONFIGS["llada2_mini"]
-    Tmax = 65536
+    if args.sweep_tokens:
+        tokens = [int(x) for x in args.sweep_tokens.split(",")]
+    else:
+        tokens = [256 << i for i in range(9)]          # 256 .. 65536
+    skews = ([float(x) for x in args.sweep_skews.split(",")] if args.sweep_skews
+             else [0.0, 0.25, 0.5, 0.75, 1.0])
+    if min(tokens) < 1 or not skews:
+        raise SystemExit("--sweep-tokens and --sweep-skews need positive values")
+    Tmax = max(tokens)
     d, E, I, S, km = cfg.d, cfg.E, cfg.inter, cfg.shared_inter, cfg.k_max
     layer = W.make_layer(cfg, args.seed, T=Tmax)
     dl = api.layer_to_device(layer, cfg.dtype, dev)
@@ -898,12 +913,11 @@ def run_sweep(args, rank, world, local_rank):
     stream = torch.cuda.current_stream(dev)
     peaks = load_peaks()
     F = B.REFLEX_FLAG_RENORM_TOPK
-    T = 256
-    while T <= Tmax:
+    for T in tokens:
         h = dl["hidden"][:T]
         out = torch.empty((T, d), dtype=moe.tdtype, device=dev)
         base_ms = None
-        for skew in (0.0, 0.25, 0.5, 0.75, 1.0):
+        for skew in skews:
             k = torch.from_numpy(W.skewed_k(T, skew, cfg.k_min, cfg.k_base, km,
                                             seed=args.seed)).to(dev)
             moe.forward(h, k, out, F)
@@ -935,9 +949,8 @@ def run_sweep(args, rank, world, local_rank):
                         roofline_frac=t_roof / (ms * 1e-3),
                         bound="hbm" if bytes_ / (peaks["hbm"] * 1e9) >= flops / (peaks["bf16"] * 1e12) else "tensor",
                         load_imbalance=float(counts.max() / max(counts.mean(), 1e-9)),
-                        vs_uniform_kbase=ms / base_ms)
+                        vs_uniform_kbase=ms / base_ms if base_ms else None)
             print(json.dumps(line), flush=True)
-        T *= 2
 
 
 ABLATIONS = [  # (name, allocation overrides): REFLEX and its App. C ablations
