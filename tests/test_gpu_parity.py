@@ -417,6 +417,8 @@ def test_screened_routing_router_rows_16_byte_aligned(T, E):
     (8192, 256, 2048, 12),   # 256 experts: eight 32-expert groups per lane
     (9000, 200, 1024, 8),    # 200 experts (a partial group), ragged last CTA
     (8192, 96, 512, 32),     # 96 experts, counts up to 32
+    (16384, 256, 1024, 8),   # 256 experts, 1024 blocks
+    (20000, 200, 512, 12),   # 200 experts, ragged last CTA
 ])
 def test_batch_screened_routing_bit_exact(T, E, d, kmax):
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=5 * T + E + d)
@@ -441,14 +443,21 @@ def test_batch_screened_routing_bit_exact(T, E, d, kmax):
     assert np.array_equal(rec["alpha"].view(np.uint32), rec_e["alpha"].view(np.uint32))
 
 
-@pytest.mark.parametrize("kind", ["ties", "all_candidates", "cancel", "wide"])
-def test_batch_screened_routing_hard_inputs(kind):
+@pytest.mark.parametrize("kind,E,T", [
+    ("ties", 64, 8192), ("all_candidates", 64, 8192), ("cancel", 64, 8192),
+    ("wide", 64, 8192),
+    # above 64 experts (16-token blocks): more candidate pairs per block
+    # than one pass of the chain loop, every expert row streamed again
+    ("all_candidates", 256, 8192), ("ties", 256, 8192),
+    ("all_candidates", 200, 16400), ("cancel", 256, 16384),
+])
+def test_batch_screened_routing_hard_inputs(kind, E, T):
     # ties: duplicated rows (the lower index wins), rows one bf16 step apart;
-    # all_candidates: every expert row equal for a third of the experts and
-    # tiny weights elsewhere, so many tokens keep more than 32 candidates and
-    # CTAs hold more pairs than one pass of the chain loop (rows streamed
-    # again); cancel / wide: the adversarial inputs of the 256-expert screen
-    T, E, d, kmax = 8192, 64, 1024, 8
+    # all_candidates: every expert row equal for 30 experts and tiny weights
+    # elsewhere, so every token keeps at least 30 candidates and CTAs hold
+    # more pairs than one pass of the chain loop (rows streamed again);
+    # cancel / wide: the adversarial inputs of the 256-expert screen
+    d, kmax = 1024, 8
     cfg, layer = _bf16_case(T, d, E, 128, 0, kmax, seed=77)
     hb, wb = layer["hidden"], layer["w_router"].copy()
     if kind == "ties":
@@ -479,7 +488,7 @@ def test_batch_screened_routing_hard_inputs(kind):
         wf = _bf16_floats(wb).astype(np.float64)
         ratio = np.abs(rec["scores"].astype(np.float64) - hf @ wf.T)[est] / \
             (np.abs(hf) @ np.abs(wf).T)[est]
-        print(f"TC_ERROR_RATIO batch kind={kind} max={float(ratio.max()):.3e} "
+        print(f"TC_ERROR_RATIO batch kind={kind} E={E} max={float(ratio.max()):.3e} "
               f"estimates={int(est.sum())}")
         assert float(ratio.max()) <= 2.0 ** -12
 
