@@ -400,10 +400,10 @@ def test_screened_routing_router_rows_16_byte_aligned(T, E):
     np.testing.assert_allclose(rec["alpha"][valid], alpha[valid], rtol=G.ALPHA_RTOL, atol=1e-7)
 
 
-# The batched screen for layers with at most 64 experts and many tokens
-# (bf16, renormalised weights, from 8192 tokens): tensor-core scores with
-# the token norms from the same GEMM, one exact chain per candidate pair in
-# a CTA of 64 tokens; ids, weights and selected scores bit for bit
+# The batched screen (bf16, renormalised weights; up to 64 experts from 8192
+# tokens, 65-256 experts from 2048): tensor-core scores with the token norms
+# from the same GEMM, one exact chain per candidate pair in a block of 32
+# tokens (16 above 64 experts); ids, weights and selected scores bit for bit
 @pytest.mark.parametrize("T,E,d,kmax", [
     (8192, 64, 2048, 12),    # whole token tiles
     (9000, 64, 1024, 8),     # ragged last tile
