@@ -1,7 +1,8 @@
 """Host logic of bench.py that needs no GPU: the two arms report the same
 config, the DRAM-traffic figure is dropped once the kernel source it was
-captured on has changed, and the count-rule ablations carry the paper's
-thresholds."""
+captured on has changed, the count-rule ablations carry the paper's
+thresholds, and the reference arm (the oracle on the host cores) prints
+its contract line."""
 import importlib
 import os
 import sys
@@ -65,3 +66,26 @@ def test_traffic_key_ignores_comments_only(bench):
     c = "int f(int x) { return 3 * x; }"
     assert bench.code_of(a) == bench.code_of(b)
     assert bench.code_of(a) != bench.code_of(c)
+
+
+def test_reference_arm_prints_the_contract_line(bench):
+    # the reference arm (the oracle on the host cores) end to end on the tiny
+    # layer: one JSON line with the GPU arm's config, metric and unit
+    import json
+    import subprocess
+    from paper_2608_01784_gb300 import workloads as W
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--config",
+                        "tiny_fp32", "--steps", "2", "--warmup", "1"],
+                       cwd=ROOT, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1, r.stdout
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC
+    assert d["unit"] == "tokens/s" and d["higher_is_better"] is True
+    assert d["steps"] == 2 and d["warmup"] == 1 and d["n_gpus"] == 1 and d["value"] > 0
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"],
+                        "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1
+    assert d["config"] == bench.layer_config(W.CONFIGS["tiny_fp32"], 1)
